@@ -1,0 +1,38 @@
+"""Model shapes and workloads (plain data, no arithmetic of the method).
+
+The shapes are those of the paper's models (Sec. IV-A, "Models": LLaMA3.3-70B;
+the 8B shape is the same family at the size that fits one GPU resident), and
+of a tiny model for exhaustive parity checks.
+"""
+
+MODELS = {
+    # 2 layers, hidden 256, 4 query heads x 64, 2 kv heads, SwiGLU 688, vocab 1024
+    "tiny": dict(n_layers=2, hidden=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=688, vocab=1024,
+                 rms_eps=1e-5, rope_theta=500000.0),
+    "llama3-8b": dict(n_layers=32, hidden=4096, n_heads=32, n_kv_heads=8, head_dim=128, ffn=14336, vocab=128256,
+                      rms_eps=1e-5, rope_theta=500000.0),
+    "llama3-70b": dict(n_layers=80, hidden=8192, n_heads=64, n_kv_heads=8, head_dim=128, ffn=28672, vocab=128256,
+                       rms_eps=1e-5, rope_theta=500000.0),
+}
+
+WEIGHT_SEED = 0x10A1B
+PROMPT_SEED = 1
+CONTEXT_SEED = 2
+
+# Workloads: decode/prefill runs on synthetic uniform token ids.
+WORKLOADS = {
+    "tiny-decode": dict(model="tiny", batch=1, prompt=32, decode=16, budget=None, n_slots=2),
+    "8b-decode": dict(model="llama3-8b", batch=1, prompt=512, decode=128, budget=None, n_slots=2),
+    "70b-offload-decode": dict(model="llama3-70b", batch=1, prompt=1024, decode=64, budget=60_000_000_000,
+                               n_slots=2),
+    "70b-offload-prefill": dict(model="llama3-70b", batch=4, prompt=512, decode=0, budget=60_000_000_000,
+                                n_slots=2),
+    "70b-offload-batched": dict(model="llama3-70b", batch=8, ctx_lo=128, ctx_hi=4096, decode=256,
+                                budget=96_000_000_000, n_slots=2),
+}
+
+
+def layer_params(m: dict) -> int:
+    H, F = m["hidden"], m["ffn"]
+    qd, kvd = m["n_heads"] * m["head_dim"], m["n_kv_heads"] * m["head_dim"]
+    return 2 * H + (qd + 2 * kvd) * H + H * qd + 2 * F * H + H * F
