@@ -1,0 +1,77 @@
+"""Pins for the planner oracle: Eq. 1 / Eq. 2 closed forms, brute force, hand cases."""
+import itertools
+
+import pytest
+
+from oracle import planner as P
+
+
+def test_memory_first_fill_hand_cases():
+    GB = 10 ** 9
+    # 80 layers of 1.7113 GB, 60 GB budget, 4.2 GB fixed, 0.36 GB KV, 2 slots:
+    # (60 - 4.2 - 0.36 - 2*1.7113) / 1.7113 = 30.4 -> 30 resident
+    R, ok = P.memory_first_fill(80, 1_711_308_800, 60 * GB, 4_200_000_000, 360_000_000, 2)
+    assert ok and R == 30
+    R3, _ = P.memory_first_fill(80, 1_711_308_800, 60 * GB, 4_200_000_000, 360_000_000, 3)
+    assert R3 == 29
+    # everything fits: no slot reserved
+    assert P.memory_first_fill(4, 100, 1000, 100, 50, 2) == (4, True)
+    # exactly one layer short of fitting -> slots are needed
+    assert P.memory_first_fill(4, 100, 549, 100, 50, 2) == (1, True)
+    # cannot hold the slots
+    assert P.memory_first_fill(4, 100, 349, 100, 50, 2) == (0, False)
+
+
+def test_evenly_spaced_counts_and_gaps():
+    for L in (8, 10, 32, 80):
+        for m in range(L + 1):
+            mask = P.evenly_spaced(L, m)
+            assert sum(mask) == m
+            if 0 < m < L:
+                idx = [i for i, o in enumerate(mask) if o]
+                gaps = [(idx[(j + 1) % m] - idx[j]) % L or L for j in range(m)]
+                assert max(gaps) - min(gaps) <= 1
+
+
+def test_single_slot_simulation_equals_eq1_when_gaps_uniform():
+    # K = 1: each load overlaps only the resident layers before its layer (Eq. 2 window).
+    L, m = 12, 4                       # gaps of 3 layers (2 resident + 1 offloaded)
+    mask = P.evenly_spaced(L, m)
+    for t, c in ((1.0, 0.5), (1.0, 2.0), (1.0, 5.0), (0.3, 0.31)):
+        comp, load = [t] * L, [c] * L
+        assert P.simulate(comp, load, mask, 1) == pytest.approx(P.eq1_single_device(comp, load, mask), rel=1e-12)
+
+
+def test_double_slot_closed_forms():
+    L, m = 10, 5
+    mask = P.evenly_spaced(L, m)
+    # link bound: the copy stream never idles -> T = m * c
+    assert P.simulate([1.0] * L, [7.0] * L, mask, 2) == pytest.approx(m * 7.0)
+    # compute bound: T = sum of compute
+    assert P.simulate([1.0] * L, [0.5] * L, mask, 2) == pytest.approx(L * 1.0)
+    # nothing offloaded
+    assert P.simulate([1.0] * L, [9.0] * L, [False] * L, 2) == pytest.approx(L)
+    # never below max(compute, copy)
+    for K in (1, 2, 3):
+        for c in (0.2, 1.0, 1.7, 4.0):
+            assert P.simulate([1.0] * L, [c] * L, mask, K) >= P.step_lower_bound([1.0] * L, [c] * L, mask) - 1e-12
+
+
+def test_evenly_spaced_is_optimal_single_slot_brute_force():
+    L = 10
+    for m in (2, 3, 4, 6):
+        for c in (1.5, 2.5, 4.0):
+            comp, load = [1.0] * L, [c] * L
+            best = min(P.simulate(comp, load, [i in s for i in range(L)], 1)
+                       for s in itertools.combinations(range(L), m))
+            assert P.simulate(comp, load, P.evenly_spaced(L, m), 1) == pytest.approx(best)
+
+
+def test_plan_and_threshold():
+    plan = P.plan(80, 1_711_308_800, 60 * 10 ** 9, 4_200_000_000, 360_000_000, 2, 6.7e12, 2.1e11)
+    assert plan["R"] == 30 and sum(plan["offloaded"]) == 50
+    assert plan["pred_step_s"] == pytest.approx(50 * 1_711_308_800 / 2.1e11, rel=1e-9)
+    assert P.plan(4, 100, 349, 100, 50, 2, 1.0, 1.0) is None
+    # Eq. 6 reading: tokens until the KV cache exhausts what is left
+    assert P.kv_threshold_tokens(1000, 100, 100, 6, 2, 10) == 10
+    assert P.kv_threshold_tokens(1000, 100, 100, 8, 2, 10) == 0
