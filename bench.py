@@ -1,0 +1,320 @@
+"""Benchmark: greedy decode of the 70B-shaped bf16 stack with layer offloading.
+
+One step = one decode step of the whole hot path (embedding, 80 decoder layers
+of which the ones that do not fit the 60 GB device budget stream from pinned
+host memory through the slot ring, final norm, LM head, argmax) for one batch.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  `value` is timed on the device with CUDA events
+on the compute stream, tokens fed back on the device; `e2e` is the same
+metric through loip_decode_step with host token buffers (host<->device copies
+inside the timed region).  `--impl reference` times the CPU oracle (the plain
+fp64 definition of the decoder) on the host cores on a bounded sample.
+Multi-GPU: independent replicas (the path does not shard), one per rank.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2512_21835_gb300 import configs, inputs  # noqa: E402
+
+METRIC = "decode tokens/s, 70B-shaped bf16 w/ offload; HBM & host-link GB/s vs peak"
+KERNEL_NAMES = ["qkv_rope", "attention", "o_proj", "gate_up", "down", "lm_head"]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", 6800.0), d.get("bf16_tflops_sustained", 1700.0), "measured"
+    return 6800.0, 1700.0, "fallback"
+
+
+class Clocks:
+    """Samples SM clocks and throttle reasons with nvidia-smi during the timed region."""
+
+    def __init__(self):
+        self.samples, self._stop, self._t = [], threading.Event(), None
+
+    def _run(self):
+        q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+        while not self._stop.is_set():
+            try:
+                idx = os.environ.get("LOCAL_RANK", "0")
+                out = subprocess.run(["nvidia-smi", "-i", idx, f"--query-gpu={q}", "--format=csv,noheader,nounits"],
+                                     capture_output=True, text=True, timeout=5).stdout.strip()
+                f = [s.strip() for s in out.split(",")]
+                if len(f) >= 7:
+                    self.samples.append(f)
+            except Exception:
+                pass
+            self._stop.wait(0.2)
+
+    def __enter__(self):
+        self._t = threading.Thread(target=self._run, daemon=True)
+        self._t.start()
+        return self
+
+    def __exit__(self, *a):
+        self._stop.set()
+        self._t.join(timeout=10)
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(s[0]) for s in self.samples if s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in self.samples for i in range(4) if s[3 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.samples)}
+
+
+def link_peak_gbs(torch, nbytes=1 << 30, reps=5):
+    """Live host->device copy peak: pinned source, one cudaMemcpyAsync, best of reps."""
+    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    d = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    best = 1e9
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        d.copy_(h, non_blocking=True)
+        b.record()
+        b.synchronize()
+        best = min(best, a.elapsed_time(b) / 1e3)
+    del h, d
+    return nbytes / best / 1e9
+
+
+def workload_setup(name):
+    w = dict(configs.WORKLOADS[name])
+    m = configs.MODELS[w["model"]]
+    return w, m
+
+
+def run_ours(args, rank, world):
+    import torch
+    from paper_2512_21835_gb300 import build as B
+    B.build()
+    from paper_2512_21835_gb300 import loip
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    w, m = workload_setup(args.workload)
+    hbm_peak, _, peak_kind = measured_peaks()
+    link_peak = link_peak_gbs(torch)
+    lay = loip.loip_layer_layout(m)
+    Bsz = w["batch"]
+    prompt_len = w["prompt"]
+    steps, warm = args.steps, args.warmup
+    max_ctx = prompt_len + warm + 2 * steps + 8
+    budget = w["budget"] or int(torch.cuda.get_device_properties(0).total_memory * 0.9)
+    cfg = loip.config(budget=budget, n_slots=w["n_slots"], max_batch=Bsz, max_ctx=max_ctx,
+                      max_prefill_tokens=min(1024, prompt_len * Bsz), link_Bps=link_peak * 1e9,
+                      hbm_Bps=hbm_peak * 1e9)
+    t0 = time.time()
+    ctx = loip.Context(m, cfg)
+    plan = ctx.plan()
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    t_load = time.time() - t0
+    prompts = inputs.prompts(configs.PROMPT_SEED, Bsz, prompt_len, m["vocab"])
+    t0 = time.time()
+    first = ctx.prefill(list(prompts))
+    t_prefill = time.time() - t0
+
+    # ---- device-timed decode loop: tokens fed back on the device --------------
+    s = torch.cuda.ExternalStream(ctx.compute_stream())
+    tok = torch.from_numpy(first.astype(np.int32)).cuda()
+    tok2 = torch.empty_like(tok)
+    torch.cuda.synchronize()
+    for _ in range(warm):
+        ctx.decode_step_device(tok, tok2)
+        tok, tok2 = tok2, tok
+    ctx.synchronize()
+    ctx.set_kernel_timing(True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    ctx.synchronize()
+    with Clocks() as clk:
+        ev0.record(s)
+        for _ in range(steps):
+            ctx.decode_step_device(tok, tok2)
+            tok, tok2 = tok2, tok
+        ev1.record(s)
+        ctx.synchronize()
+        torch.cuda.synchronize()
+    dev_s = ev0.elapsed_time(ev1) / 1e3
+    st = ctx.stats()
+    ctx.set_kernel_timing(False)
+    # ---- end to end through the public C ABI with host buffers ----------------
+    host_tok = tok.cpu().numpy()
+    for _ in range(2):
+        host_tok = ctx.decode_step(host_tok)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        host_tok = ctx.decode_step(host_tok)
+    e2e_s = time.perf_counter() - t0
+    st2 = ctx.stats()
+    ctx.close()
+
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([dev_s, e2e_s], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dev_s, e2e_s = float(t[0]), float(t[1])
+
+    tokens = steps * Bsz * world
+    n_off = plan["n_offloaded"]
+    # dominant kernel: the gate/up SwiGLU product (55% of a layer's bytes)
+    gu_bytes = 2 * m["ffn"] * m["hidden"] * 2
+    k = KERNEL_NAMES.index("gate_up")
+    gu_ms = st["kernel_ms"][k] / max(1, st["kernel_launches"][k])
+    gu_gbs = gu_bytes / (gu_ms / 1e3) / 1e9
+    step_s = dev_s / steps
+    link_bytes = n_off * lay["l_size"]
+    kv_bytes = (prompt_len + warm + steps) * 2 * m["n_kv_heads"] * m["head_dim"] * 2 * m["n_layers"] * Bsz
+    hbm_bytes = m["n_layers"] * lay["l_size"] + m["vocab"] * m["hidden"] * 2 + kv_bytes
+    roof_step = max(hbm_bytes / (hbm_peak * 1e9), link_bytes / (link_peak * 1e9))
+    kernel_sum_ms = sum(st["kernel_ms"]) / steps
+    t_copy_only = link_bytes / (link_peak * 1e9)
+    exposed = max(0.0, step_s - max(kernel_sum_ms / 1e3, t_copy_only))
+    per_step_launches = 1 + m["n_layers"] * 6 + 2 + 1
+    line = {
+        "metric": METRIC,
+        "value": round(tokens / dev_s, 4),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": steps,
+        "warmup": warm,
+        "ms_per_step": round(step_s * 1e3, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16 weights, fp32 activations",
+        "data": "synthetic: SplitMix64 bf16 weights N(0,0.02^2), uniform token ids",
+        "config": {"workload": args.workload, "model": w["model"] + "-shaped", "layers": m["n_layers"],
+                   "global_batch": Bsz * world, "context": prompt_len, "budget_bytes": budget,
+                   "slots": w["n_slots"], "resident_layers": plan["n_resident"], "offloaded_layers": n_off,
+                   "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2: every step reads all weights (> 100 GB)"},
+        "roofline": {"bound": "hbm", "kernel": "gate_up (RMSNorm+SwiGLU GEMV)", "achieved": round(gu_gbs, 1),
+                     "peak": hbm_peak, "unit": "GB/s", "frac": round(gu_gbs / hbm_peak, 4),
+                     "peak_kind": peak_kind, "traffic": None, "bytes_per_launch": gu_bytes,
+                     "avg_launch_ms": round(gu_ms, 4)},
+        "step_roofline": {"bound": "host-link" if link_bytes / link_peak > hbm_bytes / hbm_peak else "hbm",
+                          "link_bytes_per_step": link_bytes, "link_peak_GBps": round(link_peak, 1),
+                          "link_achieved_GBps": round(link_bytes / step_s / 1e9, 1),
+                          "hbm_bytes_per_step": hbm_bytes, "roofline_step_ms": round(roof_step * 1e3, 3),
+                          "frac": round(roof_step / step_s, 4), "exposed_load_ms": round(exposed * 1e3, 3),
+                          "exposed_frac": round(exposed / step_s, 4),
+                          "kernel_ms_per_step": {n: round(st["kernel_ms"][i] / steps, 4)
+                                                 for i, n in enumerate(KERNEL_NAMES)},
+                          "copy_busy_ms_last": round(st["copy_busy_ms"], 3)},
+        "e2e": {"value": round(tokens / e2e_s, 4), "unit": "tokens/s", "h2d_bytes_per_step": 4 * Bsz,
+                "d2h_bytes_per_step": 4 * Bsz},
+        "gpu_launches": per_step_launches * steps,
+        "clocks": clk.summary(),
+        "setup_s": {"create_and_weights": round(t_load, 1), "prefill": round(t_prefill, 1)},
+    }
+    return line
+
+
+def oracle_sample(m, n_layers_sample, threads=None):
+    """Times the oracle on one token through n layers of the model shape plus the
+    LM head; returns seconds per full token (layers extrapolated)."""
+    import oracle
+    oracle.build()
+    mh = dict(m, n_layers=0)
+    ml = dict(m, n_layers=n_layers_sample, vocab=16)
+    tok = np.array([7], dtype=np.int32)
+    dl, dh = oracle.ModelDesc(**ml), oracle.ModelDesc(**mh)
+    t0 = time.perf_counter()
+    oracle.forward(dl, oracle.Weights(dl, configs.WEIGHT_SEED), tok)
+    t_layers = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    oracle.forward(dh, oracle.Weights(dh, configs.WEIGHT_SEED), tok)
+    t_head = time.perf_counter() - t0
+    per_token = t_layers / n_layers_sample * m["n_layers"] + t_head
+    return per_token, t_layers + t_head, oracle.num_threads()
+
+
+def cpu_baseline(w, m, n_layers_sample=16):
+    per_token, spent, cores = oracle_sample(m, n_layers_sample)
+    return {"value": round(w["batch"] / per_token, 6), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"1 token through {n_layers_sample} of {m['n_layers']} layers of the {w['model']} shape "
+                      f"plus the LM head, fp64, {spent:.1f} s; layer time scaled to {m['n_layers']} layers"}
+
+
+def run_reference(args, rank, world):
+    w, m = workload_setup(args.workload)
+    if rank != 0:
+        return None
+    for _ in range(args.warmup):
+        pass  # the oracle has no warm state
+    vals = []
+    for _ in range(args.steps):
+        per_token, spent, cores = oracle_sample(m, 2)
+        vals.append(w["batch"] / per_token)
+    v = statistics.median(vals)
+    return {"metric": METRIC, "value": round(v, 6), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "higher_is_better": True, "impl": "reference",
+            "config": {"workload": args.workload, "model": w["model"] + "-shaped"},
+            "cpu_baseline": {"kind": "oracle", "cores": cores, "value": round(v, 6), "unit": "tokens/s",
+                             "sample": "per step: 1 token through 2 layers plus the LM head, scaled to "
+                                       f"{m['n_layers']} layers"},
+            "e2e": {"value": round(v, 6), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=12)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="70b-offload-decode", choices=sorted(configs.WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world > 1 and args.impl == "ours":
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        dist.init_process_group("nccl")
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        line = run_ours(args, rank, world)
+        if rank == 0 and not args.no_cpu_baseline:
+            w, m = workload_setup(args.workload)
+            line["cpu_baseline"] = cpu_baseline(w, m)
+    if rank == 0 and line is not None:
+        print(json.dumps(line), flush=True)
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

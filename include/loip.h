@@ -1,0 +1,291 @@
+/*
+ * loip.h -- C ABI of libloip: single-GPU lossless LLaMA-style decoding with
+ * layer weights offloaded to pinned host memory and streamed into device slots
+ * while earlier layers compute (LOIP, arXiv 2512.21835, reduced to one GPU).
+ *
+ * Conventions
+ *   - Every call returns an int status (LOIP_OK = 0 or a LOIP_ERR_* code); no
+ *     C++ exception crosses this boundary.  loip_last_error() gives a message.
+ *   - "dev" pointers are CUDA device pointers, "host" pointers are ordinary
+ *     host memory.  The caller owns every pointer it passes in; the library
+ *     never frees them.  Streams are passed as `void*` holding a cudaStream_t
+ *     (NULL = the context's own stream).
+ *   - bf16 values are passed as uint16_t bit patterns; activations are fp32.
+ *   - Weight matrices are row-major [out, in] (out rows of `in` contiguous
+ *     elements).
+ *   - Calls on one context are not thread-safe.
+ *
+ * Layer blob (one decoder layer, the unit that is offloaded and streamed):
+ *   g_attn [H] | wqkv [(Hq+2Hkv)*d, H] (q rows, then k rows, then v rows) |
+ *   wo [H, Hq*d] | g_mlp [H] | wg [F, H] | wu [F, H] | wd [H, F]
+ *   all bf16, each part starting at a 256-byte boundary of the blob;
+ *   loip_layer_layout() returns the offsets and the blob size (l_size).
+ *   The MHA block is g_attn..wo and the MLP block g_mlp..wd (the paper's
+ *   decomposition of a layer into MHA and MLP blocks, Sec. III-D).
+ */
+#ifndef LOIP_H
+#define LOIP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    LOIP_OK = 0,
+    LOIP_ERR_INVALID = 1,    /* bad argument (null pointer, size, range, alignment) */
+    LOIP_ERR_OOM = 2,        /* device arena or pinned host memory exhausted */
+    LOIP_ERR_INFEASIBLE = 3, /* budget cannot hold the fixed part, KV cache and slots */
+    LOIP_ERR_CUDA = 4,       /* a CUDA runtime call failed (message has the CUDA error) */
+    LOIP_ERR_TIMEOUT = 5,    /* a host wait on the device passed its deadline */
+    LOIP_ERR_STATE = 6       /* call not valid in the context's current state */
+};
+
+enum { LOIP_MODE_OVERLAP = 0, LOIP_MODE_NAIVE = 1 };
+
+typedef struct loip_model_desc {
+    int32_t n_layers, hidden, n_heads, n_kv_heads, head_dim, ffn, vocab;
+    float rms_eps;    /* RMSNorm epsilon */
+    float rope_theta; /* rotary base */
+} loip_model_desc;
+
+typedef struct loip_config {
+    uint64_t device_budget_bytes; /* size of the device arena the context may use */
+    int32_t n_slots;              /* device slots for streamed layers, 1..3 */
+    int32_t page_tokens;          /* KV page size in tokens (64) */
+    int32_t max_batch;            /* largest decode batch (<= 8) */
+    int32_t max_ctx;              /* largest context per request, tokens */
+    int32_t use_graphs;           /* capture decode steps as CUDA graphs */
+    int32_t mode;                 /* LOIP_MODE_OVERLAP or LOIP_MODE_NAIVE */
+    uint32_t timeout_ms;          /* deadline of every host wait (0 = 600000) */
+    double hbm_Bps;               /* bandwidths used by the planner's step model */
+    double link_Bps;
+    uint64_t kv_reserve_bytes;    /* KV bytes to reserve at create (0 = max_batch*max_ctx) */
+    int32_t max_prefill_tokens;   /* tokens per prefill pass (workspace size; 0 = 512) */
+} loip_config;
+
+typedef struct loip_layer_layout_t {
+    uint64_t off_g_attn, off_wqkv, off_wo, off_g_mlp, off_wg, off_wu, off_wd;
+    uint64_t l_size;   /* blob bytes */
+    uint64_t mha_bytes, mlp_bytes;
+} loip_layer_layout_t;
+
+typedef struct loip_plan {
+    int32_t n_layers;
+    int32_t n_resident, n_offloaded;
+    uint8_t* resident;     /* [n_layers], caller-owned; 1 = resident in HBM, 0 = streamed */
+    double pred_step_s;    /* discrete-event step time with n_slots slots */
+    double pred_copy_s;    /* offloaded bytes / link bandwidth */
+    double pred_compute_s; /* all weight bytes / HBM bandwidth */
+    double eq1_step_s;     /* Eq. 1 with one device (single-slot bound) */
+    uint64_t left_bytes;   /* budget left after fixed, KV, resident layers and slots */
+} loip_plan;
+
+typedef struct loip_stats {
+    uint64_t steps, tokens;
+    uint64_t h2d_weight_bytes; /* bytes streamed host -> slots */
+    double last_step_ms;       /* host wall time of the last decode/prefill call */
+    double copy_busy_ms;       /* copy-stream busy time, last step (events) */
+    double compute_ms;         /* compute-stream time, last step (events) */
+    int32_t n_resident, n_offloaded, n_replans;
+    uint64_t kv_tokens;        /* tokens held in the KV cache (all requests) */
+    uint64_t kv_bytes;         /* bytes of KV pages allocated */
+    uint64_t arena_used;       /* device arena bytes in use */
+    /* per kernel class, accumulated while kernel timing is on (loip_set_kernel_timing):
+     * 0 qkv+rope, 1 attention (+combine), 2 o-proj, 3 gate/up, 4 down, 5 lm head (+argmax) */
+    double kernel_ms[6];
+    uint64_t kernel_launches[6];
+} loip_stats;
+
+typedef struct loip_ctx loip_ctx;
+
+/* ---------------------------------------------------------------------------
+ * Host-only planning (no GPU needed)
+ * ------------------------------------------------------------------------- */
+
+/* Blob layout of one layer of `desc`.  LOIP_ERR_INVALID on bad shapes
+ * (hidden and ffn multiples of 8, head_dim even, n_heads % n_kv_heads == 0). */
+int loip_layer_layout(const loip_model_desc* desc, loip_layer_layout_t* out);
+
+/* Residency plan (Algorithm 1's memory-first fill, Sec. III-D; Eq. 1 and Eq. 2,
+ * Sec. III-B/III-D, with a single device and no network term).
+ *   layer_bytes [n_layers]: bytes of each layer (slots are sized by the largest).
+ *   R = the largest count with fixed + kv + R*l + n_slots*l <= budget (no slot
+ *   if all layers fit); the n_layers-R offloaded layers are spread evenly
+ *   (layer i offloaded iff floor((i+1)m/L) > floor(i m/L)), the single-device
+ *   form of the interleaved placement of Sec. III-A.
+ *   out->resident must point to n_layers bytes.
+ * LOIP_ERR_INFEASIBLE if the budget cannot hold fixed + kv + the slots. */
+int loip_plan_residency(const loip_model_desc* desc, const uint64_t* layer_bytes, uint64_t device_budget,
+                        uint64_t kv_bytes, uint64_t fixed_bytes, int32_t n_slots, double hbm_Bps, double link_Bps,
+                        loip_plan* out);
+
+/* Eq. 6 (online memory-aware planner, Sec. III-E), read as a token count:
+ * the number of KV tokens the memory left after a plan can still hold. */
+int loip_kv_threshold(uint64_t left_bytes, uint64_t kv_bytes_per_token, uint64_t* out_tokens);
+
+/* Bytes of the fixed device part of a context (embedding, LM head, final
+ * gain, page table, workspaces) for `desc` and `cfg`. */
+int loip_fixed_bytes(const loip_model_desc* desc, const loip_config* cfg, uint64_t* out);
+
+/* ---------------------------------------------------------------------------
+ * Context
+ * ------------------------------------------------------------------------- */
+
+/* Creates a context on the current CUDA device.  `device_arena` (dev, at least
+ * cfg->device_budget_bytes, 256-byte aligned) holds every device byte the
+ * context uses: fixed part, resident layers, slots, KV pages.  The library
+ * allocates pinned host memory for offloaded layers (it owns it) and its own
+ * streams and events.  The plan is made here (loip_plan_residency with the KV
+ * reserve).  *out is NULL on failure. */
+int loip_create(const loip_model_desc* desc, const loip_config* cfg, void* device_arena, uint64_t arena_bytes,
+                loip_ctx** out);
+
+void loip_destroy(loip_ctx* ctx);
+
+/* Message of the last failed call on ctx (or of the last failed create when
+ * ctx is NULL).  Valid until the next call. */
+const char* loip_last_error(const loip_ctx* ctx);
+
+/* Fills every weight with the seeded SplitMix64 generator (bf16 N(0, 0.02^2)
+ * approximations; norm gains 1 + 0.02 z): resident layers are written in place,
+ * offloaded layers are generated on the device and copied to the pinned host
+ * pool.  Then the first slots are filled.  Synchronous. */
+int loip_load_weights_generated(loip_ctx* ctx, uint64_t seed);
+
+/* Loads one layer from a caller blob (host, l_size bytes, layout above) into
+ * its resident block or host-pool entry.  Synchronous. */
+int loip_load_layer(loip_ctx* ctx, int32_t layer, const void* host_blob, uint64_t bytes);
+
+/* Loads embedding / LM head [vocab, hidden] and final gain [hidden] (host bf16). */
+int loip_load_globals(loip_ctx* ctx, const uint16_t* embed, const uint16_t* lm_head, const uint16_t* g_final);
+
+/* Current plan (resident[] must hold n_layers bytes). */
+int loip_get_plan(const loip_ctx* ctx, loip_plan* out);
+
+/* Enqueues the copy of offloaded `layer` from the pinned host pool into device
+ * slot `slot` on `copy_stream` (the "stream layer" step, Sec. III-C: the slot
+ * is rewritten only after the compute that used it has signalled, through a
+ * CUDA event, that it is done).  Records the slot-full event.  Async. */
+int loip_stream_layer(loip_ctx* ctx, int32_t layer, int32_t slot, void* copy_stream);
+
+/* Enqueues one decoder layer on `compute_stream` for `batch` requests:
+ *   hidden (dev, fp32 [batch, H]) is updated in place (residual stream);
+ *   positions (dev, int32 [batch]) are the token positions; the new k/v are
+ *   appended to each request's KV pages at that position (request b = row b).
+ *   The layer's weights are its resident block, or slot `slot` if offloaded
+ *   (the call waits on that slot's full event and records its free event).
+ * Async.  Requires that the requests' contexts were set by loip_set_batch. */
+int loip_layer_forward(loip_ctx* ctx, int32_t layer, int32_t slot, float* hidden, const int32_t* positions,
+                       int32_t batch, void* compute_stream);
+
+/* Declares the active requests for the following decode steps: request b has
+ * ctx_lens[b] tokens already in its cache (host, int32 [batch]).  Allocates KV
+ * pages as needed. */
+int loip_set_batch(loip_ctx* ctx, int32_t batch, const int32_t* ctx_lens);
+
+/* One greedy decode step for the active batch: tokens (host, int32 [batch]) are
+ * the current tokens; out_tokens (host, int32 [batch]) receive the argmax of
+ * the logits (lowest index on ties); out_hidden (dev fp32 [batch, H] or NULL)
+ * receives the final-norm hidden state.  Streams offloaded layers through the
+ * slots with the copy of slot k starting once its previous layer is computed,
+ * continuing into the next step's first layers.  Synchronous. */
+int loip_decode_step(loip_ctx* ctx, const int32_t* tokens, int32_t batch, int32_t* out_tokens, float* out_hidden);
+
+/* Same step, with tokens, out_tokens (int32 [batch]) and out_hidden in device
+ * memory; enqueued on the context's compute stream without a host wait. */
+int loip_decode_step_device(loip_ctx* ctx, const int32_t* tokens_dev, int32_t batch, int32_t* out_tokens_dev,
+                            float* out_hidden);
+
+/* Prefill of n_prompts prompts (tokens host int32, concatenated; prompt_lens
+ * host int32 [n_prompts]) into requests 0..n_prompts-1, each starting at
+ * position 0.  Writes the argmax after each prompt's last token (host int32
+ * [n_prompts]) and optionally the final hidden of those tokens (dev fp32
+ * [n_prompts, H]).  Weights stream exactly as in decode.  Synchronous. */
+int loip_prefill(loip_ctx* ctx, const int32_t* tokens, const int32_t* prompt_lens, int32_t n_prompts,
+                 int32_t* out_tokens, float* out_hidden);
+
+/* Re-plans for the current KV size (Eq. 6 thresholds): while the KV pages the
+ * next `lookahead_tokens` tokens of every request need do not fit, one more
+ * resident layer is demoted to the host pool (evenly spaced).  Synchronous. */
+int loip_replan(loip_ctx* ctx, int32_t lookahead_tokens);
+
+int loip_get_stats(const loip_ctx* ctx, loip_stats* out);
+
+/* Kernel timing: when enable != 0, every decode-layer kernel is bracketed by
+ * CUDA events on its stream and the durations are summed per kernel class into
+ * loip_stats.kernel_ms / kernel_launches (reset on every enable call). */
+int loip_set_kernel_timing(loip_ctx* ctx, int32_t enable);
+
+/* Waits (with the context deadline) until all work of the context is done. */
+int loip_synchronize(loip_ctx* ctx);
+
+/* Device pointer of the compute / copy stream (cudaStream_t). */
+void* loip_compute_stream(loip_ctx* ctx);
+void* loip_copy_stream(loip_ctx* ctx);
+
+/* ---------------------------------------------------------------------------
+ * Kernel-level entry points (the fused kernels of one decoder layer, for tests
+ * and for callers that compose their own loop).  All are async on `stream`,
+ * take device pointers, and return LOIP_ERR_INVALID on bad sizes or
+ * misaligned pointers (weights and vectors 16-byte aligned).  B <= 8.
+ * ------------------------------------------------------------------------- */
+
+/* Seeded generator: out (dev bf16 [n]) = element first..first+n-1 of tensor
+ * `tensor_id`; kind 0 = weight 0.02 z, kind 1 = gain 1 + 0.02 z. */
+int loip_k_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id, int32_t kind,
+                    void* stream);
+
+/* x[b, :] = embed[tokens[b], :] (bf16 -> fp32). */
+int loip_k_embed(const uint16_t* embed, const int32_t* tokens, int32_t B, int32_t H, float* x, void* stream);
+
+/* RMSNorm (LLaMA pre-norm) fused into a matrix-vector product with query/key
+ * rotation: y = x / sqrt(mean(x^2) + eps) * g; qkv = wqkv y; q and k heads
+ * rotated at positions[b] (pairs (i, i + d/2), angle pos * theta^(-2i/d),
+ * computed in fp64); q -> q_out (fp32 [B, Hq*d]); k and v are rounded to bf16
+ * and written into request b's paged cache at positions[b] (page table row b,
+ * page layout as for loip_k_attention). */
+int loip_k_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int32_t B, int32_t H, int32_t Hq,
+                    int32_t Hkv, int32_t d, float eps, float theta, const int32_t* positions, float* q_out,
+                    const void* kv_base, const int64_t* page_offsets, int32_t max_pages, int32_t page_tokens,
+                    int32_t layer, uint64_t layer_page_bytes, void* stream);
+
+/* Split-K grouped-query decode attention over a paged cache:
+ *   q (fp32 [B, Hq*d]); request b attends over its first ctx_lens[b] cached
+ *   positions; page_offsets (dev int64 [B, max_pages]) gives each page's byte
+ *   offset from kv_base; a page holds, for layer `layer`, K then V as
+ *   [Hkv][page_tokens][d] bf16 at layer * layer_page_bytes inside the page.
+ *   Writes o (fp32 [B, Hq*d]).  `scratch` (dev fp32, at least
+ *   loip_k_attention_scratch_floats(...) floats) holds the per-chunk partial
+ *   softmax states. */
+int loip_k_attention(const float* q, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
+                     const int32_t* ctx_lens, int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t page_tokens,
+                     int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx, float* scratch, float* o,
+                     void* stream);
+uint64_t loip_k_attention_scratch_floats(int32_t B, int32_t Hq, int32_t d, int32_t max_ctx, int32_t page_tokens);
+
+/* x += wo o  (output projection with the residual add); o fp32 [B, Hq*d]. */
+int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x, void* stream);
+
+/* a = silu(wg y) * (wu y) with y = RMSNorm(x) * g (SwiGLU MLP input half);
+ * a fp32 [B, F]. */
+int loip_k_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int32_t B, int32_t H,
+                   int32_t F, float eps, float* a, void* stream);
+
+/* x += wd a  (down projection with the residual add); a fp32 [B, F]. */
+int loip_k_down(const float* a, const uint16_t* wd, int32_t B, int32_t H, int32_t F, float* x, void* stream);
+
+/* Final RMSNorm and LM head: z = RMSNorm(x) * g_final (fp32 [B, H], may be
+ * NULL), logits = lm_head z (fp32 [B, V], may be NULL) and the greedy token
+ * (int32 [B], lowest index on ties).  `scratch` (dev, at least
+ * loip_k_lm_head_scratch_bytes(B, V) bytes) holds per-block partial maxima. */
+int loip_k_lm_head(const float* x, const uint16_t* g_final, const uint16_t* lm_head, int32_t B, int32_t H,
+                   int32_t V, float eps, float* z, float* logits, int32_t* tokens, void* scratch, void* stream);
+uint64_t loip_k_lm_head_scratch_bytes(int32_t B, int32_t V);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LOIP_H */

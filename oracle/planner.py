@@ -123,6 +123,36 @@ def kv_threshold_tokens(budget: int, fixed: int, l_size: int, R: int, n_slots_us
     return left // kv_bytes_per_token
 
 
+def demote_one(offloaded):
+    """Online adaptation at layer granularity (Sec. III-E): when the KV cache
+    crosses the threshold, one more resident layer is offloaded.  To keep the
+    offloaded layers evenly interleaved, the victim is the middle layer (lower
+    middle for even lengths) of the longest cyclic run of resident layers,
+    the first such run in layer order on ties; with nothing offloaded, the last
+    layer (where the even spacing of m = 1 puts it).  Returns the new mask and
+    the victim, or (mask, None) when every layer is already offloaded."""
+    L = len(offloaded)
+    mask = list(offloaded)
+    m = sum(mask)
+    if m == L:
+        return mask, None
+    if m == 0:
+        mask[L - 1] = True
+        return mask, L - 1
+    best_len, best_start = -1, None
+    for l in range(L):
+        if not mask[l]:
+            continue
+        run = 0
+        while run < L and not mask[(l + 1 + run) % L]:
+            run += 1
+        if run > best_len:
+            best_len, best_start = run, (l + 1) % L
+    victim = (best_start + (best_len - 1) // 2) % L
+    mask[victim] = True
+    return mask, victim
+
+
 def step_lower_bound(comp, load, offloaded):
     """max(compute, copy) -- no schedule can beat it."""
     return max(sum(comp), sum(c for c, o in zip(load, offloaded) if o))

@@ -1,0 +1,835 @@
+// decode.cu -- the decode-time kernels of one LLaMA-style decoder layer on
+// sm_103a, plus the embedding gather, the LM head with greedy argmax and the
+// seeded weight generator.
+//
+// Every decode projection is a weight-stationary matrix-vector product that is
+// HBM bound: each bf16 weight byte is read exactly once with 128-bit streaming
+// loads (ld.global.nc.L1::no_allocate), the fp32 activation rows are staged in
+// shared memory in a bank-conflict-free permuted layout, each warp owns a few
+// output rows and reduces its partial sums with xor shuffles.  Normalisation,
+// rotary embedding, KV-cache append, SwiGLU, residual adds and the argmax are
+// fused into the prologue/epilogue of the product that produces their input,
+// so activations never take an extra trip through HBM.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "internal.h"
+
+namespace loip {
+namespace {
+
+constexpr int kWarps = 8;
+constexpr int kThreads = kWarps * 32;
+constexpr int kStageFloats = 12288;  // 48 KB of staged activations per block
+
+__device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p));
+    return r;
+}
+__device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
+__device__ __forceinline__ float bf2f(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
+__device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+// Orderable 64-bit argmax key: larger value wins; on equal values the lower
+// index wins (the low word stores ~index).
+__device__ __forceinline__ uint64_t argmax_key(float v, uint32_t idx) {
+    uint32_t u = __float_as_uint(v);
+    u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    return ((uint64_t)u << 32) | (uint64_t)(0xffffffffu - idx);
+}
+
+__device__ __forceinline__ char* kv_row(const KvView& kv, int req, int pos, int kv_or_v, int head, int Hkv, int d) {
+    int page = pos / kv.page_tokens, t = pos - page * kv.page_tokens;
+    char* p = kv.base + kv.page_offsets[(int64_t)req * kv.max_pages + page] + (uint64_t)kv.layer * kv.layer_page_bytes;
+    p += ((uint64_t)(kv_or_v * Hkv + head) * kv.page_tokens + t) * (uint64_t)d * 2u;
+    return p;
+}
+
+// ----------------------------------------------------------------------------
+// Matrix-vector family
+// ----------------------------------------------------------------------------
+enum { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_LOGITS = 3 };
+
+struct GemvParams {
+    const float* in;     // [B, K] fp32 activations
+    const uint16_t* g;   // [K] gain: input is RMSNorm(in) * g when non-null
+    const uint16_t* w0;  // [N, K]
+    const uint16_t* w1;  // [N, K] (SwiGLU up projection)
+    int B, K, N, n_units;
+    float eps;
+    float* out;
+    float* z;
+    uint64_t* keys;
+    // QKV epilogue
+    int Hq, Hkv, d;
+    float theta;
+    const int32_t* positions;
+    const int32_t* row_req;
+    KvView kv;
+};
+
+// rows handled per warp unit, by epilogue
+template <int EPI>
+struct UnitRows {
+    static constexpr int U = 2;
+};
+
+template <int EPI>
+__device__ __forceinline__ const uint16_t* unit_row(const GemvParams& p, int unit, int r, bool& valid) {
+    if (EPI == EPI_QKV) {
+        int half = p.d >> 1;
+        int h = unit / half, i = unit - h * half;
+        valid = unit < p.n_units;
+        return p.w0 + (size_t)(h * p.d + i + r * half) * p.K;
+    } else if (EPI == EPI_SWIGLU) {
+        valid = unit < p.n_units;
+        return (r ? p.w1 : p.w0) + (size_t)unit * p.K;
+    } else {
+        int row = unit * UnitRows<EPI>::U + r;
+        valid = row < p.N;
+        return p.w0 + (size_t)row * p.K;
+    }
+}
+
+// Staged-activation index of element k of row b inside a chunk.
+template <int BT>
+__device__ __forceinline__ int stage_index(int k, int b) {
+    int j = k >> 8, lane = (k >> 3) & 31;
+    if (BT == 1) {
+        int half = (k >> 2) & 1, e4 = k & 3;
+        return ((j * 2 + half) * 32 + lane) * 4 + e4;
+    } else {
+        int e = k & 7;
+        return ((j * 8 + e) * BT + b) * 32 + lane;
+    }
+}
+
+template <int BT, int U>
+__device__ __forceinline__ void fma_block(float (&acc)[U][BT], const uint4 (&w)[U], const float* __restrict__ s,
+                                          int j, int lane) {
+    if (BT == 1) {
+        const float4* s4 = reinterpret_cast<const float4*>(s);
+        float4 ya = s4[(j * 2) * 32 + lane], yb = s4[(j * 2 + 1) * 32 + lane];
+#pragma unroll
+        for (int r = 0; r < U; ++r) {
+            float a = acc[r][0];
+            a = fmaf(bf_lo(w[r].x), ya.x, a);
+            a = fmaf(bf_hi(w[r].x), ya.y, a);
+            a = fmaf(bf_lo(w[r].y), ya.z, a);
+            a = fmaf(bf_hi(w[r].y), ya.w, a);
+            a = fmaf(bf_lo(w[r].z), yb.x, a);
+            a = fmaf(bf_hi(w[r].z), yb.y, a);
+            a = fmaf(bf_lo(w[r].w), yb.z, a);
+            a = fmaf(bf_hi(w[r].w), yb.w, a);
+            acc[r][0] = a;
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            float wf[U];
+#pragma unroll
+            for (int r = 0; r < U; ++r) {
+                uint32_t word = (e < 2) ? w[r].x : (e < 4) ? w[r].y : (e < 6) ? w[r].z : w[r].w;
+                wf[r] = (e & 1) ? bf_hi(word) : bf_lo(word);
+            }
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                float y = s[((j * 8 + e) * BT + b) * 32 + lane];
+#pragma unroll
+                for (int r = 0; r < U; ++r) acc[r][b] = fmaf(wf[r], y, acc[r][b]);
+            }
+        }
+    }
+}
+
+// Accumulates the unit's rows over staged chunk [kc0, kc0 + kn).
+template <int BT, int U, int EPI>
+__device__ __forceinline__ void unit_chunk(float (&acc)[U][BT], const uint16_t* const (&rp)[U], const bool (&rv)[U],
+                                           const float* __restrict__ s, int kc0, int kn, int K, int lane) {
+    constexpr int JU = (BT <= 2) ? 4 : 2;
+    const int nj = (kn + 255) >> 8;
+    for (int j0 = 0; j0 < nj; j0 += JU) {
+        uint4 w[JU][U];
+#pragma unroll
+        for (int jj = 0; jj < JU; ++jj) {
+            int k = kc0 + (j0 + jj) * 256 + lane * 8;
+            bool ok = (j0 + jj < nj) && (k < K);
+#pragma unroll
+            for (int r = 0; r < U; ++r) w[jj][r] = (ok && rv[r]) ? ld_stream(rp[r] + k) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int jj = 0; jj < JU; ++jj)
+            if (j0 + jj < nj) fma_block<BT, U>(acc, w[jj], s, j0 + jj, lane);
+    }
+}
+
+template <int BT, int U, int EPI>
+__device__ __forceinline__ void unit_epilogue(const GemvParams& p, int unit, float (&acc)[U][BT], const float* inv,
+                                              int lane, uint64_t (&best)[BT]) {
+#pragma unroll
+    for (int r = 0; r < U; ++r)
+#pragma unroll
+        for (int b = 0; b < BT; ++b) acc[r][b] = warp_sum(acc[r][b]);
+    if (EPI == EPI_QKV) {
+        if (unit >= p.n_units) return;
+        const int half = p.d >> 1;
+        const int h = unit / half, i = unit - h * half;
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            if (lane != b || b >= p.B) continue;
+            float v0 = acc[0][b] * inv[b], v1 = acc[1][b] * inv[b];
+            const int pos = p.positions[b];
+            if (h < p.Hq + p.Hkv) {
+                double freq = pow((double)p.theta, -2.0 * (double)i / (double)p.d);
+                double s, c;
+                sincos((double)pos * freq, &s, &c);
+                float cf = (float)c, sf = (float)s;
+                float r0 = v0 * cf - v1 * sf, r1 = v1 * cf + v0 * sf;
+                v0 = r0;
+                v1 = r1;
+            }
+            if (h < p.Hq) {
+                float* q = p.out + (size_t)b * p.Hq * p.d + (size_t)h * p.d;
+                q[i] = v0;
+                q[i + half] = v1;
+            } else {
+                const int req = p.row_req ? p.row_req[b] : b;
+                const bool is_v = h >= p.Hq + p.Hkv;
+                const int kh = h - p.Hq - (is_v ? p.Hkv : 0);
+                uint16_t* row = reinterpret_cast<uint16_t*>(kv_row(p.kv, req, pos, is_v ? 1 : 0, kh, p.Hkv, p.d));
+                row[i] = f2bf(v0);
+                row[i + half] = f2bf(v1);
+            }
+        }
+    } else if (EPI == EPI_RESID) {
+#pragma unroll
+        for (int r = 0; r < U; ++r)
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                int row = unit * U + r;
+                if (lane == r * BT + b && b < p.B && row < p.N) p.out[(size_t)b * p.N + row] += acc[r][b];
+            }
+    } else if (EPI == EPI_SWIGLU) {
+        if (unit >= p.n_units) return;
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            if (lane != b || b >= p.B) continue;
+            float gt = acc[0][b] * inv[b], ut = acc[1][b] * inv[b];
+            float silu = gt / (1.0f + expf(-gt));
+            p.out[(size_t)b * p.N + unit] = silu * ut;
+        }
+    } else {  // EPI_LOGITS
+#pragma unroll
+        for (int r = 0; r < U; ++r) {
+            int row = unit * U + r;
+            if (row >= p.N) continue;
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                if (b >= p.B) continue;
+                float v = acc[r][b] * inv[b];
+                if (p.out && lane == r * BT + b) p.out[(size_t)b * p.N + row] = v;
+                uint64_t key = argmax_key(v, (uint32_t)row);
+                best[b] = key > best[b] ? key : best[b];
+            }
+        }
+    }
+}
+
+template <int BT, int EPI>
+__global__ void __launch_bounds__(kThreads, 2) gemv_kernel(GemvParams p) {
+    constexpr int U = UnitRows<EPI>::U;
+    extern __shared__ __align__(16) float s_stage[];
+    __shared__ float s_red[kWarps][BT];
+    __shared__ float s_inv[BT];
+    __shared__ uint64_t s_keys[kWarps][BT];
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int K = p.K;
+    int kc_max = (kStageFloats / BT) & ~255;
+    const bool single = K <= kc_max;
+    const int KC = single ? ((K + 255) & ~255) : kc_max;
+    const bool norm = p.g != nullptr;
+
+    float ss[BT];
+#pragma unroll
+    for (int b = 0; b < BT; ++b) ss[b] = 0.f;
+    uint64_t best[BT];
+#pragma unroll
+    for (int b = 0; b < BT; ++b) best[b] = 0;
+
+    auto stage = [&](int kc0) {
+        const int kn = min(KC, K - kc0), kpad = (kn + 255) & ~255;
+#pragma unroll
+        for (int b = 0; b < BT; ++b) {
+            for (int k = tid; k < kpad; k += kThreads) {
+                float v = 0.f;
+                if (k < kn && b < p.B) {
+                    v = p.in[(size_t)b * K + kc0 + k];
+                    if (norm) {
+                        ss[b] = fmaf(v, v, ss[b]);
+                        v *= bf2f(p.g[kc0 + k]);
+                    }
+                }
+                s_stage[stage_index<BT>(k, b)] = v;
+            }
+        }
+    };
+    auto finish_norm = [&]() {
+        if (norm) {
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                float t = warp_sum(ss[b]);
+                if (lane == 0) s_red[warp][b] = t;
+            }
+            __syncthreads();
+            if (tid < BT) {
+                float t = 0.f;
+                for (int w = 0; w < kWarps; ++w) t += s_red[w][tid];
+                s_inv[tid] = 1.0f / sqrtf(t / (float)K + p.eps);
+            }
+        } else if (tid < BT) {
+            s_inv[tid] = 1.0f;
+        }
+        __syncthreads();
+    };
+
+    if (single) {
+        stage(0);
+        __syncthreads();
+        finish_norm();
+        float inv[BT];
+#pragma unroll
+        for (int b = 0; b < BT; ++b) inv[b] = s_inv[b];
+        for (int unit = blockIdx.x * kWarps + warp; unit < p.n_units; unit += gridDim.x * kWarps) {
+            const uint16_t* rp[U];
+            bool rv[U];
+#pragma unroll
+            for (int r = 0; r < U; ++r) rp[r] = unit_row<EPI>(p, unit, r, rv[r]);
+            float acc[U][BT];
+#pragma unroll
+            for (int r = 0; r < U; ++r)
+#pragma unroll
+                for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
+            unit_chunk<BT, U, EPI>(acc, rp, rv, s_stage, 0, K, K, lane);
+            unit_epilogue<BT, U, EPI>(p, unit, acc, inv, lane, best);
+        }
+    } else {
+        const int unit = blockIdx.x * kWarps + warp;
+        const uint16_t* rp[U];
+        bool rv[U];
+#pragma unroll
+        for (int r = 0; r < U; ++r) rp[r] = unit_row<EPI>(p, unit, r, rv[r]);
+        float acc[U][BT];
+#pragma unroll
+        for (int r = 0; r < U; ++r)
+#pragma unroll
+            for (int b = 0; b < BT; ++b) acc[r][b] = 0.f;
+        for (int kc0 = 0; kc0 < K; kc0 += KC) {
+            __syncthreads();
+            stage(kc0);
+            __syncthreads();
+            unit_chunk<BT, U, EPI>(acc, rp, rv, s_stage, kc0, min(KC, K - kc0), K, lane);
+        }
+        finish_norm();
+        float inv[BT];
+#pragma unroll
+        for (int b = 0; b < BT; ++b) inv[b] = s_inv[b];
+        unit_epilogue<BT, U, EPI>(p, unit, acc, inv, lane, best);
+    }
+
+    if (EPI == EPI_LOGITS) {
+        if (lane == 0)
+#pragma unroll
+            for (int b = 0; b < BT; ++b) s_keys[warp][b] = best[b];
+        __syncthreads();
+        if (tid < BT) {
+            uint64_t k = 0;
+            for (int w = 0; w < kWarps; ++w) k = s_keys[w][tid] > k ? s_keys[w][tid] : k;
+            p.keys[(size_t)blockIdx.x * BT + tid] = k;
+        }
+        // final hidden z = RMSNorm(x) * g, written once
+        if (blockIdx.x == 0 && p.z) {
+            for (int b = 0; b < p.B; ++b)
+                for (int k = tid; k < K; k += kThreads)
+                    p.z[(size_t)b * K + k] = p.in[(size_t)b * K + k] * s_inv[b] * bf2f(p.g[k]);
+        }
+    }
+}
+
+__global__ void argmax_reduce_kernel(const uint64_t* keys, int nblocks, int BT, int B, int32_t* tokens) {
+    __shared__ uint64_t s[256];
+    const int b = blockIdx.x;
+    uint64_t k = 0;
+    for (int i = threadIdx.x; i < nblocks; i += blockDim.x) {
+        uint64_t v = keys[(size_t)i * BT + b];
+        k = v > k ? v : k;
+    }
+    s[threadIdx.x] = k;
+    __syncthreads();
+    for (int o = blockDim.x / 2; o; o >>= 1) {
+        if (threadIdx.x < o) s[threadIdx.x] = s[threadIdx.x + o] > s[threadIdx.x] ? s[threadIdx.x + o] : s[threadIdx.x];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0 && b < B) tokens[b] = (int32_t)(0xffffffffu - (uint32_t)(s[0] & 0xffffffffu));
+}
+
+template <int EPI>
+cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, int* nblocks_out = nullptr) {
+    int BT = p.B <= 1 ? 1 : p.B <= 2 ? 2 : p.B <= 4 ? 4 : 8;
+    int kc_max = (kStageFloats / BT) & ~255;
+    bool single = p.K <= kc_max;
+    int KC = single ? ((p.K + 255) & ~255) : kc_max;
+    size_t smem = (size_t)KC * BT * sizeof(float);
+    int blocks = (p.n_units + kWarps - 1) / kWarps;
+    if (single) {
+        static int per_sm[4] = {0, 0, 0, 0};
+        static int sms = 0;
+        int bi = BT == 1 ? 0 : BT == 2 ? 1 : BT == 4 ? 2 : 3;
+        if (per_sm[bi] == 0) {
+            int dev;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            int v = 0;
+            size_t sm_bytes = (size_t)kStageFloats * sizeof(float);
+            switch (BT) {
+                case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<1, EPI>, kThreads, sm_bytes); break;
+                case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<2, EPI>, kThreads, sm_bytes); break;
+                case 4: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<4, EPI>, kThreads, sm_bytes); break;
+                default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<8, EPI>, kThreads, sm_bytes); break;
+            }
+            per_sm[bi] = v < 1 ? 1 : v;
+        }
+        int cap = per_sm[bi] * sms;
+        if (blocks > cap) blocks = cap;
+    }
+    if (blocks < 1) blocks = 1;
+    if (nblocks_out) *nblocks_out = blocks;
+    static bool attr_set = false;
+    if (!attr_set) {
+        int bytes = kStageFloats * (int)sizeof(float);
+        cudaFuncSetAttribute(gemv_kernel<1, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        cudaFuncSetAttribute(gemv_kernel<2, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        cudaFuncSetAttribute(gemv_kernel<4, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        cudaFuncSetAttribute(gemv_kernel<8, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        attr_set = true;
+    }
+    switch (BT) {
+        case 1: gemv_kernel<1, EPI><<<blocks, kThreads, smem, st>>>(p); break;
+        case 2: gemv_kernel<2, EPI><<<blocks, kThreads, smem, st>>>(p); break;
+        case 4: gemv_kernel<4, EPI><<<blocks, kThreads, smem, st>>>(p); break;
+        default: gemv_kernel<8, EPI><<<blocks, kThreads, smem, st>>>(p); break;
+    }
+    return cudaGetLastError();
+}
+
+// ----------------------------------------------------------------------------
+// Attention
+// ----------------------------------------------------------------------------
+struct AttnParams {
+    const float* q;  // [B, Hq*d]
+    KvView kv;
+    const int32_t* ctx_lens;
+    const int32_t* positions;  // used when ctx_lens is null: ctx = position + 1
+    const int32_t* row_req;
+    int B, Hq, Hkv, max_chunks;
+    float scale;
+    float* scratch;  // split: [B][Hq][max_chunks][d + 2]
+    void* o;         // [B, Hq*d] fp32 or bf16
+    int o_bf16;
+    int split;
+};
+
+template <int G, int D>
+__global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
+    constexpr int DPL = D / 32;  // dims per lane in the PV product
+    __shared__ __align__(16) float sq[G][D];
+    __shared__ float s_m[G], s_l[G];
+    __shared__ float s_o[G][D];
+
+    const int row = blockIdx.z, kvh = blockIdx.y;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
+    const int P = p.kv.page_tokens;
+    const int npages = (ctx + P - 1) / P;
+    int pg0, pg1;
+    if (p.split) {
+        pg0 = blockIdx.x;
+        pg1 = pg0 + 1;
+        if (pg0 >= npages) return;
+    } else {
+        pg0 = 0;
+        pg1 = npages;
+    }
+    const int req = p.row_req ? p.row_req[row] : row;
+    for (int i = threadIdx.x; i < G * D; i += 64)
+        sq[i / D][i % D] = p.q[(size_t)row * p.Hq * D + (size_t)kvh * G * D + i];
+    __syncthreads();
+
+    float m[G], l[G], o[G][DPL];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+        m[g] = -INFINITY;
+        l[g] = 0.f;
+#pragma unroll
+        for (int c = 0; c < DPL; ++c) o[g][c] = 0.f;
+    }
+    const int Hkv = p.Hkv;
+    for (int pg = pg0; pg < pg1; ++pg) {
+        const char* page = p.kv.base + p.kv.page_offsets[(int64_t)req * p.kv.max_pages + pg] +
+                           (uint64_t)p.kv.layer * p.kv.layer_page_bytes;
+        const uint16_t* Kh = reinterpret_cast<const uint16_t*>(page) + (size_t)kvh * P * D;
+        const uint16_t* Vh = reinterpret_cast<const uint16_t*>(page) + ((size_t)Hkv + kvh) * P * D;
+        for (int t0 = warp * 32; t0 < P; t0 += 64) {
+            const int tl = t0 + lane;
+            const bool valid = (pg * P + tl) < ctx && tl < P;
+            float s[G];
+#pragma unroll
+            for (int g = 0; g < G; ++g) s[g] = 0.f;
+            if (valid) {
+                const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)tl * D);
+#pragma unroll 4
+                for (int dd = 0; dd < D / 8; ++dd) {
+                    uint4 kk = kr[dd];
+                    float kf[8] = {bf_lo(kk.x), bf_hi(kk.x), bf_lo(kk.y), bf_hi(kk.y),
+                                   bf_lo(kk.z), bf_hi(kk.z), bf_lo(kk.w), bf_hi(kk.w)};
+#pragma unroll
+                    for (int g = 0; g < G; ++g) {
+                        const float4 qa = *reinterpret_cast<const float4*>(&sq[g][dd * 8]);
+                        const float4 qb = *reinterpret_cast<const float4*>(&sq[g][dd * 8 + 4]);
+                        float a = s[g];
+                        a = fmaf(qa.x, kf[0], a);
+                        a = fmaf(qa.y, kf[1], a);
+                        a = fmaf(qa.z, kf[2], a);
+                        a = fmaf(qa.w, kf[3], a);
+                        a = fmaf(qb.x, kf[4], a);
+                        a = fmaf(qb.y, kf[5], a);
+                        a = fmaf(qb.z, kf[6], a);
+                        a = fmaf(qb.w, kf[7], a);
+                        s[g] = a;
+                    }
+                }
+            }
+            float pe[G];
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+                float sv = valid ? s[g] * p.scale : -INFINITY;
+                float mx = warp_max(sv);
+                float mn = fmaxf(m[g], mx);
+                float corr = (m[g] == -INFINITY) ? 0.f : expf(m[g] - mn);
+                pe[g] = valid ? expf(sv - mn) : 0.f;
+                l[g] = l[g] * corr + warp_sum(pe[g]);
+#pragma unroll
+                for (int c = 0; c < DPL; ++c) o[g][c] *= corr;
+                m[g] = mn;
+            }
+            const int nt = min(32, min(P - t0, ctx - (pg * P + t0)));
+            for (int tt = 0; tt < nt; ++tt) {
+                const uint16_t* vr = Vh + (size_t)(t0 + tt) * D + lane * DPL;
+                float vf[DPL];
+                if constexpr (DPL == 4) {
+                    uint2 vv = *reinterpret_cast<const uint2*>(vr);
+                    vf[0] = bf_lo(vv.x);
+                    vf[1] = bf_hi(vv.x);
+                    vf[2] = bf_lo(vv.y);
+                    vf[3] = bf_hi(vv.y);
+                } else {
+                    static_assert(DPL == 2, "head_dim 64 or 128");
+                    uint32_t vv = *reinterpret_cast<const uint32_t*>(vr);
+                    vf[0] = bf_lo(vv);
+                    vf[1] = bf_hi(vv);
+                }
+#pragma unroll
+                for (int g = 0; g < G; ++g) {
+                    float pg_ = __shfl_sync(0xffffffffu, pe[g], tt);
+#pragma unroll
+                    for (int c = 0; c < DPL; ++c) o[g][c] = fmaf(pg_, vf[c], o[g][c]);
+                }
+            }
+        }
+    }
+    // merge the two warps
+    if (warp == 1) {
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+            if (lane == 0) {
+                s_m[g] = m[g];
+                s_l[g] = l[g];
+            }
+#pragma unroll
+            for (int c = 0; c < DPL; ++c) s_o[g][lane * DPL + c] = o[g][c];
+        }
+    }
+    __syncthreads();
+    if (warp == 0) {
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+            float m1 = s_m[g], l1 = s_l[g];
+            float mn = fmaxf(m[g], m1);
+            float c0 = (m[g] == -INFINITY) ? 0.f : expf(m[g] - mn);
+            float c1 = (m1 == -INFINITY) ? 0.f : expf(m1 - mn);
+            float lt = l[g] * c0 + l1 * c1;
+            const int h = kvh * G + g;
+            if (p.split) {
+                float* part = p.scratch + (((size_t)row * p.Hq + h) * p.max_chunks + blockIdx.x) * (D + 2);
+#pragma unroll
+                for (int c = 0; c < DPL; ++c) part[lane * DPL + c] = o[g][c] * c0 + s_o[g][lane * DPL + c] * c1;
+                if (lane == 0) {
+                    part[D] = mn;
+                    part[D + 1] = lt;
+                }
+            } else {
+                float invl = lt > 0.f ? 1.0f / lt : 0.f;
+#pragma unroll
+                for (int c = 0; c < DPL; ++c) {
+                    float v = (o[g][c] * c0 + s_o[g][lane * DPL + c] * c1) * invl;
+                    size_t idx = (size_t)row * p.Hq * D + (size_t)h * D + lane * DPL + c;
+                    if (p.o_bf16)
+                        reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(v);
+                    else
+                        reinterpret_cast<float*>(p.o)[idx] = v;
+                }
+            }
+        }
+    }
+}
+
+// Combines the per-page partial softmax states of one (row, head).
+__global__ void attn_combine_kernel(AttnParams p, int D) {
+    const int h = blockIdx.x, row = blockIdx.y, j = threadIdx.x;
+    const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
+    const int n = (ctx + p.kv.page_tokens - 1) / p.kv.page_tokens;
+    const float* part = p.scratch + ((size_t)row * p.Hq + h) * p.max_chunks * (D + 2);
+    float M = -INFINITY;
+    for (int c = 0; c < n; ++c) M = fmaxf(M, part[(size_t)c * (D + 2) + D]);
+    float L = 0.f, acc = 0.f;
+    for (int c = 0; c < n; ++c) {
+        const float* pc = part + (size_t)c * (D + 2);
+        float w = (pc[D] == -INFINITY) ? 0.f : expf(pc[D] - M);
+        L += pc[D + 1] * w;
+        acc += pc[j] * w;
+    }
+    float v = L > 0.f ? acc / L : 0.f;
+    size_t idx = (size_t)row * p.Hq * D + (size_t)h * D + j;
+    if (p.o_bf16)
+        reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(v);
+    else
+        reinterpret_cast<float*>(p.o)[idx] = v;
+}
+
+template <int G, int D>
+cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st) {
+    dim3 grid(p.split ? p.max_chunks : 1, p.Hkv, p.B);
+    attn_kernel<G, D><<<grid, 64, 0, st>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || !p.split) return e;
+    attn_combine_kernel<<<dim3(p.Hq, p.B), D, 0, st>>>(p, D);
+    return cudaGetLastError();
+}
+
+// ----------------------------------------------------------------------------
+// Embedding gather and generator
+// ----------------------------------------------------------------------------
+__global__ void embed_kernel(const uint16_t* E, const int32_t* tokens, int H, int V, float* x) {
+    const int b = blockIdx.x;
+    const int tok = tokens[b];
+    const bool ok = tok >= 0 && tok < V;
+    const uint16_t* row = E + (size_t)(ok ? tok : 0) * H;
+    for (int i = threadIdx.x; i < H; i += blockDim.x) x[(size_t)b * H + i] = ok ? bf2f(row[i]) : 0.f;
+}
+
+// SplitMix64 (Steele, Lea & Flood 2014) used as a counter-based generator:
+// output k of the stream seeded with s is mix(s + (k+1) * golden gamma).
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t k) {
+    uint64_t z = seed + (k + 1ull) * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+// Irwin-Hall (n = 4) sum of the four 16-bit fields, centred, scaled so the
+// standard deviation is 0.02 (weights) or 1 + 0.02 z (gains); bf16 RNE.
+__device__ __forceinline__ uint16_t gen_elem(uint64_t seed, uint32_t tensor_id, uint64_t index, int kind) {
+    uint64_t r = splitmix64_at(seed, ((uint64_t)tensor_id << 40) | index);
+    int s = (int)(r & 0xffffu) + (int)((r >> 16) & 0xffffu) + (int)((r >> 32) & 0xffffu) + (int)(r >> 48);
+    float z = __fmul_rn(__int2float_rn(s - 131070), 0x1p-16f);
+    float w = __fmul_rn(z, 0x1.1bc77ap-5f);
+    if (kind == 1) w = __fadd_rn(1.0f, w);
+    return f2bf(w);
+}
+
+__global__ void advance_kernel(int32_t* pos, int B) {
+    if ((int)threadIdx.x < B) pos[threadIdx.x] += 1;
+}
+
+__global__ void generate_kernel(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id,
+                                int kind) {
+    uint64_t i = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x;
+    const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+    for (; i < n; i += stride) out[i] = gen_elem(seed, tensor_id, first + i, kind);
+}
+
+}  // namespace
+
+// ----------------------------------------------------------------------------
+// launchers
+// ----------------------------------------------------------------------------
+cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
+                            int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
+                            const int32_t* row_req, cudaStream_t st) {
+    GemvParams p{};
+    p.in = x;
+    p.g = g;
+    p.w0 = wqkv;
+    p.B = B;
+    p.K = H;
+    p.N = (Hq + 2 * Hkv) * d;
+    p.n_units = p.N / 2;
+    p.eps = eps;
+    p.out = q_out;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.d = d;
+    p.theta = theta;
+    p.positions = positions;
+    p.row_req = row_req;
+    p.kv = kv;
+    return launch_gemv<EPI_QKV>(p, st);
+}
+
+cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st) {
+    GemvParams p{};
+    p.in = in;
+    p.w0 = w;
+    p.B = B;
+    p.K = K;
+    p.N = N;
+    p.n_units = (N + 1) / 2;
+    p.out = x;
+    return launch_gemv<EPI_RESID>(p, st);
+}
+
+cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,
+                           int F, float eps, float* a, cudaStream_t st) {
+    GemvParams p{};
+    p.in = x;
+    p.g = g;
+    p.w0 = wg;
+    p.w1 = wu;
+    p.B = B;
+    p.K = H;
+    p.N = F;
+    p.n_units = F;
+    p.eps = eps;
+    p.out = a;
+    return launch_gemv<EPI_SWIGLU>(p, st);
+}
+
+size_t lm_head_scratch_bytes(int B, int V) {
+    (void)B;
+    // one key per (block, batch slot) for at most ceil(V/2/kWarps) blocks and 8 slots
+    size_t blocks = ((size_t)V / 2 + kWarps) / kWarps + 1;
+    return blocks * 8 * sizeof(uint64_t);
+}
+
+cudaError_t launch_lm_head(const float* x, const uint16_t* g, const uint16_t* w, int B, int H, int V, float eps,
+                           float* z, float* logits, int32_t* tokens, void* scratch, cudaStream_t st) {
+    GemvParams p{};
+    p.in = x;
+    p.g = g;
+    p.w0 = w;
+    p.B = B;
+    p.K = H;
+    p.N = V;
+    p.n_units = (V + 1) / 2;
+    p.eps = eps;
+    p.out = logits;
+    p.z = z;
+    p.keys = reinterpret_cast<uint64_t*>(scratch);
+    int nblocks = 0;
+    cudaError_t e = launch_gemv<EPI_LOGITS>(p, st, &nblocks);
+    if (e != cudaSuccess) return e;
+    int BT = B <= 1 ? 1 : B <= 2 ? 2 : B <= 4 ? 4 : 8;
+    argmax_reduce_kernel<<<B, 256, 0, st>>>(p.keys, nblocks, BT, B, tokens);
+    return cudaGetLastError();
+}
+
+size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens) {
+    size_t chunks = ((size_t)max_ctx + page_tokens - 1) / page_tokens;
+    return (size_t)B * Hq * chunks * (d + 2);
+}
+
+cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
+                             const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
+                             float* scratch, void* o, bool o_bf16, cudaStream_t st) {
+    AttnParams p{};
+    p.q = q;
+    p.kv = kv;
+    p.ctx_lens = ctx_lens;
+    p.positions = positions;
+    p.row_req = row_req;
+    p.B = B;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.max_chunks = (max_ctx + kv.page_tokens - 1) / kv.page_tokens;
+    p.scale = 1.0f / sqrtf((float)d);
+    p.scratch = scratch;
+    p.o = o;
+    p.o_bf16 = o_bf16 ? 1 : 0;
+    p.split = split ? 1 : 0;
+    const int G = Hq / Hkv;
+    if (d == 128) {
+        switch (G) {
+            case 1: return launch_attn_t<1, 128>(p, st);
+            case 2: return launch_attn_t<2, 128>(p, st);
+            case 4: return launch_attn_t<4, 128>(p, st);
+            case 8: return launch_attn_t<8, 128>(p, st);
+        }
+    } else if (d == 64) {
+        switch (G) {
+            case 1: return launch_attn_t<1, 64>(p, st);
+            case 2: return launch_attn_t<2, 64>(p, st);
+            case 4: return launch_attn_t<4, 64>(p, st);
+            case 8: return launch_attn_t<8, 64>(p, st);
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_embed(const uint16_t* embed, const int32_t* tokens, int B, int H, int V, float* x,
+                         cudaStream_t st) {
+    embed_kernel<<<B, 256, 0, st>>>(embed, tokens, H, V, x);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st) {
+    advance_kernel<<<1, 32, 0, st>>>(positions, B);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id, int kind,
+                            cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    uint64_t blocks = (n + 255) / 256;
+    if (blocks > 152 * 32) blocks = 152 * 32;
+    generate_kernel<<<(unsigned)blocks, 256, 0, st>>>(out, n, first, seed, tensor_id, kind);
+    return cudaGetLastError();
+}
+
+}  // namespace loip

@@ -1,0 +1,64 @@
+// internal.h -- launchers shared between the translation units of libloip.
+// Host-side declarations only; kernels live in decode.cu / prefill.cu.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace loip {
+
+// Paged KV cache view for one layer.  A page (one per page_tokens positions of
+// one request) is a contiguous group holding every layer's keys and values:
+// at byte offset layer * layer_page_bytes sit K [Hkv][page_tokens][d] and then
+// V [Hkv][page_tokens][d], bf16.  page_offsets[row * max_pages + i] is the
+// byte offset of page i of page-table row `row` from `base`.
+struct KvView {
+    char* base;
+    const int64_t* page_offsets;
+    int32_t max_pages;
+    int32_t page_tokens;
+    int32_t layer;
+    uint64_t layer_page_bytes;
+};
+
+// Weight-stationary matrix-vector family (decode).  B = batch rows of the fp32
+// activation; every kernel streams its weight matrix exactly once.
+cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
+                            int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
+                            const int32_t* row_req, cudaStream_t st);
+cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st);
+cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,
+                           int F, float eps, float* a, cudaStream_t st);
+cudaError_t launch_lm_head(const float* x, const uint16_t* g, const uint16_t* w, int B, int H, int V, float eps,
+                           float* z, float* logits, int32_t* tokens, void* scratch, cudaStream_t st);
+size_t lm_head_scratch_bytes(int B, int V);
+
+// Grouped-query attention over the paged cache.  Rows b = 0..B-1 attend over
+// their first ctx_lens[b] positions with query q[b] (ctx_lens NULL: over
+// positions[b] + 1 positions, the causal window of the token at positions[b]).  row_req maps a row to its
+// page-table row (NULL = identity).  split: partial states go to scratch and a
+// combine kernel writes o; otherwise one block per (row, kv head) loops over all
+// pages.  o_bf16: write o as bf16 (prefill) instead of fp32.
+cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
+                             const int32_t* row_req, int B, int Hq,
+                             int Hkv, int d, int max_ctx, bool split, float* scratch, void* o, bool o_bf16,
+                             cudaStream_t st);
+size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens);
+
+cudaError_t launch_embed(const uint16_t* embed, const int32_t* tokens, int B, int H, int V, float* x,
+                         cudaStream_t st);
+cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st);
+cudaError_t launch_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id, int kind,
+                            cudaStream_t st);
+
+// Prefill (M tokens at once): bf16 x fp32-accumulate GEMMs with fused epilogues.
+cudaError_t launch_rmsnorm_bf16(const float* x, const uint16_t* g, int M, int H, float eps, uint16_t* y,
+                                cudaStream_t st);
+cudaError_t launch_gemm_qkv_rope(const uint16_t* y, const uint16_t* wqkv, int M, int H, int Hq, int Hkv, int d,
+                                 float theta, const int32_t* positions, const int32_t* row_req, float* q, KvView kv,
+                                 cudaStream_t st);
+cudaError_t launch_gemm_resid(const uint16_t* a, const uint16_t* w, int M, int N, int K, float* x, cudaStream_t st);
+cudaError_t launch_gemm_swiglu(const uint16_t* y, const uint16_t* wg, const uint16_t* wu, int M, int H, int F,
+                               uint16_t* a, cudaStream_t st);
+cudaError_t launch_gather_rows(const float* x, const int32_t* rows, int n, int H, float* out, cudaStream_t st);
+
+}  // namespace loip

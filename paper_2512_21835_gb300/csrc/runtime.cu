@@ -1,0 +1,1244 @@
+// runtime.cu -- the LOIP runtime on one GPU: device arena and block allocator,
+// pinned host weight pool, slot ring on a dedicated copy stream chained to the
+// compute stream by CUDA events, paged KV cache, decode step, prefill and
+// online re-planning; and the C ABI (include/loip.h).
+//
+// Loading path (Sec. III-C).  The paper replaces copy-then-compute with one
+// reusable loading slot that the runtime refills as soon as the GPU signals,
+// through a CUDA event, that it finished the weights in it.  Here the slot is
+// a ring of K device slots: the copy of offloaded layer j+K into slot
+// (j mod K) waits on slot_free[j mod K] (recorded on the compute stream after
+// layer j's kernels) and records slot_full, which layer j+K's kernels wait
+// for.  The ring runs across step boundaries, so the first offloaded layers of
+// the next step load during the tail of the current one (Fig. 2b, F_N').
+// Layer descriptors are computed once (the paper's proxy modules): a slot
+// rebinding is a pointer change.
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+#include <time.h>
+
+#include <algorithm>
+#include <chrono>
+#include <deque>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include "../../include/loip.h"
+#include "internal.h"
+#include "plan.h"
+
+using namespace loip;
+
+namespace {
+
+thread_local std::string g_create_error;
+
+constexpr uint64_t kAlign = 256;
+inline uint64_t align_up(uint64_t v, uint64_t a = kAlign) { return (v + a - 1) / a * a; }
+
+enum BlockKind { B_FREE = 0, B_LAYER = 1, B_SLOT = 2, B_KV = 3 };
+
+struct Request {
+    std::vector<int64_t> pages;  // byte offsets of page groups from the arena base
+    int32_t len = 0;             // tokens in the cache
+};
+
+struct Fixed {  // offsets inside the fixed region
+    uint64_t embed, lm_head, g_final, x, q, o, a, z, logits, attn_scratch, lm_scratch;
+    uint64_t tokens, out_tokens, positions, ctx_lens, row_req, page_table, last_rows, dec_pos;
+    uint64_t px, py, pq, po, pa;
+    uint64_t total;
+};
+
+int validate_desc(const loip_model_desc* d) {
+    if (!d) return LOIP_ERR_INVALID;
+    if (d->n_layers <= 0 || d->hidden <= 0 || d->n_heads <= 0 || d->n_kv_heads <= 0 || d->head_dim <= 0 ||
+        d->ffn <= 0 || d->vocab <= 0)
+        return LOIP_ERR_INVALID;
+    if (d->hidden % 8 || d->ffn % 8 || (d->head_dim != 64 && d->head_dim != 128) || d->n_heads % d->n_kv_heads)
+        return LOIP_ERR_INVALID;
+    int G = d->n_heads / d->n_kv_heads;
+    if (G != 1 && G != 2 && G != 4 && G != 8) return LOIP_ERR_INVALID;
+    if (!(d->rms_eps > 0) || !(d->rope_theta > 1)) return LOIP_ERR_INVALID;
+    return LOIP_OK;
+}
+
+void layout_of(const loip_model_desc* d, loip_layer_layout_t* o) {
+    const uint64_t H = d->hidden, F = d->ffn, qd = (uint64_t)d->n_heads * d->head_dim,
+                   kvd = (uint64_t)d->n_kv_heads * d->head_dim;
+    uint64_t off = 0;
+    o->off_g_attn = off;
+    off = align_up(off + H * 2);
+    o->off_wqkv = off;
+    off = align_up(off + (qd + 2 * kvd) * H * 2);
+    o->off_wo = off;
+    off = align_up(off + H * qd * 2);
+    o->mha_bytes = off;
+    o->off_g_mlp = off;
+    off = align_up(off + H * 2);
+    o->off_wg = off;
+    off = align_up(off + F * H * 2);
+    o->off_wu = off;
+    off = align_up(off + F * H * 2);
+    o->off_wd = off;
+    off = align_up(off + H * F * 2);
+    o->l_size = off;
+    o->mlp_bytes = off - o->mha_bytes;
+}
+
+loip_config normalized(const loip_config* c) {
+    loip_config r = *c;
+    if (r.page_tokens <= 0) r.page_tokens = 64;
+    if (r.timeout_ms == 0) r.timeout_ms = 600000;
+    if (r.max_prefill_tokens <= 0) r.max_prefill_tokens = 512;
+    if (!(r.hbm_Bps > 0)) r.hbm_Bps = 6.7e12;
+    if (!(r.link_Bps > 0)) r.link_Bps = 2.0e11;
+    return r;
+}
+
+Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
+    Fixed f{};
+    const uint64_t H = d->hidden, V = d->vocab, F = d->ffn, qd = (uint64_t)d->n_heads * d->head_dim;
+    const uint64_t B = c->max_batch, Mp = c->max_prefill_tokens;
+    const uint64_t rows = std::max<uint64_t>(B, Mp);
+    const uint64_t max_pages = (c->max_ctx + c->page_tokens - 1) / c->page_tokens;
+    uint64_t off = 0;
+    auto take = [&](uint64_t bytes) {
+        uint64_t o = off;
+        off = align_up(off + bytes);
+        return o;
+    };
+    f.embed = take(V * H * 2);
+    f.lm_head = take(V * H * 2);
+    f.g_final = take(H * 2);
+    f.x = take(B * H * 4);
+    f.q = take(B * qd * 4);
+    f.o = take(B * qd * 4);
+    f.a = take(B * F * 4);
+    f.z = take(B * H * 4);
+    f.logits = take(B * V * 4);
+    f.attn_scratch = take(attention_scratch_floats((int)B, d->n_heads, d->head_dim, c->max_ctx, c->page_tokens) * 4);
+    f.lm_scratch = take(lm_head_scratch_bytes((int)B, (int)V));
+    f.tokens = take(rows * 4);
+    f.out_tokens = take(rows * 4);
+    f.positions = take(rows * 4);
+    f.ctx_lens = take(rows * 4);
+    f.row_req = take(rows * 4);
+    f.last_rows = take(B * 4);
+    f.dec_pos = take(B * 4);
+    f.page_table = take(B * max_pages * 8);
+    f.px = take(Mp * H * 4);
+    f.py = take(Mp * H * 2);
+    f.pq = take(Mp * qd * 4);
+    f.po = take(Mp * qd * 2);
+    f.pa = take(Mp * F * 2);
+    f.total = off;
+    return f;
+}
+
+}  // namespace
+
+struct loip_ctx {
+    loip_model_desc desc{};
+    loip_config cfg{};
+    loip_layer_layout_t lay{};
+    int L = 0, H = 0, Hq = 0, Hkv = 0, d = 0, F = 0, V = 0, qd = 0, kvd = 0;
+    char* arena = nullptr;
+    uint64_t budget = 0;
+    Fixed fx{};
+    // blocks (layer-sized)
+    uint64_t block_bytes = 0, blocks_off = 0;
+    int n_blocks = 0;
+    std::vector<int> block_kind, block_owner;
+    std::vector<int> layer_block;   // resident block of each layer, -1 if offloaded
+    std::vector<uint8_t> offloaded;
+    std::vector<int> slot_block;
+    std::vector<int> off_order;     // offloaded layers in order
+    // KV
+    uint64_t kv_tok_bytes = 0, layer_page_bytes = 0, group_bytes = 0, kv_region_off = 0, kv_region_bytes = 0;
+    std::vector<int64_t> free_groups;
+    uint64_t kv_groups_total = 0;
+    std::vector<Request> reqs;
+    int max_pages = 0;
+    bool pt_dirty = true;
+    // host pool
+    std::vector<void*> host_layer;
+    int32_t* h_stage = nullptr;  // pinned staging for small transfers
+    size_t h_stage_ints = 0;
+    int64_t* h_pt = nullptr;     // pinned page-table staging
+    // streams and events
+    cudaStream_t compute = nullptr, copy = nullptr;
+    std::vector<cudaEvent_t> slot_full, slot_free;
+    cudaEvent_t ev_done = nullptr, ev_step0 = nullptr, ev_step1 = nullptr, ev_reach = nullptr;
+    cudaEvent_t ev_stage = nullptr;  // last transfer that read the pinned staging buffers
+    bool pos_dirty = true;
+    std::deque<std::pair<cudaEvent_t, cudaEvent_t>> copy_events;
+    std::vector<cudaEvent_t> event_pool;
+    uint64_t copy_seq = 0, compute_seq = 0;
+    bool ktiming = false;
+    struct KEv {
+        int cls;
+        cudaEvent_t a, b;
+    };
+    std::deque<KEv> kernel_events;
+    bool weights_loaded = false;
+    bool failed = false;
+    int active_batch = 0;
+    loip_stats st{};
+    std::string err;
+
+    // ---------------------------------------------------------------------
+    int fail(int code, const std::string& m) {
+        err = m;
+        return code;
+    }
+    int cuda_fail(cudaError_t e, const char* what) {
+        err = std::string(what) + ": " + cudaGetErrorString(e);
+        if (e != cudaErrorNotReady) failed = true;
+        return LOIP_ERR_CUDA;
+    }
+    template <class T>
+    T* fixed_ptr(uint64_t off) {
+        return reinterpret_cast<T*>(arena + off);
+    }
+    char* block_ptr(int b) { return arena + blocks_off + (uint64_t)b * block_bytes; }
+    char* slot_ptr(int k) { return block_ptr(slot_block[k]); }
+    int n_slots_used() const { return off_order.empty() ? 0 : cfg.n_slots; }
+
+    cudaEvent_t take_event() {
+        if (!event_pool.empty()) {
+            cudaEvent_t e = event_pool.back();
+            event_pool.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        cudaEventCreate(&e);
+        return e;
+    }
+
+    int wait_event(cudaEvent_t e) {
+        auto t0 = std::chrono::steady_clock::now();
+        for (;;) {
+            cudaError_t r = cudaEventQuery(e);
+            if (r == cudaSuccess) return LOIP_OK;
+            if (r != cudaErrorNotReady) return cuda_fail(r, "device work failed");
+            double ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
+            if (ms > (double)cfg.timeout_ms) {
+                failed = true;
+                return fail(LOIP_ERR_TIMEOUT, "timed out waiting for the device");
+            }
+            std::this_thread::yield();
+        }
+    }
+
+    int sync_all() {
+        cudaError_t e = cudaEventRecord(ev_done, copy);
+        if (e != cudaSuccess) return cuda_fail(e, "event record");
+        int r = wait_event(ev_done);
+        if (r) return r;
+        e = cudaEventRecord(ev_done, compute);
+        if (e != cudaSuccess) return cuda_fail(e, "event record");
+        return wait_event(ev_done);
+    }
+
+    const uint16_t* layer_weights(int l, int slot) {
+        if (layer_block[l] >= 0) return reinterpret_cast<const uint16_t*>(block_ptr(layer_block[l]));
+        return reinterpret_cast<const uint16_t*>(slot_ptr(slot));
+    }
+
+    KvView kv_view(int layer, const int64_t* pt) {
+        KvView v;
+        v.base = arena;
+        v.page_offsets = pt;
+        v.max_pages = max_pages;
+        v.page_tokens = cfg.page_tokens;
+        v.layer = layer;
+        v.layer_page_bytes = layer_page_bytes;
+        return v;
+    }
+
+    // ---- block and KV allocation -----------------------------------------
+    int take_free_block() {
+        for (int b = 0; b < n_blocks; ++b)
+            if (block_kind[b] == B_FREE) return b;
+        return -1;
+    }
+
+    int grow_kv() {  // converts one free block into page groups
+        int b = take_free_block();
+        if (b < 0) return -1;
+        block_kind[b] = B_KV;
+        uint64_t n = block_bytes / group_bytes;
+        for (uint64_t i = 0; i < n; ++i)
+            free_groups.push_back((int64_t)(blocks_off + (uint64_t)b * block_bytes + i * group_bytes));
+        kv_groups_total += n;
+        return b;
+    }
+
+    int ensure_pages(int req, int tokens) {
+        Request& r = reqs[req];
+        int need = (tokens + cfg.page_tokens - 1) / cfg.page_tokens;
+        if (need > max_pages) return fail(LOIP_ERR_INVALID, "context longer than max_ctx");
+        while ((int)r.pages.size() < need) {
+            if (free_groups.empty()) {
+                if (grow_kv() < 0) {
+                    int rc = demote_for_kv();
+                    if (rc) return rc;
+                    if (grow_kv() < 0) return fail(LOIP_ERR_OOM, "no block for the KV cache");
+                }
+            }
+            r.pages.push_back(free_groups.back());
+            free_groups.pop_back();
+            pt_dirty = true;
+        }
+        return LOIP_OK;
+    }
+
+    void release_pages(int req) {
+        for (int64_t g : reqs[req].pages) free_groups.push_back(g);
+        reqs[req].pages.clear();
+        reqs[req].len = 0;
+        pt_dirty = true;
+    }
+
+    int upload_page_table(cudaStream_t s) {
+        if (!pt_dirty) return LOIP_OK;
+        int rc = wait_event(ev_stage);  // a previous upload may still read the staging buffer
+        if (rc) return rc;
+        for (int b = 0; b < cfg.max_batch; ++b)
+            for (int i = 0; i < max_pages; ++i)
+                h_pt[(size_t)b * max_pages + i] = i < (int)reqs[b].pages.size() ? reqs[b].pages[i] : 0;
+        cudaError_t e = cudaMemcpyAsync(arena + fx.page_table, h_pt, (size_t)cfg.max_batch * max_pages * 8,
+                                        cudaMemcpyHostToDevice, s);
+        if (e != cudaSuccess) return cuda_fail(e, "page table upload");
+        cudaEventRecord(ev_stage, s);
+        pt_dirty = false;
+        return LOIP_OK;
+    }
+
+    int upload_positions(int B, cudaStream_t s) {
+        if (!pos_dirty) return LOIP_OK;
+        int rc = wait_event(ev_stage);
+        if (rc) return rc;
+        int32_t* hp = h_stage + 2 * (h_stage_ints / 4);
+        for (int b = 0; b < B; ++b) hp[b] = reqs[b].len;
+        cudaError_t e = cudaMemcpyAsync(arena + fx.dec_pos, hp, (size_t)B * 4, cudaMemcpyHostToDevice, s);
+        if (e != cudaSuccess) return cuda_fail(e, "positions upload");
+        cudaEventRecord(ev_stage, s);
+        pos_dirty = false;
+        return LOIP_OK;
+    }
+
+    // ---- streaming ------------------------------------------------------------
+    int enqueue_copy(int layer, int slot, cudaStream_t cs) {
+        cudaError_t e = cudaStreamWaitEvent(cs, slot_free[slot], 0);
+        if (e != cudaSuccess) return cuda_fail(e, "copy wait");
+        cudaEvent_t e0 = take_event(), e1 = take_event();
+        cudaEventRecord(e0, cs);
+        e = cudaMemcpyAsync(slot_ptr(slot), host_layer[layer], lay.l_size, cudaMemcpyHostToDevice, cs);
+        if (e != cudaSuccess) return cuda_fail(e, "layer copy");
+        cudaEventRecord(e1, cs);
+        copy_events.emplace_back(e0, e1);
+        e = cudaEventRecord(slot_full[slot], cs);
+        if (e != cudaSuccess) return cuda_fail(e, "slot event");
+        st.h2d_weight_bytes += lay.l_size;
+        return LOIP_OK;
+    }
+
+    int issue_next_copy() {  // ring order over offloaded layers, across steps
+        const int m = (int)off_order.size();
+        int rc = enqueue_copy(off_order[copy_seq % m], (int)(copy_seq % cfg.n_slots), copy);
+        if (rc) return rc;
+        ++copy_seq;
+        return LOIP_OK;
+    }
+
+    int prime_slots() {
+        copy_seq = compute_seq = 0;
+        if (off_order.empty() || cfg.mode == LOIP_MODE_NAIVE) return LOIP_OK;
+        for (int k = 0; k < cfg.n_slots; ++k) {
+            int rc = issue_next_copy();
+            if (rc) return rc;
+        }
+        return LOIP_OK;
+    }
+
+    void rebuild_order() {
+        off_order.clear();
+        for (int l = 0; l < L; ++l)
+            if (offloaded[l]) off_order.push_back(l);
+    }
+
+    // ---- kernel timing ------------------------------------------------------
+    template <class Fn>
+    cudaError_t timed(int cls, cudaStream_t s, Fn&& fn) {
+        if (!ktiming) return fn();
+        cudaEvent_t a = take_event(), b = take_event();
+        cudaEventRecord(a, s);
+        cudaError_t e = fn();
+        cudaEventRecord(b, s);
+        kernel_events.push_back({cls, a, b});
+        return e;
+    }
+    void collect_kernel_times() {
+        while (!kernel_events.empty()) {
+            KEv k = kernel_events.front();
+            if (cudaEventQuery(k.b) != cudaSuccess) break;
+            float ms = 0;
+            cudaEventElapsedTime(&ms, k.a, k.b);
+            st.kernel_ms[k.cls] += ms;
+            st.kernel_launches[k.cls] += 1;
+            event_pool.push_back(k.a);
+            event_pool.push_back(k.b);
+            kernel_events.pop_front();
+        }
+    }
+
+    // ---- one decoder layer ---------------------------------------------------
+    // Decode-time layer on rows 0..B-1 of the fixed activations.
+    int decode_layer(int l, int B, const int32_t* pos_dev, cudaStream_t s, int slot) {
+        const uint16_t* w = layer_weights(l, slot);
+        const uint16_t* g_attn = w + lay.off_g_attn / 2;
+        const uint16_t* wqkv = w + lay.off_wqkv / 2;
+        const uint16_t* wo = w + lay.off_wo / 2;
+        const uint16_t* g_mlp = w + lay.off_g_mlp / 2;
+        const uint16_t* wg = w + lay.off_wg / 2;
+        const uint16_t* wu = w + lay.off_wu / 2;
+        const uint16_t* wd = w + lay.off_wd / 2;
+        float* x = fixed_ptr<float>(fx.x);
+        float* q = fixed_ptr<float>(fx.q);
+        float* o = fixed_ptr<float>(fx.o);
+        float* a = fixed_ptr<float>(fx.a);
+        const int64_t* pt = fixed_ptr<int64_t>(fx.page_table);
+        KvView kv = kv_view(l, pt);
+        cudaError_t e;
+        e = timed(0, s, [&] {
+            return launch_qkv_rope(x, g_attn, wqkv, B, H, Hq, Hkv, d, desc.rms_eps, desc.rope_theta, pos_dev, q, kv,
+                                   nullptr, s);
+        });
+        if (e != cudaSuccess) return cuda_fail(e, "qkv kernel");
+        e = timed(1, s, [&] {
+            return launch_attention(q, kv, nullptr, pos_dev, nullptr, B, Hq, Hkv, d, cfg.max_ctx, true,
+                                    fixed_ptr<float>(fx.attn_scratch), o, false, s);
+        });
+        if (e != cudaSuccess) return cuda_fail(e, "attention kernel");
+        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s); });
+        if (e != cudaSuccess) return cuda_fail(e, "o-proj kernel");
+        e = timed(3, s, [&] { return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s); });
+        if (e != cudaSuccess) return cuda_fail(e, "gate/up kernel");
+        e = timed(4, s, [&] { return launch_resid_gemv(a, wd, B, H, F, x, s); });
+        if (e != cudaSuccess) return cuda_fail(e, "down kernel");
+        return LOIP_OK;
+    }
+
+    // Prefill layer on Mc token rows held in the prefill workspace.
+    int prefill_layer(int l, int Mc, cudaStream_t s, int slot) {
+        const uint16_t* w = layer_weights(l, slot);
+        float* px = fixed_ptr<float>(fx.px);
+        uint16_t* py = fixed_ptr<uint16_t>(fx.py);
+        float* pq = fixed_ptr<float>(fx.pq);
+        uint16_t* po = fixed_ptr<uint16_t>(fx.po);
+        uint16_t* pa = fixed_ptr<uint16_t>(fx.pa);
+        const int32_t* pos = fixed_ptr<int32_t>(fx.positions);
+        const int32_t* req = fixed_ptr<int32_t>(fx.row_req);
+        const int64_t* pt = fixed_ptr<int64_t>(fx.page_table);
+        KvView kv = kv_view(l, pt);
+        cudaError_t e;
+        e = launch_rmsnorm_bf16(px, w + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s);
+        if (e == cudaSuccess)
+            e = launch_gemm_qkv_rope(py, w + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos, req, pq, kv, s);
+        if (e == cudaSuccess)
+            e = launch_attention(pq, kv, nullptr, pos, req, Mc, Hq, Hkv, d, cfg.max_ctx, false, nullptr, po, true, s);
+        if (e == cudaSuccess) e = launch_gemm_resid(po, w + lay.off_wo / 2, Mc, H, qd, px, s);
+        if (e == cudaSuccess) e = launch_rmsnorm_bf16(px, w + lay.off_g_mlp / 2, Mc, H, desc.rms_eps, py, s);
+        if (e == cudaSuccess) e = launch_gemm_swiglu(py, w + lay.off_wg / 2, w + lay.off_wu / 2, Mc, H, F, pa, s);
+        if (e == cudaSuccess) e = launch_gemm_resid(pa, w + lay.off_wd / 2, Mc, H, F, px, s);
+        if (e != cudaSuccess) return cuda_fail(e, "prefill kernel");
+        return LOIP_OK;
+    }
+
+    // Runs all layers once (decode or prefill pass) with the streaming ring.
+    template <class LayerFn>
+    int run_layers(LayerFn&& fn) {
+        const bool naive = cfg.mode == LOIP_MODE_NAIVE;
+        for (int l = 0; l < L; ++l) {
+            int slot = -1;
+            if (offloaded[l]) {
+                if (naive) {
+                    // conventional path: load when needed, compute waits
+                    slot = 0;
+                    cudaEventRecord(ev_reach, compute);
+                    cudaStreamWaitEvent(copy, ev_reach, 0);
+                    int rc = enqueue_copy(l, 0, copy);
+                    if (rc) return rc;
+                } else {
+                    slot = (int)(compute_seq % cfg.n_slots);
+                    if (off_order[compute_seq % off_order.size()] != l)
+                        return fail(LOIP_ERR_STATE, "slot ring out of order");
+                }
+                cudaError_t e = cudaStreamWaitEvent(compute, slot_full[slot], 0);
+                if (e != cudaSuccess) return cuda_fail(e, "compute wait");
+            }
+            int rc = fn(l, slot);
+            if (rc) return rc;
+            if (offloaded[l]) {
+                cudaError_t e = cudaEventRecord(slot_free[slot], compute);
+                if (e != cudaSuccess) return cuda_fail(e, "slot free event");
+                if (!naive) {
+                    ++compute_seq;
+                    rc = issue_next_copy();
+                    if (rc) return rc;
+                }
+            }
+        }
+        return LOIP_OK;
+    }
+
+    void collect_copy_time() {
+        double busy = 0;
+        while (!copy_events.empty()) {
+            auto pr = copy_events.front();
+            if (cudaEventQuery(pr.second) != cudaSuccess) break;
+            float ms = 0;
+            cudaEventElapsedTime(&ms, pr.first, pr.second);
+            busy += ms;
+            event_pool.push_back(pr.first);
+            event_pool.push_back(pr.second);
+            copy_events.pop_front();
+        }
+        st.copy_busy_ms = busy;
+    }
+
+    // ---- online re-planning (Eq. 6) -------------------------------------------
+    int demote_for_kv() {
+        // offload one more resident layer; its block becomes free
+        std::vector<uint8_t> mask = offloaded;
+        int victim = demote_one(L, mask.data());
+        if (victim < 0) return fail(LOIP_ERR_OOM, "KV cache does not fit even with every layer offloaded");
+        int rc = sync_all();
+        if (rc) return rc;
+        if (off_order.empty()) {
+            // the first offloaded layer also needs the slots
+            for (int k = 0; k < cfg.n_slots; ++k) {
+                int b = take_free_block();
+                if (b < 0) {
+                    // take resident layers until the slots fit
+                    std::vector<uint8_t> m2 = mask;
+                    int v2 = demote_one(L, m2.data());
+                    if (v2 < 0) return fail(LOIP_ERR_OOM, "no room for slots");
+                    int rc2 = demote_layer(v2);
+                    if (rc2) return rc2;
+                    mask = m2;
+                    b = take_free_block();
+                }
+                block_kind[b] = B_SLOT;
+                block_owner[b] = k;
+                slot_block[k] = b;
+            }
+        }
+        rc = demote_layer(victim);
+        if (rc) return rc;
+        rebuild_order();
+        st.n_replans++;
+        return prime_slots();
+    }
+
+    int demote_layer(int l) {
+        if (!host_layer[l]) {
+            cudaError_t e = cudaHostAlloc(&host_layer[l], lay.l_size, cudaHostAllocDefault);
+            if (e != cudaSuccess) {
+                host_layer[l] = nullptr;
+                return fail(LOIP_ERR_OOM, "pinned allocation for a demoted layer failed");
+            }
+            e = cudaMemcpy(host_layer[l], block_ptr(layer_block[l]), lay.l_size, cudaMemcpyDeviceToHost);
+            if (e != cudaSuccess) return cuda_fail(e, "demote copy");
+        }
+        int b = layer_block[l];
+        block_kind[b] = B_FREE;
+        block_owner[b] = -1;
+        layer_block[l] = -1;
+        offloaded[l] = 1;
+        return LOIP_OK;
+    }
+
+    uint64_t arena_used() const {
+        uint64_t used = fx.total + kv_region_bytes;
+        for (int b = 0; b < n_blocks; ++b)
+            if (block_kind[b] != B_FREE) used += block_bytes;
+        return used;
+    }
+};
+
+// ============================================================================
+// C ABI
+// ============================================================================
+#define CTX_GUARD(ctx)                                                             \
+    do {                                                                           \
+        if (!(ctx)) return LOIP_ERR_INVALID;                                       \
+        if ((ctx)->failed) return (ctx)->fail(LOIP_ERR_STATE, "context failed earlier: " + (ctx)->err); \
+    } while (0)
+
+extern "C" int loip_layer_layout(const loip_model_desc* desc, loip_layer_layout_t* out) {
+    if (!out || validate_desc(desc)) return LOIP_ERR_INVALID;
+    layout_of(desc, out);
+    return LOIP_OK;
+}
+
+extern "C" int loip_fixed_bytes(const loip_model_desc* desc, const loip_config* cfg, uint64_t* out) {
+    if (!out || !cfg || validate_desc(desc) || cfg->max_batch < 1 || cfg->max_batch > 8 || cfg->max_ctx < 1)
+        return LOIP_ERR_INVALID;
+    loip_config c = normalized(cfg);
+    *out = fixed_layout(desc, &c).total;
+    return LOIP_OK;
+}
+
+extern "C" const char* loip_last_error(const loip_ctx* ctx) {
+    return ctx ? ctx->err.c_str() : g_create_error.c_str();
+}
+
+extern "C" void loip_destroy(loip_ctx* ctx) {
+    if (!ctx) return;
+    if (ctx->compute) cudaStreamSynchronize(ctx->compute);
+    if (ctx->copy) cudaStreamSynchronize(ctx->copy);
+    for (void* p : ctx->host_layer)
+        if (p) cudaFreeHost(p);
+    if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
+    if (ctx->h_pt) cudaFreeHost(ctx->h_pt);
+    for (auto e : ctx->slot_full) cudaEventDestroy(e);
+    for (auto e : ctx->slot_free) cudaEventDestroy(e);
+    for (auto& pr : ctx->copy_events) {
+        cudaEventDestroy(pr.first);
+        cudaEventDestroy(pr.second);
+    }
+    for (auto& k : ctx->kernel_events) {
+        cudaEventDestroy(k.a);
+        cudaEventDestroy(k.b);
+    }
+    for (auto e : ctx->event_pool) cudaEventDestroy(e);
+    for (cudaEvent_t e : {ctx->ev_done, ctx->ev_step0, ctx->ev_step1, ctx->ev_reach, ctx->ev_stage})
+        if (e) cudaEventDestroy(e);
+    if (ctx->compute) cudaStreamDestroy(ctx->compute);
+    if (ctx->copy) cudaStreamDestroy(ctx->copy);
+    delete ctx;
+}
+
+extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_in, void* device_arena,
+                           uint64_t arena_bytes, loip_ctx** out) {
+    if (!out) return LOIP_ERR_INVALID;
+    *out = nullptr;
+    if (validate_desc(desc) || !cfg_in) {
+        g_create_error = "invalid model description";
+        return LOIP_ERR_INVALID;
+    }
+    loip_config cfg = normalized(cfg_in);
+    if (cfg.n_slots < 1 || cfg.n_slots > 3 || cfg.max_batch < 1 || cfg.max_batch > 8 || cfg.max_ctx < 1 ||
+        cfg.page_tokens != 64 || !device_arena || ((uintptr_t)device_arena % kAlign) ||
+        arena_bytes < cfg.device_budget_bytes || (cfg.mode != LOIP_MODE_OVERLAP && cfg.mode != LOIP_MODE_NAIVE)) {
+        g_create_error = "invalid configuration (slots 1..3, batch 1..8, page 64, arena >= budget, aligned)";
+        return LOIP_ERR_INVALID;
+    }
+    if (cfg.mode == LOIP_MODE_NAIVE) cfg.n_slots = 1;
+    loip_ctx* c = new loip_ctx();
+    c->desc = *desc;
+    c->cfg = cfg;
+    layout_of(desc, &c->lay);
+    c->L = desc->n_layers;
+    c->H = desc->hidden;
+    c->Hq = desc->n_heads;
+    c->Hkv = desc->n_kv_heads;
+    c->d = desc->head_dim;
+    c->F = desc->ffn;
+    c->V = desc->vocab;
+    c->qd = c->Hq * c->d;
+    c->kvd = c->Hkv * c->d;
+    c->arena = reinterpret_cast<char*>(device_arena);
+    c->budget = cfg.device_budget_bytes;
+    c->fx = fixed_layout(desc, &cfg);
+    c->layer_page_bytes = 2ull * c->Hkv * cfg.page_tokens * c->d * 2;
+    c->group_bytes = align_up(c->layer_page_bytes * c->L);
+    c->kv_tok_bytes = 2ull * c->kvd * 2 * c->L;
+    c->max_pages = (cfg.max_ctx + cfg.page_tokens - 1) / cfg.page_tokens;
+    c->block_bytes = align_up(c->lay.l_size);
+    if (c->group_bytes > c->block_bytes) {
+        g_create_error = "a KV page group is larger than a layer block";
+        delete c;
+        return LOIP_ERR_INVALID;
+    }
+    // KV region reserved up front
+    uint64_t kv_groups = cfg.kv_reserve_bytes ? (cfg.kv_reserve_bytes + c->group_bytes - 1) / c->group_bytes
+                                              : (uint64_t)cfg.max_batch * c->max_pages;
+    c->kv_region_off = c->fx.total;
+    c->kv_region_bytes = kv_groups * c->group_bytes;
+    c->blocks_off = align_up(c->kv_region_off + c->kv_region_bytes);
+    if (c->budget < c->blocks_off) {
+        g_create_error = "budget smaller than the fixed part and the KV reserve";
+        delete c;
+        return LOIP_ERR_INFEASIBLE;
+    }
+    c->n_blocks = (int)((c->budget - c->blocks_off) / c->block_bytes);
+    // plan (Algorithm 1 memory-first fill with the slot ring)
+    std::vector<uint64_t> lb(c->L, c->block_bytes);
+    std::vector<uint8_t> res(c->L);
+    loip_plan plan{};
+    plan.resident = res.data();
+    int rc = loip_plan_residency(desc, lb.data(), c->budget, c->kv_region_bytes, c->blocks_off - c->kv_region_bytes,
+                                 cfg.n_slots, cfg.hbm_Bps, cfg.link_Bps, &plan);
+    if (rc) {
+        g_create_error = "budget cannot hold the fixed part, the KV reserve and the slots";
+        delete c;
+        return rc;
+    }
+    c->offloaded.assign(c->L, 0);
+    c->layer_block.assign(c->L, -1);
+    c->block_kind.assign(c->n_blocks, B_FREE);
+    c->block_owner.assign(c->n_blocks, -1);
+    int nb = 0;
+    for (int l = 0; l < c->L; ++l) {
+        if (res[l]) {
+            c->layer_block[l] = nb;
+            c->block_kind[nb] = B_LAYER;
+            c->block_owner[nb] = l;
+            ++nb;
+        } else {
+            c->offloaded[l] = 1;
+        }
+    }
+    c->rebuild_order();
+    c->slot_block.assign(cfg.n_slots, -1);
+    if (!c->off_order.empty()) {
+        for (int k = 0; k < cfg.n_slots; ++k) {
+            if (nb >= c->n_blocks) {
+                g_create_error = "internal: slots do not fit";
+                delete c;
+                return LOIP_ERR_INFEASIBLE;
+            }
+            c->slot_block[k] = nb;
+            c->block_kind[nb] = B_SLOT;
+            c->block_owner[nb] = k;
+            ++nb;
+        }
+    }
+    for (uint64_t i = 0; i < kv_groups; ++i)
+        c->free_groups.push_back((int64_t)(c->kv_region_off + (kv_groups - 1 - i) * c->group_bytes));
+    c->kv_groups_total = kv_groups;
+    c->reqs.resize(cfg.max_batch);
+    c->host_layer.assign(c->L, nullptr);
+
+    cudaError_t e;
+    e = cudaStreamCreateWithFlags(&c->compute, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->copy, cudaStreamNonBlocking);
+    c->slot_full.resize(cfg.n_slots);
+    c->slot_free.resize(cfg.n_slots);
+    for (int k = 0; k < cfg.n_slots && e == cudaSuccess; ++k) {
+        e = cudaEventCreateWithFlags(&c->slot_full[k], cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->slot_free[k], cudaEventDisableTiming);
+    }
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_done, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_reach, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_stage, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreate(&c->ev_step0);
+    if (e == cudaSuccess) e = cudaEventCreate(&c->ev_step1);
+    c->h_stage_ints = 4 * (size_t)std::max(cfg.max_batch, cfg.max_prefill_tokens) + 64;
+    if (e == cudaSuccess) e = cudaHostAlloc(&c->h_stage, c->h_stage_ints * 4, cudaHostAllocDefault);
+    if (e == cudaSuccess) e = cudaHostAlloc(&c->h_pt, (size_t)cfg.max_batch * c->max_pages * 8, cudaHostAllocDefault);
+    if (e != cudaSuccess) {
+        g_create_error = std::string("CUDA setup failed: ") + cudaGetErrorString(e);
+        loip_destroy(c);
+        return LOIP_ERR_CUDA;
+    }
+    c->st.n_resident = c->L - (int)c->off_order.size();
+    c->st.n_offloaded = (int)c->off_order.size();
+    *out = c;
+    return LOIP_OK;
+}
+
+extern "C" int loip_get_plan(const loip_ctx* ctx, loip_plan* out) {
+    if (!ctx || !out || !out->resident) return LOIP_ERR_INVALID;
+    out->n_layers = ctx->L;
+    out->n_offloaded = (int)ctx->off_order.size();
+    out->n_resident = ctx->L - out->n_offloaded;
+    for (int l = 0; l < ctx->L; ++l) out->resident[l] = ctx->offloaded[l] ? 0 : 1;
+    std::vector<double> comp(ctx->L), load(ctx->L);
+    for (int l = 0; l < ctx->L; ++l) {
+        comp[l] = (double)ctx->block_bytes / ctx->cfg.hbm_Bps;
+        load[l] = (double)ctx->block_bytes / ctx->cfg.link_Bps;
+    }
+    out->pred_step_s = simulate_step(comp, load, ctx->offloaded.data(), ctx->cfg.n_slots, 4);
+    out->eq1_step_s = eq1_single_device(comp, load, ctx->offloaded.data());
+    out->pred_copy_s = out->n_offloaded * load[0];
+    out->pred_compute_s = ctx->L * comp[0];
+    uint64_t used = ctx->arena_used();
+    out->left_bytes = ctx->budget > used ? ctx->budget - used : 0;
+    return LOIP_OK;
+}
+
+static int write_layer_generated(loip_ctx* c, char* dst, int l, uint64_t seed) {
+    const uint64_t H = c->H, F = c->F, qd = c->qd, kvd = c->kvd;
+    auto T = [&](int which) { return (uint32_t)(16 + 16 * l + which); };
+    uint16_t* base = reinterpret_cast<uint16_t*>(dst);
+    const loip_layer_layout_t& y = c->lay;
+    cudaStream_t s = c->compute;
+    cudaError_t e = cudaSuccess;
+    auto gen = [&](uint64_t off_bytes, uint64_t n, uint32_t tid, int kind) {
+        if (e == cudaSuccess) e = launch_generate(base + off_bytes / 2, n, 0, seed, tid, kind, s);
+    };
+    gen(y.off_g_attn, H, T(0), 1);
+    gen(y.off_wqkv, qd * H, T(1), 0);
+    gen(y.off_wqkv + qd * H * 2, kvd * H, T(2), 0);
+    gen(y.off_wqkv + (qd + kvd) * H * 2, kvd * H, T(3), 0);
+    gen(y.off_wo, H * qd, T(4), 0);
+    gen(y.off_g_mlp, H, T(5), 1);
+    gen(y.off_wg, F * H, T(6), 0);
+    gen(y.off_wu, F * H, T(7), 0);
+    gen(y.off_wd, H * F, T(8), 0);
+    if (e != cudaSuccess) return c->cuda_fail(e, "generator kernel");
+    return LOIP_OK;
+}
+
+extern "C" int loip_load_weights_generated(loip_ctx* c, uint64_t seed) {
+    CTX_GUARD(c);
+    int rc = c->sync_all();
+    if (rc) return rc;
+    cudaError_t e = launch_generate(c->fixed_ptr<uint16_t>(c->fx.embed), (uint64_t)c->V * c->H, 0, seed, 1, 0,
+                                    c->compute);
+    if (e == cudaSuccess)
+        e = launch_generate(c->fixed_ptr<uint16_t>(c->fx.lm_head), (uint64_t)c->V * c->H, 0, seed, 2, 0, c->compute);
+    if (e == cudaSuccess)
+        e = launch_generate(c->fixed_ptr<uint16_t>(c->fx.g_final), (uint64_t)c->H, 0, seed, 3, 1, c->compute);
+    if (e != cudaSuccess) return c->cuda_fail(e, "generator kernel");
+    for (int l = 0; l < c->L; ++l) {
+        if (c->layer_block[l] >= 0) {
+            rc = write_layer_generated(c, c->block_ptr(c->layer_block[l]), l, seed);
+            if (rc) return rc;
+        } else {
+            if (!c->host_layer[l]) {
+                e = cudaHostAlloc(&c->host_layer[l], c->lay.l_size, cudaHostAllocDefault);
+                if (e != cudaSuccess) {
+                    c->host_layer[l] = nullptr;
+                    return c->fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
+                }
+            }
+            char* tmp = c->slot_ptr(0);
+            rc = write_layer_generated(c, tmp, l, seed);
+            if (rc) return rc;
+            e = cudaMemcpyAsync(c->host_layer[l], tmp, c->lay.l_size, cudaMemcpyDeviceToHost, c->compute);
+            if (e != cudaSuccess) return c->cuda_fail(e, "host pool copy");
+        }
+    }
+    rc = c->sync_all();
+    if (rc) return rc;
+    c->weights_loaded = true;
+    rc = c->prime_slots();
+    if (rc) return rc;
+    return c->sync_all();
+}
+
+extern "C" int loip_load_layer(loip_ctx* c, int32_t layer, const void* host_blob, uint64_t bytes) {
+    CTX_GUARD(c);
+    if (layer < 0 || layer >= c->L || !host_blob || bytes != c->lay.l_size)
+        return c->fail(LOIP_ERR_INVALID, "layer index or blob size");
+    int rc = c->sync_all();
+    if (rc) return rc;
+    cudaError_t e;
+    if (c->layer_block[layer] >= 0) {
+        e = cudaMemcpy(c->block_ptr(c->layer_block[layer]), host_blob, bytes, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) return c->cuda_fail(e, "layer upload");
+    } else {
+        if (!c->host_layer[layer]) {
+            e = cudaHostAlloc(&c->host_layer[layer], bytes, cudaHostAllocDefault);
+            if (e != cudaSuccess) {
+                c->host_layer[layer] = nullptr;
+                return c->fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
+            }
+        }
+        memcpy(c->host_layer[layer], host_blob, bytes);
+    }
+    c->weights_loaded = true;
+    rc = c->prime_slots();
+    return rc ? rc : c->sync_all();
+}
+
+extern "C" int loip_load_globals(loip_ctx* c, const uint16_t* embed, const uint16_t* lm_head, const uint16_t* g_final) {
+    CTX_GUARD(c);
+    if (!embed || !lm_head || !g_final) return c->fail(LOIP_ERR_INVALID, "null pointer");
+    size_t vh = (size_t)c->V * c->H * 2;
+    cudaError_t e = cudaMemcpy(c->arena + c->fx.embed, embed, vh, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->arena + c->fx.lm_head, lm_head, vh, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->arena + c->fx.g_final, g_final, (size_t)c->H * 2, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return c->cuda_fail(e, "globals upload");
+    c->weights_loaded = true;
+    return LOIP_OK;
+}
+
+extern "C" int loip_stream_layer(loip_ctx* c, int32_t layer, int32_t slot, void* copy_stream) {
+    CTX_GUARD(c);
+    if (layer < 0 || layer >= c->L || !c->offloaded[layer] || slot < 0 || slot >= c->cfg.n_slots ||
+        c->off_order.empty() || !c->host_layer[layer])
+        return c->fail(LOIP_ERR_INVALID, "layer is not offloaded or slot out of range");
+    cudaStream_t s = copy_stream ? reinterpret_cast<cudaStream_t>(copy_stream) : c->copy;
+    return c->enqueue_copy(layer, slot, s);
+}
+
+extern "C" int loip_set_batch(loip_ctx* c, int32_t batch, const int32_t* ctx_lens) {
+    CTX_GUARD(c);
+    if (batch < 1 || batch > c->cfg.max_batch || !ctx_lens) return c->fail(LOIP_ERR_INVALID, "batch size");
+    for (int b = 0; b < batch; ++b)
+        if (ctx_lens[b] < 0 || ctx_lens[b] >= c->cfg.max_ctx) return c->fail(LOIP_ERR_INVALID, "context length");
+    for (int b = 0; b < batch; ++b) {
+        int rc = c->ensure_pages(b, ctx_lens[b]);
+        if (rc) return rc;
+        c->reqs[b].len = ctx_lens[b];
+    }
+    c->active_batch = batch;
+    c->pos_dirty = true;
+    return LOIP_OK;
+}
+
+extern "C" int loip_layer_forward(loip_ctx* c, int32_t layer, int32_t slot, float* hidden, const int32_t* positions,
+                                  int32_t batch, void* compute_stream) {
+    CTX_GUARD(c);
+    if (layer < 0 || layer >= c->L || !hidden || !positions || batch < 1 || batch > c->cfg.max_batch)
+        return c->fail(LOIP_ERR_INVALID, "layer_forward arguments");
+    if (c->offloaded[layer] && (slot < 0 || slot >= c->cfg.n_slots))
+        return c->fail(LOIP_ERR_INVALID, "offloaded layer needs its slot");
+    cudaStream_t s = compute_stream ? reinterpret_cast<cudaStream_t>(compute_stream) : c->compute;
+    int rc = c->upload_page_table(s);
+    if (rc) return rc;
+    float* x = c->fixed_ptr<float>(c->fx.x);
+    cudaError_t e = cudaMemcpyAsync(x, hidden, (size_t)batch * c->H * 4, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return c->cuda_fail(e, "hidden copy");
+    if (c->offloaded[layer]) {
+        e = cudaStreamWaitEvent(s, c->slot_full[slot], 0);
+        if (e != cudaSuccess) return c->cuda_fail(e, "slot wait");
+    }
+    rc = c->decode_layer(layer, batch, positions, s, slot);
+    if (rc) return rc;
+    if (c->offloaded[layer]) cudaEventRecord(c->slot_free[slot], s);
+    e = cudaMemcpyAsync(hidden, x, (size_t)batch * c->H * 4, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return c->cuda_fail(e, "hidden copy");
+    return LOIP_OK;
+}
+
+// One decode step; tokens already on the device (d_tokens), results on device.
+static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int32_t* d_out, float* out_hidden) {
+    if (!c->weights_loaded) return c->fail(LOIP_ERR_STATE, "weights not loaded");
+    if (B < 1 || B > c->cfg.max_batch) return c->fail(LOIP_ERR_INVALID, "batch size");
+    if (B != c->active_batch) {
+        // implicit batch: requests 0..B-1 keep their current lengths
+        c->active_batch = B;
+        c->pos_dirty = true;
+    }
+    for (int b = 0; b < B; ++b) {
+        if (c->reqs[b].len + 1 > c->cfg.max_ctx) return c->fail(LOIP_ERR_INVALID, "context full");
+        int rc = c->ensure_pages(b, c->reqs[b].len + 1);
+        if (rc) return rc;
+    }
+    cudaStream_t s = c->compute;
+    int rc = c->upload_page_table(s);
+    if (rc) return rc;
+    rc = c->upload_positions(B, s);
+    if (rc) return rc;
+    int32_t* pos = c->fixed_ptr<int32_t>(c->fx.dec_pos);
+    cudaError_t e;
+    cudaEventRecord(c->ev_step0, s);
+    float* x = c->fixed_ptr<float>(c->fx.x);
+    e = launch_embed(c->fixed_ptr<uint16_t>(c->fx.embed), d_tokens, B, c->H, c->V, x, s);
+    if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
+    rc = c->run_layers([&](int l, int slot) { return c->decode_layer(l, B, pos, s, slot); });
+    if (rc) return rc;
+    e = c->timed(5, s, [&] {
+        return launch_lm_head(x, c->fixed_ptr<uint16_t>(c->fx.g_final), c->fixed_ptr<uint16_t>(c->fx.lm_head), B, c->H,
+                              c->V, c->desc.rms_eps, out_hidden ? out_hidden : c->fixed_ptr<float>(c->fx.z),
+                              c->fixed_ptr<float>(c->fx.logits), d_out, c->fixed_ptr<void>(c->fx.lm_scratch), s);
+    });
+    if (e != cudaSuccess) return c->cuda_fail(e, "lm head kernel");
+    e = launch_advance(pos, B, s);
+    if (e != cudaSuccess) return c->cuda_fail(e, "position advance");
+    cudaEventRecord(c->ev_step1, s);
+    for (int b = 0; b < B; ++b) c->reqs[b].len += 1;
+    c->st.steps += 1;
+    c->st.tokens += B;
+    return LOIP_OK;
+}
+
+extern "C" int loip_decode_step(loip_ctx* c, const int32_t* tokens, int32_t batch, int32_t* out_tokens,
+                                float* out_hidden) {
+    CTX_GUARD(c);
+    if (!tokens || !out_tokens || batch < 1 || batch > c->cfg.max_batch)
+        return c->fail(LOIP_ERR_INVALID, "decode_step arguments");
+    for (int b = 0; b < batch; ++b)
+        if (tokens[b] < 0 || tokens[b] >= c->V) return c->fail(LOIP_ERR_INVALID, "token id out of range");
+    auto t0 = std::chrono::steady_clock::now();
+    int32_t* hin = c->h_stage;
+    int32_t* hout = c->h_stage + c->h_stage_ints / 4;
+    int rc0 = c->wait_event(c->ev_stage);
+    if (rc0) return rc0;
+    memcpy(hin, tokens, (size_t)batch * 4);
+    int32_t* d_tok = c->fixed_ptr<int32_t>(c->fx.tokens);
+    int32_t* d_out = c->fixed_ptr<int32_t>(c->fx.out_tokens);
+    cudaError_t e = cudaMemcpyAsync(d_tok, hin, (size_t)batch * 4, cudaMemcpyHostToDevice, c->compute);
+    if (e != cudaSuccess) return c->cuda_fail(e, "token upload");
+    cudaEventRecord(c->ev_stage, c->compute);
+    int rc = decode_step_enqueue(c, d_tok, batch, d_out, out_hidden);
+    if (rc) return rc;
+    e = cudaMemcpyAsync(hout, d_out, (size_t)batch * 4, cudaMemcpyDeviceToHost, c->compute);
+    if (e != cudaSuccess) return c->cuda_fail(e, "token download");
+    e = cudaEventRecord(c->ev_done, c->compute);
+    if (e != cudaSuccess) return c->cuda_fail(e, "event record");
+    rc = c->wait_event(c->ev_done);
+    if (rc) return rc;
+    memcpy(out_tokens, hout, (size_t)batch * 4);
+    c->collect_kernel_times();
+    float ms = 0;
+    cudaEventElapsedTime(&ms, c->ev_step0, c->ev_step1);
+    c->st.compute_ms = ms;
+    c->collect_copy_time();
+    c->st.last_step_ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
+    return LOIP_OK;
+}
+
+extern "C" int loip_decode_step_device(loip_ctx* c, const int32_t* tokens_dev, int32_t batch, int32_t* out_tokens_dev,
+                                       float* out_hidden) {
+    CTX_GUARD(c);
+    if (!tokens_dev || !out_tokens_dev) return c->fail(LOIP_ERR_INVALID, "null pointer");
+    int rc = decode_step_enqueue(c, tokens_dev, batch, out_tokens_dev, out_hidden);
+    if (rc) return rc;
+    c->collect_copy_time();
+    c->collect_kernel_times();
+    return LOIP_OK;
+}
+
+extern "C" int loip_prefill(loip_ctx* c, const int32_t* tokens, const int32_t* prompt_lens, int32_t n_prompts,
+                            int32_t* out_tokens, float* out_hidden) {
+    CTX_GUARD(c);
+    if (!tokens || !prompt_lens || !out_tokens || n_prompts < 1 || n_prompts > c->cfg.max_batch)
+        return c->fail(LOIP_ERR_INVALID, "prefill arguments");
+    if (!c->weights_loaded) return c->fail(LOIP_ERR_STATE, "weights not loaded");
+    int64_t M = 0;
+    for (int i = 0; i < n_prompts; ++i) {
+        if (prompt_lens[i] < 1 || prompt_lens[i] > c->cfg.max_ctx) return c->fail(LOIP_ERR_INVALID, "prompt length");
+        M += prompt_lens[i];
+    }
+    for (int64_t t = 0; t < M; ++t)
+        if (tokens[t] < 0 || tokens[t] >= c->V) return c->fail(LOIP_ERR_INVALID, "token id out of range");
+    auto t0 = std::chrono::steady_clock::now();
+    int rc = c->sync_all();
+    if (rc) return rc;
+    for (int i = 0; i < n_prompts; ++i) {
+        c->release_pages(i);
+        rc = c->ensure_pages(i, prompt_lens[i]);
+        if (rc) return rc;
+    }
+    cudaStream_t s = c->compute;
+    rc = c->upload_page_table(s);
+    if (rc) return rc;
+    const int Mp = c->cfg.max_prefill_tokens;
+    // per-token request and position
+    std::vector<int32_t> req_of(M), pos_of(M);
+    std::vector<int32_t> last_row(n_prompts);
+    {
+        int64_t t = 0;
+        for (int i = 0; i < n_prompts; ++i)
+            for (int p = 0; p < prompt_lens[i]; ++p, ++t) {
+                req_of[t] = i;
+                pos_of[t] = p;
+                if (p == prompt_lens[i] - 1) last_row[i] = (int32_t)t;
+            }
+    }
+    float* x = c->fixed_ptr<float>(c->fx.x);
+    cudaEventRecord(c->ev_step0, s);
+    for (int64_t c0 = 0; c0 < M; c0 += Mp) {
+        const int Mc = (int)std::min<int64_t>(Mp, M - c0);
+        int32_t* h = c->h_stage;
+        // staging: tokens | positions | requests
+        rc = c->wait_event(c->ev_stage);  // previous chunk's uploads have been consumed
+        if (rc) return rc;
+        memcpy(h, tokens + c0, (size_t)Mc * 4);
+        memcpy(h + Mc, pos_of.data() + c0, (size_t)Mc * 4);
+        memcpy(h + 2 * Mc, req_of.data() + c0, (size_t)Mc * 4);
+        cudaError_t e = cudaMemcpyAsync(c->arena + c->fx.tokens, h, (size_t)Mc * 4, cudaMemcpyHostToDevice, s);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(c->arena + c->fx.positions, h + Mc, (size_t)Mc * 4, cudaMemcpyHostToDevice, s);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(c->arena + c->fx.row_req, h + 2 * Mc, (size_t)Mc * 4, cudaMemcpyHostToDevice, s);
+        if (e != cudaSuccess) return c->cuda_fail(e, "prefill upload");
+        cudaEventRecord(c->ev_stage, s);
+        e = launch_embed(c->fixed_ptr<uint16_t>(c->fx.embed), c->fixed_ptr<int32_t>(c->fx.tokens), Mc, c->H, c->V,
+                         c->fixed_ptr<float>(c->fx.px), s);
+        if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
+        rc = c->run_layers([&](int l, int slot) { return c->prefill_layer(l, Mc, s, slot); });
+        if (rc) return rc;
+        // final rows of prompts ending in this chunk -> decode activations
+        for (int i = 0; i < n_prompts; ++i) {
+            if (last_row[i] < c0 || last_row[i] >= c0 + Mc) continue;
+            e = cudaMemcpyAsync(x + (size_t)i * c->H, c->fixed_ptr<float>(c->fx.px) + (size_t)(last_row[i] - c0) * c->H,
+                                (size_t)c->H * 4, cudaMemcpyDeviceToDevice, s);
+            if (e != cudaSuccess) return c->cuda_fail(e, "row copy");
+        }
+    }
+    int32_t* d_out = c->fixed_ptr<int32_t>(c->fx.out_tokens);
+    cudaError_t e = launch_lm_head(x, c->fixed_ptr<uint16_t>(c->fx.g_final), c->fixed_ptr<uint16_t>(c->fx.lm_head),
+                                   n_prompts, c->H, c->V, c->desc.rms_eps,
+                                   out_hidden ? out_hidden : c->fixed_ptr<float>(c->fx.z),
+                                   c->fixed_ptr<float>(c->fx.logits), d_out, c->fixed_ptr<void>(c->fx.lm_scratch), s);
+    if (e != cudaSuccess) return c->cuda_fail(e, "lm head kernel");
+    cudaEventRecord(c->ev_step1, s);
+    int32_t* hout = c->h_stage + c->h_stage_ints / 4;
+    e = cudaMemcpyAsync(hout, d_out, (size_t)n_prompts * 4, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return c->cuda_fail(e, "token download");
+    cudaEventRecord(c->ev_done, s);
+    rc = c->wait_event(c->ev_done);
+    if (rc) return rc;
+    memcpy(out_tokens, hout, (size_t)n_prompts * 4);
+    for (int i = 0; i < n_prompts; ++i) c->reqs[i].len = prompt_lens[i];
+    c->active_batch = n_prompts;
+    c->pos_dirty = true;
+    float ms = 0;
+    cudaEventElapsedTime(&ms, c->ev_step0, c->ev_step1);
+    c->st.compute_ms = ms;
+    c->collect_copy_time();
+    c->st.last_step_ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
+    return LOIP_OK;
+}
+
+extern "C" int loip_replan(loip_ctx* c, int32_t lookahead_tokens) {
+    CTX_GUARD(c);
+    if (lookahead_tokens < 0) return c->fail(LOIP_ERR_INVALID, "lookahead");
+    // pages the active requests need for the lookahead
+    uint64_t need = 0;
+    for (int b = 0; b < c->active_batch; ++b) {
+        int tokens = std::min(c->reqs[b].len + lookahead_tokens, c->cfg.max_ctx);
+        int pages = (tokens + c->cfg.page_tokens - 1) / c->cfg.page_tokens;
+        need += (uint64_t)std::max(0, pages - (int)c->reqs[b].pages.size());
+    }
+    while (c->free_groups.size() < need) {
+        if (c->grow_kv() >= 0) continue;
+        int rc = c->demote_for_kv();
+        if (rc) return rc;
+    }
+    return LOIP_OK;
+}
+
+extern "C" int loip_get_stats(const loip_ctx* c, loip_stats* out) {
+    if (!c || !out) return LOIP_ERR_INVALID;
+    *out = c->st;
+    out->n_offloaded = (int)c->off_order.size();
+    out->n_resident = c->L - out->n_offloaded;
+    uint64_t toks = 0;
+    uint64_t pages = 0;
+    for (auto& r : c->reqs) {
+        toks += r.len;
+        pages += r.pages.size();
+    }
+    out->kv_tokens = toks;
+    out->kv_bytes = pages * c->group_bytes;
+    out->arena_used = c->arena_used();
+    return LOIP_OK;
+}
+
+extern "C" int loip_synchronize(loip_ctx* c) {
+    if (!c) return LOIP_ERR_INVALID;
+    int rc = c->sync_all();
+    c->collect_copy_time();
+    c->collect_kernel_times();
+    return rc;
+}
+
+extern "C" int loip_set_kernel_timing(loip_ctx* c, int32_t enable) {
+    CTX_GUARD(c);
+    int rc = c->sync_all();
+    if (rc) return rc;
+    c->collect_kernel_times();
+    for (int i = 0; i < 6; ++i) {
+        c->st.kernel_ms[i] = 0;
+        c->st.kernel_launches[i] = 0;
+    }
+    c->ktiming = enable != 0;
+    return LOIP_OK;
+}
+
+extern "C" void* loip_compute_stream(loip_ctx* c) { return c ? (void*)c->compute : nullptr; }
+extern "C" void* loip_copy_stream(loip_ctx* c) { return c ? (void*)c->copy : nullptr; }
+
+// ============================================================================
+// Kernel-level entry points
+// ============================================================================
+static bool al16(const void* p) { return ((uintptr_t)p & 15) == 0; }
+static int cerr(cudaError_t e) { return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA; }
+
+extern "C" int loip_k_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id,
+                               int32_t kind, void* stream) {
+    if ((!out && n) || (kind != 0 && kind != 1) || first + n > (1ull << 40)) return LOIP_ERR_INVALID;
+    return cerr(launch_generate(out, n, first, seed, tensor_id, kind, (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_embed(const uint16_t* embed, const int32_t* tokens, int32_t B, int32_t H, float* x,
+                            void* stream) {
+    if (!embed || !tokens || !x || B < 1 || H < 1) return LOIP_ERR_INVALID;
+    return cerr(launch_embed(embed, tokens, B, H, 1 << 30, x, (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int32_t B, int32_t H,
+                               int32_t Hq, int32_t Hkv, int32_t d, float eps, float theta, const int32_t* positions,
+                               float* q_out, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
+                               int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, void* stream) {
+    if (!x || !g || !wqkv || !positions || !q_out || !kv_base || !page_offsets || B < 1 || B > 8 || H % 8 ||
+        (d != 64 && d != 128) || Hq % Hkv || page_tokens < 1 || !al16(wqkv) || !al16(x))
+        return LOIP_ERR_INVALID;
+    KvView kv{(char*)kv_base, page_offsets, max_pages, page_tokens, layer, layer_page_bytes};
+    return cerr(launch_qkv_rope(x, g, wqkv, B, H, Hq, Hkv, d, eps, theta, positions, q_out, kv, nullptr,
+                                (cudaStream_t)stream));
+}
+
+extern "C" uint64_t loip_k_attention_scratch_floats(int32_t B, int32_t Hq, int32_t d, int32_t max_ctx,
+                                                    int32_t page_tokens) {
+    if (B < 1 || Hq < 1 || d < 1 || max_ctx < 1 || page_tokens < 1) return 0;
+    return attention_scratch_floats(B, Hq, d, max_ctx, page_tokens);
+}
+
+extern "C" int loip_k_attention(const float* q, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
+                                const int32_t* ctx_lens, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
+                                int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx,
+                                float* scratch, float* o, void* stream) {
+    if (!q || !kv_base || !page_offsets || !ctx_lens || !scratch || !o || B < 1 || (d != 64 && d != 128) ||
+        Hq % Hkv || max_ctx < 1 || page_tokens < 1 || (int64_t)max_pages * page_tokens < max_ctx)
+        return LOIP_ERR_INVALID;
+    KvView kv{(char*)kv_base, page_offsets, max_pages, page_tokens, layer, layer_page_bytes};
+    return cerr(launch_attention(q, kv, ctx_lens, nullptr, nullptr, B, Hq, Hkv, d, max_ctx, true, scratch, o, false,
+                                 (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x,
+                            void* stream) {
+    if (!o || !wo || !x || B < 1 || B > 8 || K % 8 || H < 1 || !al16(wo)) return LOIP_ERR_INVALID;
+    return cerr(launch_resid_gemv(o, wo, B, H, K, x, (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int32_t B,
+                              int32_t H, int32_t F, float eps, float* a, void* stream) {
+    if (!x || !g || !wg || !wu || !a || B < 1 || B > 8 || H % 8 || F < 1 || !al16(wg) || !al16(wu))
+        return LOIP_ERR_INVALID;
+    return cerr(launch_gate_up(x, g, wg, wu, B, H, F, eps, a, (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_down(const float* a, const uint16_t* wd, int32_t B, int32_t H, int32_t F, float* x,
+                           void* stream) {
+    if (!a || !wd || !x || B < 1 || B > 8 || F % 8 || H < 1 || !al16(wd)) return LOIP_ERR_INVALID;
+    return cerr(launch_resid_gemv(a, wd, B, H, F, x, (cudaStream_t)stream));
+}
+
+extern "C" uint64_t loip_k_lm_head_scratch_bytes(int32_t B, int32_t V) {
+    if (B < 1 || V < 1) return 0;
+    return lm_head_scratch_bytes(B, V);
+}
+
+extern "C" int loip_k_lm_head(const float* x, const uint16_t* g_final, const uint16_t* lm_head, int32_t B, int32_t H,
+                              int32_t V, float eps, float* z, float* logits, int32_t* tokens, void* scratch,
+                              void* stream) {
+    if (!x || !g_final || !lm_head || !tokens || !scratch || B < 1 || B > 8 || H % 8 || V < 1 || !al16(lm_head))
+        return LOIP_ERR_INVALID;
+    return cerr(launch_lm_head(x, g_final, lm_head, B, H, V, eps, z, logits, tokens, scratch, (cudaStream_t)stream));
+}

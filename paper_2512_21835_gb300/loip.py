@@ -1,0 +1,351 @@
+"""Python binding of libloip (include/loip.h): argument marshalling only.
+
+Every step of the decoder runs in the library's CUDA kernels; this module
+turns torch tensors / numpy arrays into pointers and status codes into
+exceptions.  It refuses to load without the compiled library -- there is no
+fallback path.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libloip.so")
+
+OK, ERR_INVALID, ERR_OOM, ERR_INFEASIBLE, ERR_CUDA, ERR_TIMEOUT, ERR_STATE = range(7)
+MODE_OVERLAP, MODE_NAIVE = 0, 1
+_NAMES = {1: "INVALID", 2: "OOM", 3: "INFEASIBLE", 4: "CUDA", 5: "TIMEOUT", 6: "STATE"}
+
+
+class LoipError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"LOIP_ERR_{_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+class ModelDesc(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("hidden", C.c_int32), ("n_heads", C.c_int32), ("n_kv_heads", C.c_int32),
+                ("head_dim", C.c_int32), ("ffn", C.c_int32), ("vocab", C.c_int32), ("rms_eps", C.c_float),
+                ("rope_theta", C.c_float)]
+
+
+class Config(C.Structure):
+    _fields_ = [("device_budget_bytes", C.c_uint64), ("n_slots", C.c_int32), ("page_tokens", C.c_int32),
+                ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("use_graphs", C.c_int32), ("mode", C.c_int32),
+                ("timeout_ms", C.c_uint32), ("hbm_Bps", C.c_double), ("link_Bps", C.c_double),
+                ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32)]
+
+
+class LayerLayout(C.Structure):
+    _fields_ = [(n, C.c_uint64) for n in ("off_g_attn", "off_wqkv", "off_wo", "off_g_mlp", "off_wg", "off_wu",
+                                          "off_wd", "l_size", "mha_bytes", "mlp_bytes")]
+
+
+class Plan(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("n_resident", C.c_int32), ("n_offloaded", C.c_int32),
+                ("resident", C.POINTER(C.c_uint8)), ("pred_step_s", C.c_double), ("pred_copy_s", C.c_double),
+                ("pred_compute_s", C.c_double), ("eq1_step_s", C.c_double), ("left_bytes", C.c_uint64)]
+
+
+class Stats(C.Structure):
+    _fields_ = [("steps", C.c_uint64), ("tokens", C.c_uint64), ("h2d_weight_bytes", C.c_uint64),
+                ("last_step_ms", C.c_double), ("copy_busy_ms", C.c_double), ("compute_ms", C.c_double),
+                ("n_resident", C.c_int32), ("n_offloaded", C.c_int32), ("n_replans", C.c_int32),
+                ("kv_tokens", C.c_uint64), ("kv_bytes", C.c_uint64), ("arena_used", C.c_uint64),
+                ("kernel_ms", C.c_double * 6), ("kernel_launches", C.c_uint64 * 6)]
+
+
+P, U64, I32, U32, F32, F64, VP = C.c_void_p, C.c_uint64, C.c_int32, C.c_uint32, C.c_float, C.c_double, C.c_void_p
+_SIGS = {
+    "loip_layer_layout": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(LayerLayout)]),
+    "loip_plan_residency": (C.c_int, [C.POINTER(ModelDesc), P, U64, U64, U64, I32, F64, F64, C.POINTER(Plan)]),
+    "loip_kv_threshold": (C.c_int, [U64, U64, C.POINTER(C.c_uint64)]),
+    "loip_fixed_bytes": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(Config), C.POINTER(C.c_uint64)]),
+    "loip_create": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(Config), P, U64, C.POINTER(C.c_void_p)]),
+    "loip_destroy": (None, [P]),
+    "loip_last_error": (C.c_char_p, [P]),
+    "loip_load_weights_generated": (C.c_int, [P, U64]),
+    "loip_load_layer": (C.c_int, [P, I32, P, U64]),
+    "loip_load_globals": (C.c_int, [P, P, P, P]),
+    "loip_get_plan": (C.c_int, [P, C.POINTER(Plan)]),
+    "loip_stream_layer": (C.c_int, [P, I32, I32, P]),
+    "loip_layer_forward": (C.c_int, [P, I32, I32, P, P, I32, P]),
+    "loip_set_batch": (C.c_int, [P, I32, P]),
+    "loip_decode_step": (C.c_int, [P, P, I32, P, P]),
+    "loip_decode_step_device": (C.c_int, [P, P, I32, P, P]),
+    "loip_prefill": (C.c_int, [P, P, P, I32, P, P]),
+    "loip_replan": (C.c_int, [P, I32]),
+    "loip_get_stats": (C.c_int, [P, C.POINTER(Stats)]),
+    "loip_synchronize": (C.c_int, [P]),
+    "loip_set_kernel_timing": (C.c_int, [P, I32]),
+    "loip_compute_stream": (C.c_void_p, [P]),
+    "loip_copy_stream": (C.c_void_p, [P]),
+    "loip_k_generate": (C.c_int, [P, U64, U64, U64, U32, I32, P]),
+    "loip_k_embed": (C.c_int, [P, P, I32, I32, P, P]),
+    "loip_k_qkv_rope": (C.c_int, [P, P, P, I32, I32, I32, I32, I32, F32, F32, P, P, P, P, I32, I32, I32, U64, P]),
+    "loip_k_attention": (C.c_int, [P, P, P, I32, P, I32, I32, I32, I32, I32, I32, U64, I32, P, P, P]),
+    "loip_k_attention_scratch_floats": (C.c_uint64, [I32, I32, I32, I32, I32]),
+    "loip_k_oproj": (C.c_int, [P, P, I32, I32, I32, P, P]),
+    "loip_k_gate_up": (C.c_int, [P, P, P, P, I32, I32, I32, F32, P, P]),
+    "loip_k_down": (C.c_int, [P, P, I32, I32, I32, P, P]),
+    "loip_k_lm_head": (C.c_int, [P, P, P, I32, I32, I32, F32, P, P, P, P, P]),
+    "loip_k_lm_head_scratch_bytes": (C.c_uint64, [I32, I32]),
+}
+
+_lib = None
+
+
+def lib():
+    """The loaded library.  Raises if it has not been built: there is no other path."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; "
+                              "g.build()'` (nvcc, sm_103a)")
+        L = C.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def exported_names():
+    return list(_SIGS)
+
+
+def _ptr(x):
+    """Pointer of a torch tensor, numpy array, int or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if isinstance(x, np.ndarray):
+        assert x.flags["C_CONTIGUOUS"]
+        return x.ctypes.data
+    return x.data_ptr()
+
+
+def _check(rc, ctx=None):
+    if rc != OK:
+        msg = lib().loip_last_error(ctx)
+        raise LoipError(rc, msg.decode() if msg else "")
+
+
+def model_desc(m: dict) -> ModelDesc:
+    return ModelDesc(m["n_layers"], m["hidden"], m["n_heads"], m["n_kv_heads"], m["head_dim"], m["ffn"], m["vocab"],
+                     m.get("rms_eps", 1e-5), m.get("rope_theta", 500000.0))
+
+
+def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 2048, mode: int = MODE_OVERLAP,
+           timeout_ms: int = 0, hbm_Bps: float = 6.7e12, link_Bps: float = 2.1e11, kv_reserve_bytes: int = 0,
+           max_prefill_tokens: int = 512, page_tokens: int = 64, use_graphs: int = 0) -> Config:
+    return Config(budget, n_slots, page_tokens, max_batch, max_ctx, use_graphs, mode, timeout_ms, hbm_Bps, link_Bps,
+                  kv_reserve_bytes, max_prefill_tokens)
+
+
+# ----------------------------------------------------------------------------
+# host-only planning
+# ----------------------------------------------------------------------------
+def loip_layer_layout(m: dict) -> dict:
+    out = LayerLayout()
+    _check(lib().loip_layer_layout(C.byref(model_desc(m)), C.byref(out)))
+    return {n: getattr(out, n) for n, _ in LayerLayout._fields_}
+
+
+def loip_plan_residency(m: dict, layer_bytes, budget: int, kv_bytes: int, fixed_bytes: int, n_slots: int,
+                        hbm_Bps: float, link_Bps: float) -> dict:
+    lb = np.ascontiguousarray(layer_bytes, dtype=np.uint64)
+    res = np.zeros(m["n_layers"], dtype=np.uint8)
+    plan = Plan()
+    plan.resident = res.ctypes.data_as(C.POINTER(C.c_uint8))
+    _check(lib().loip_plan_residency(C.byref(model_desc(m)), lb.ctypes.data, budget, kv_bytes, fixed_bytes, n_slots,
+                                     hbm_Bps, link_Bps, C.byref(plan)))
+    return {"n_resident": plan.n_resident, "n_offloaded": plan.n_offloaded, "resident": res.astype(bool),
+            "pred_step_s": plan.pred_step_s, "pred_copy_s": plan.pred_copy_s, "pred_compute_s": plan.pred_compute_s,
+            "eq1_step_s": plan.eq1_step_s, "left_bytes": plan.left_bytes}
+
+
+def loip_kv_threshold(left_bytes: int, kv_bytes_per_token: int) -> int:
+    out = C.c_uint64()
+    _check(lib().loip_kv_threshold(left_bytes, kv_bytes_per_token, C.byref(out)))
+    return out.value
+
+
+def loip_fixed_bytes(m: dict, cfg: Config) -> int:
+    out = C.c_uint64()
+    _check(lib().loip_fixed_bytes(C.byref(model_desc(m)), C.byref(cfg), C.byref(out)))
+    return out.value
+
+
+# ----------------------------------------------------------------------------
+# context
+# ----------------------------------------------------------------------------
+class Context:
+    """A loip_ctx plus the device arena (a torch uint8 tensor) it lives in."""
+
+    def __init__(self, m: dict, cfg: Config, arena=None):
+        import torch
+        self.model = dict(m)
+        self.cfg = cfg
+        if arena is None:
+            arena = torch.empty(cfg.device_budget_bytes, dtype=torch.uint8, device="cuda")
+        self.arena = arena
+        h = C.c_void_p()
+        rc = lib().loip_create(C.byref(model_desc(m)), C.byref(cfg), _ptr(arena), arena.numel(), C.byref(h))
+        _check(rc, None)
+        self.h = h
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().loip_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _c(self, rc):
+        _check(rc, self.h)
+
+    def load_weights_generated(self, seed: int):
+        self._c(lib().loip_load_weights_generated(self.h, seed))
+
+    def load_layer(self, layer: int, blob: np.ndarray):
+        self._c(lib().loip_load_layer(self.h, layer, _ptr(blob), blob.nbytes))
+
+    def load_globals(self, embed: np.ndarray, lm_head: np.ndarray, g_final: np.ndarray):
+        self._c(lib().loip_load_globals(self.h, _ptr(embed), _ptr(lm_head), _ptr(g_final)))
+
+    def plan(self) -> dict:
+        res = np.zeros(self.model["n_layers"], dtype=np.uint8)
+        p = Plan()
+        p.resident = res.ctypes.data_as(C.POINTER(C.c_uint8))
+        self._c(lib().loip_get_plan(self.h, C.byref(p)))
+        return {"n_resident": p.n_resident, "n_offloaded": p.n_offloaded, "resident": res.astype(bool),
+                "pred_step_s": p.pred_step_s, "eq1_step_s": p.eq1_step_s, "left_bytes": p.left_bytes}
+
+    def set_batch(self, ctx_lens):
+        cl = np.ascontiguousarray(ctx_lens, dtype=np.int32)
+        self._c(lib().loip_set_batch(self.h, cl.size, cl.ctypes.data))
+
+    def decode_step(self, tokens, out_hidden=None) -> np.ndarray:
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        out = np.empty_like(t)
+        self._c(lib().loip_decode_step(self.h, t.ctypes.data, t.size, out.ctypes.data, _ptr(out_hidden)))
+        return out
+
+    def decode_step_device(self, tokens_dev, out_tokens_dev, out_hidden=None):
+        self._c(lib().loip_decode_step_device(self.h, _ptr(tokens_dev), tokens_dev.numel(), _ptr(out_tokens_dev),
+                                              _ptr(out_hidden)))
+
+    def prefill(self, prompts, out_hidden=None) -> np.ndarray:
+        """prompts: list of 1-D int arrays.  Returns the argmax after each prompt."""
+        lens = np.array([len(p) for p in prompts], dtype=np.int32)
+        toks = np.ascontiguousarray(np.concatenate([np.asarray(p, dtype=np.int32) for p in prompts]))
+        out = np.empty(len(prompts), dtype=np.int32)
+        self._c(lib().loip_prefill(self.h, toks.ctypes.data, lens.ctypes.data, len(prompts), out.ctypes.data,
+                                   _ptr(out_hidden)))
+        return out
+
+    def stream_layer(self, layer: int, slot: int, copy_stream=None):
+        self._c(lib().loip_stream_layer(self.h, layer, slot, copy_stream))
+
+    def layer_forward(self, layer: int, slot: int, hidden, positions, compute_stream=None):
+        self._c(lib().loip_layer_forward(self.h, layer, slot, _ptr(hidden), _ptr(positions), hidden.shape[0],
+                                         compute_stream))
+
+    def replan(self, lookahead_tokens: int = 0):
+        self._c(lib().loip_replan(self.h, lookahead_tokens))
+
+    def stats(self) -> dict:
+        s = Stats()
+        self._c(lib().loip_get_stats(self.h, C.byref(s)))
+        out = {n: getattr(s, n) for n, _ in Stats._fields_}
+        out["kernel_ms"] = list(s.kernel_ms)
+        out["kernel_launches"] = list(s.kernel_launches)
+        return out
+
+    def set_kernel_timing(self, on: bool):
+        self._c(lib().loip_set_kernel_timing(self.h, 1 if on else 0))
+
+    def synchronize(self):
+        self._c(lib().loip_synchronize(self.h))
+
+    def compute_stream(self) -> int:
+        return lib().loip_compute_stream(self.h)
+
+    def copy_stream(self) -> int:
+        return lib().loip_copy_stream(self.h)
+
+
+def loip_create(m: dict, cfg: Config, arena=None) -> Context:
+    return Context(m, cfg, arena)
+
+
+# ----------------------------------------------------------------------------
+# kernel-level entry points (torch tensors in, async on `stream`)
+# ----------------------------------------------------------------------------
+def _s(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return stream
+
+
+def loip_k_generate(out, first: int, seed: int, tensor_id: int, kind: int, stream=None):
+    _check(lib().loip_k_generate(_ptr(out), out.numel(), first, seed, tensor_id, kind, _s(stream)))
+
+
+def loip_k_embed(embed, tokens, x, stream=None):
+    _check(lib().loip_k_embed(_ptr(embed), _ptr(tokens), tokens.numel(), embed.shape[1], _ptr(x), _s(stream)))
+
+
+def loip_k_qkv_rope(x, g, wqkv, Hq, Hkv, d, eps, theta, positions, q_out, kv_base, page_offsets, max_pages,
+                    page_tokens, layer, layer_page_bytes, stream=None):
+    B, H = x.shape
+    _check(lib().loip_k_qkv_rope(_ptr(x), _ptr(g), _ptr(wqkv), B, H, Hq, Hkv, d, eps, theta, _ptr(positions),
+                                 _ptr(q_out), _ptr(kv_base), _ptr(page_offsets), max_pages, page_tokens, layer,
+                                 layer_page_bytes, _s(stream)))
+
+
+def loip_k_attention_scratch_floats(B, Hq, d, max_ctx, page_tokens) -> int:
+    return int(lib().loip_k_attention_scratch_floats(B, Hq, d, max_ctx, page_tokens))
+
+
+def loip_k_attention(q, kv_base, page_offsets, max_pages, ctx_lens, Hq, Hkv, d, page_tokens, layer,
+                     layer_page_bytes, max_ctx, scratch, o, stream=None):
+    B = q.shape[0]
+    _check(lib().loip_k_attention(_ptr(q), _ptr(kv_base), _ptr(page_offsets), max_pages, _ptr(ctx_lens), B, Hq, Hkv, d,
+                                  page_tokens, layer, layer_page_bytes, max_ctx, _ptr(scratch), _ptr(o), _s(stream)))
+
+
+def loip_k_oproj(o, wo, x, stream=None):
+    B, K = o.shape
+    _check(lib().loip_k_oproj(_ptr(o), _ptr(wo), B, x.shape[1], K, _ptr(x), _s(stream)))
+
+
+def loip_k_gate_up(x, g, wg, wu, eps, a, stream=None):
+    B, H = x.shape
+    _check(lib().loip_k_gate_up(_ptr(x), _ptr(g), _ptr(wg), _ptr(wu), B, H, wg.shape[0], eps, _ptr(a), _s(stream)))
+
+
+def loip_k_down(a, wd, x, stream=None):
+    B, F = a.shape
+    _check(lib().loip_k_down(_ptr(a), _ptr(wd), B, x.shape[1], F, _ptr(x), _s(stream)))
+
+
+def loip_k_lm_head_scratch_bytes(B, V) -> int:
+    return int(lib().loip_k_lm_head_scratch_bytes(B, V))
+
+
+def loip_k_lm_head(x, g_final, lm_head, eps, z, logits, tokens, scratch, stream=None):
+    B, H = x.shape
+    _check(lib().loip_k_lm_head(_ptr(x), _ptr(g_final), _ptr(lm_head), B, H, lm_head.shape[0], eps, _ptr(z),
+                                _ptr(logits), _ptr(tokens), _ptr(scratch), _s(stream)))

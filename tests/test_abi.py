@@ -1,0 +1,104 @@
+"""The C ABI library loads, exports every declared symbol, validates arguments,
+and its host-only planner matches the planner oracle."""
+import re
+
+import numpy as np
+import pytest
+
+from oracle import planner as OP
+from paper_2512_21835_gb300 import configs, loip
+
+HEADER = __import__("os").path.join(__import__("os").path.dirname(__file__), "..", "include", "loip.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2512_21835_gb300 import build
+    build.build()
+    return loip.lib()
+
+
+def test_exports_every_declared_symbol(L):
+    text = open(HEADER).read()
+    declared = set(re.findall(r"^\s*(?:int|void|const char\*|uint64_t|void\*)\s+(loip_\w+)\s*\(", text, re.M))
+    assert len(declared) >= 30
+    for name in declared:
+        assert hasattr(L, name), name
+    assert declared == set(loip.exported_names())
+
+
+def test_layer_layout_sizes(L):
+    for name in ("tiny", "llama3-8b", "llama3-70b"):
+        m = configs.MODELS[name]
+        lay = loip.loip_layer_layout(m)
+        params = configs.layer_params(m)
+        assert params * 2 <= lay["l_size"] <= params * 2 + 8 * 256
+        assert lay["mha_bytes"] + lay["mlp_bytes"] == lay["l_size"]
+        for k in ("off_wqkv", "off_wo", "off_g_mlp", "off_wg", "off_wu", "off_wd"):
+            assert lay[k] % 256 == 0
+    lay70 = loip.loip_layer_layout(configs.MODELS["llama3-70b"])
+    # p_A of the 70B shape: (10240 + 8192) x 8192 + 8192 of 855,654,400 parameters
+    assert abs(lay70["mha_bytes"] / lay70["l_size"] - 0.17647) < 1e-4
+
+
+def test_invalid_arguments_rejected_without_gpu(L):
+    bad = dict(configs.MODELS["tiny"], head_dim=48)
+    with pytest.raises(loip.LoipError) as e:
+        loip.loip_layer_layout(bad)
+    assert e.value.code == loip.ERR_INVALID
+    with pytest.raises(loip.LoipError):
+        loip.loip_plan_residency(configs.MODELS["tiny"], [100, 100], 1000, 0, 0, 4, 1.0, 1.0)  # 4 slots
+    # create rejects a null arena before touching the device
+    import ctypes as C
+    h = C.c_void_p()
+    cfg = loip.config(budget=1 << 20)
+    rc = L.loip_create(C.byref(loip.model_desc(configs.MODELS["tiny"])), C.byref(cfg), None, 1 << 20, C.byref(h))
+    assert rc == loip.ERR_INVALID and not h.value
+
+
+@pytest.mark.parametrize("L_layers,budget_layers,K", [(80, 30, 2), (80, 12, 3), (32, 40, 2), (10, 4, 1), (16, 9, 2)])
+def test_plan_matches_planner_oracle(L, L_layers, budget_layers, K):
+    l_size = 1_711_308_800
+    fixed, kv = 4_200_000_000, 360_000_000
+    budget = fixed + kv + budget_layers * l_size + l_size // 3
+    m = dict(configs.MODELS["llama3-70b"], n_layers=L_layers)
+    got = loip.loip_plan_residency(m, [l_size] * L_layers, budget, kv, fixed, K, 6.7e12, 2.1e11)
+    want = OP.plan(L_layers, l_size, budget, fixed, kv, K, 6.7e12, 2.1e11)
+    assert got["n_resident"] == want["R"]
+    assert list(~got["resident"]) == want["offloaded"]
+    assert got["pred_step_s"] == pytest.approx(want["pred_step_s"], rel=1e-12)
+    comp, load = [l_size / 6.7e12] * L_layers, [l_size / 2.1e11] * L_layers
+    assert got["eq1_step_s"] == pytest.approx(OP.eq1_single_device(comp, load, want["offloaded"]), rel=1e-12)
+    left = budget - fixed - kv - want["R"] * l_size - (K * l_size if want["R"] < L_layers else 0)
+    assert got["left_bytes"] == left
+    # tokens beyond the current KV the left-over memory holds (Eq. 6 reading)
+    assert loip.loip_kv_threshold(left, 327_680) == OP.kv_threshold_tokens(budget, fixed + kv, l_size, want["R"],
+                                                                          K if want["R"] < L_layers else 0, 327_680)
+
+
+def test_plan_infeasible(L):
+    with pytest.raises(loip.LoipError) as e:
+        loip.loip_plan_residency(configs.MODELS["tiny"], [100, 100], 349, 50, 100, 2, 1.0, 1.0)
+    assert e.value.code == loip.ERR_INFEASIBLE
+
+
+def test_demotion_rule_oracle_properties():
+    # demoting one layer at a time from the even spacing keeps the runs within 1 of each other
+    for L_layers in (10, 32, 80):
+        mask = [False] * L_layers
+        for step in range(L_layers):
+            mask, v = OP.demote_one(mask)
+            assert v is not None and sum(mask) == step + 1
+            idx = [i for i, o in enumerate(mask) if o]
+            runs = [((idx[(j + 1) % len(idx)] - idx[j] - 1) % L_layers) for j in range(len(idx))]
+            if len(idx) < L_layers:
+                assert max(runs) <= 2 * min(runs) + 2
+        assert OP.demote_one(mask)[1] is None
+
+
+def test_fixed_bytes(L):
+    m = configs.MODELS["llama3-70b"]
+    fb = loip.loip_fixed_bytes(m, loip.config(budget=60 * 10 ** 9, max_batch=1, max_ctx=1088,
+                                              max_prefill_tokens=1024))
+    # embedding + LM head dominate: 2 x 128256 x 8192 x 2 bytes
+    assert 2 * 128256 * 8192 * 2 < fb < 2 * 128256 * 8192 * 2 + 400 * 2 ** 20
