@@ -266,6 +266,30 @@ int loip_k_attention(const float* q, const void* kv_base, const int64_t* page_of
                      void* stream);
 uint64_t loip_k_attention_scratch_floats(int32_t B, int32_t Hq, int32_t d, int32_t max_ctx, int32_t page_tokens);
 
+/* Scratch of loip_k_attention_noalloc: 4 Mi floats (16 MiB) per GPU. */
+#define LOIP_NOALLOC_SCRATCH_FLOATS (4ull << 20)
+
+/* loip_k_attention for callers that cannot allocate device memory: a process
+ * whose HBM is fully reserved by another allocator (a fixed arena, a caching
+ * allocator), where cudaMalloc would fail or break the memory budget, or a
+ * latency-critical path that must not pay the device-wide synchronisation of
+ * cudaMalloc/cudaFree.  The paper has no counterpart; this is a library
+ * convenience.  Same arguments and result as loip_k_attention without
+ * `scratch`: the partial softmax states go to a file-scope device array of
+ * LOIP_NOALLOC_SCRATCH_FLOATS floats that every GPU loading the library holds
+ * until the process exits.  LOIP_ERR_INVALID when
+ * B * Hq * ceil(max_ctx / page_tokens) * (d + 2) exceeds that size.  It
+ * allocates nothing (no cudaMalloc, cudaFree or allocating library call).
+ * The first call on a device, with that device current, looks up the array's
+ * device address (cudaGetSymbolAddress); make that first call before any
+ * stream capture.  All calls on a device share the array and it keeps the last
+ * call's contents (nothing in it needs to start at zero): calls that overlap on
+ * the GPU race. */
+int loip_k_attention_noalloc(const float* q, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
+                             const int32_t* ctx_lens, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
+                             int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx, float* o,
+                             void* stream);
+
 /* x += wo o  (output projection with the residual add); o fp32 [B, Hq*d]. */
 int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x, void* stream);
 

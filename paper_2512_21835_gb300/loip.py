@@ -88,6 +88,7 @@ _SIGS = {
     "loip_k_qkv_rope": (C.c_int, [P, P, P, I32, I32, I32, I32, I32, F32, F32, P, P, P, P, I32, I32, I32, U64, P]),
     "loip_k_attention": (C.c_int, [P, P, P, I32, P, I32, I32, I32, I32, I32, I32, U64, I32, P, P, P]),
     "loip_k_attention_scratch_floats": (C.c_uint64, [I32, I32, I32, I32, I32]),
+    "loip_k_attention_noalloc": (C.c_int, [P, P, P, I32, P, I32, I32, I32, I32, I32, I32, U64, I32, P, P]),
     "loip_k_oproj": (C.c_int, [P, P, I32, I32, I32, P, P]),
     "loip_k_gate_up": (C.c_int, [P, P, P, P, I32, I32, I32, F32, P, P]),
     "loip_k_down": (C.c_int, [P, P, I32, I32, I32, P, P]),
@@ -324,6 +325,18 @@ def loip_k_attention(q, kv_base, page_offsets, max_pages, ctx_lens, Hq, Hkv, d, 
     B = q.shape[0]
     _check(lib().loip_k_attention(_ptr(q), _ptr(kv_base), _ptr(page_offsets), max_pages, _ptr(ctx_lens), B, Hq, Hkv, d,
                                   page_tokens, layer, layer_page_bytes, max_ctx, _ptr(scratch), _ptr(o), _s(stream)))
+
+
+NOALLOC_SCRATCH_FLOATS = 4 << 20
+
+
+def loip_k_attention_noalloc(q, kv_base, page_offsets, max_pages, ctx_lens, Hq, Hkv, d, page_tokens, layer,
+                             layer_page_bytes, max_ctx, o, stream=None):
+    """loip_k_attention for callers that cannot allocate device memory: the
+    partial-state scratch is the library's own 16 MiB device array per GPU."""
+    B = q.shape[0]
+    _check(lib().loip_k_attention_noalloc(_ptr(q), _ptr(kv_base), _ptr(page_offsets), max_pages, _ptr(ctx_lens), B, Hq,
+                                          Hkv, d, page_tokens, layer, layer_page_bytes, max_ctx, _ptr(o), _s(stream)))
 
 
 def loip_k_oproj(o, wo, x, stream=None):
