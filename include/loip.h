@@ -94,9 +94,10 @@ typedef struct loip_stats {
     uint64_t kv_bytes;         /* bytes of KV pages allocated */
     uint64_t arena_used;       /* device arena bytes in use */
     /* per kernel class, accumulated while kernel timing is on (loip_set_kernel_timing):
-     * 0 qkv+rope, 1 attention (+combine), 2 o-proj, 3 gate/up, 4 down, 5 lm head (+argmax) */
-    double kernel_ms[6];
-    uint64_t kernel_launches[6];
+     * decode: 0 qkv+rope, 1 attention (+combine), 2 o-proj, 3 gate/up, 4 down, 5 lm head (+argmax);
+     * prefill: 6 qkv GEMM, 7 attention, 8 o-proj GEMM, 9 gate/up GEMM, 10 down GEMM, 11 RMSNorm */
+    double kernel_ms[12];
+    uint64_t kernel_launches[12];
 } loip_stats;
 
 typedef struct loip_ctx loip_ctx;
@@ -300,6 +301,16 @@ int loip_k_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const 
 
 /* x += wd a  (down projection with the residual add); a fp32 [B, F]. */
 int loip_k_down(const float* a, const uint16_t* wd, int32_t B, int32_t H, int32_t F, float* x, void* stream);
+
+/* Prefill projection on the tensor cores: x[M, N] += A[M, K] * W[N, K]^T with
+ * A and W bf16 row-major (K-contiguous, K % 8 == 0, 16-byte aligned), x fp32
+ * (N % 4 == 0), fp32 accumulation (tcgen05, TMA; the product the prefill runs
+ * for the output and down projections). */
+int loip_k_gemm_bf16(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N, int32_t K, float* x, void* stream);
+
+/* 0 if no tensor-core GEMM launch has recorded a failure (a bounded pipeline
+ * wait that ran out); otherwise the first failure code.  -1 if unreadable. */
+int loip_k_tc_status(void);
 
 /* Final RMSNorm and LM head: z = RMSNorm(x) * g_final (fp32 [B, H], may be
  * NULL), logits = lm_head z (fp32 [B, V], may be NULL) and the greedy token

@@ -15,6 +15,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "internal.h"
 
 namespace loip {
@@ -22,7 +24,7 @@ namespace {
 
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
-constexpr int kStageFloats = 12288;  // 48 KB of staged activations per block
+constexpr int kStageFloats = 16384;  // 64 KB of staged activations per block
 
 __device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
     uint4 r;
@@ -35,6 +37,15 @@ __device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u <<
 __device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 __device__ __forceinline__ float bf2f(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
 __device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
+
+// Programmatic dependent launch: let the next kernel of the stream start its
+// independent prologue, and wait for the previous kernel's results.  Both are
+// no-ops for a kernel launched without the attribute.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -79,16 +90,16 @@ struct GemvParams {
     uint64_t* keys;
     // QKV epilogue
     int Hq, Hkv, d;
-    float theta;
     const int32_t* positions;
     const int32_t* row_req;
     KvView kv;
+    RopeFreqs rope;
 };
 
 // rows handled per warp unit, by epilogue
 template <int EPI>
 struct UnitRows {
-    static constexpr int U = 2;
+    static constexpr int U = EPI == EPI_RESID ? 1 : 2;
 };
 
 template <int EPI>
@@ -159,24 +170,38 @@ __device__ __forceinline__ void fma_block(float (&acc)[U][BT], const uint4 (&w)[
     }
 }
 
-// Accumulates the unit's rows over staged chunk [kc0, kc0 + kn).
+// Accumulates the unit's rows over staged chunk [kc0, kc0 + kn).  Two register
+// batches of JU 128-bit loads per row alternate, so the next batch is in flight
+// while the current one is consumed.
+template <int BT, int U>
+__device__ __forceinline__ void load_batch(uint4 (&w)[4][U], const uint16_t* const (&rp)[U], const bool (&rv)[U],
+                                           int kc0, int j0, int nj, int K, int lane, int JU) {
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+        if (jj >= JU) break;
+        const int k = kc0 + (j0 + jj) * 256 + lane * 8;
+        const bool ok = (j0 + jj < nj) && (k < K);
+#pragma unroll
+        for (int r = 0; r < U; ++r) w[jj][r] = (ok && rv[r]) ? ld_stream(rp[r] + k) : make_uint4(0, 0, 0, 0);
+    }
+}
+
 template <int BT, int U, int EPI>
 __device__ __forceinline__ void unit_chunk(float (&acc)[U][BT], const uint16_t* const (&rp)[U], const bool (&rv)[U],
                                            const float* __restrict__ s, int kc0, int kn, int K, int lane) {
     constexpr int JU = (BT <= 2) ? 4 : 2;
     const int nj = (kn + 255) >> 8;
-    for (int j0 = 0; j0 < nj; j0 += JU) {
-        uint4 w[JU][U];
-#pragma unroll
-        for (int jj = 0; jj < JU; ++jj) {
-            int k = kc0 + (j0 + jj) * 256 + lane * 8;
-            bool ok = (j0 + jj < nj) && (k < K);
-#pragma unroll
-            for (int r = 0; r < U; ++r) w[jj][r] = (ok && rv[r]) ? ld_stream(rp[r] + k) : make_uint4(0, 0, 0, 0);
-        }
+    uint4 wa[4][U], wb[4][U];
+    load_batch<BT, U>(wa, rp, rv, kc0, 0, nj, K, lane, JU);
+    for (int j0 = 0; j0 < nj; j0 += 2 * JU) {
+        load_batch<BT, U>(wb, rp, rv, kc0, j0 + JU, nj, K, lane, JU);
 #pragma unroll
         for (int jj = 0; jj < JU; ++jj)
-            if (j0 + jj < nj) fma_block<BT, U>(acc, w[jj], s, j0 + jj, lane);
+            if (j0 + jj < nj) fma_block<BT, U>(acc, wa[jj], s, j0 + jj, lane);
+        load_batch<BT, U>(wa, rp, rv, kc0, j0 + 2 * JU, nj, K, lane, JU);
+#pragma unroll
+        for (int jj = 0; jj < JU; ++jj)
+            if (j0 + JU + jj < nj) fma_block<BT, U>(acc, wb[jj], s, j0 + JU + jj, lane);
     }
 }
 
@@ -197,10 +222,8 @@ __device__ __forceinline__ void unit_epilogue(const GemvParams& p, int unit, flo
             float v0 = acc[0][b] * inv[b], v1 = acc[1][b] * inv[b];
             const int pos = p.positions[b];
             if (h < p.Hq + p.Hkv) {
-                double freq = pow((double)p.theta, -2.0 * (double)i / (double)p.d);
-                double s, c;
-                sincos((double)pos * freq, &s, &c);
-                float cf = (float)c, sf = (float)s;
+                float cf, sf;
+                rope_cos_sin(pos, p.rope.inv_freq[i], &cf, &sf);
                 float r0 = v0 * cf - v1 * sf, r1 = v1 * cf + v0 * sf;
                 v0 = r0;
                 v1 = r1;
@@ -266,6 +289,20 @@ __global__ void __launch_bounds__(kThreads, 2) gemv_kernel(GemvParams p) {
     const bool single = K <= kc_max;
     const int KC = single ? ((K + 255) & ~255) : kc_max;
     const bool norm = p.g != nullptr;
+
+    // weights never depend on the previous kernel: start pulling this warp's
+    // first rows into L2 before waiting for the activations
+    pdl_trigger();
+    {
+        const int u0 = blockIdx.x * kWarps + warp;
+        if (lane < U && u0 < p.n_units) {
+            bool v;
+            const uint16_t* r = unit_row<EPI>(p, u0, lane, v);
+            const uint32_t bytes = (uint32_t)min(K * 2, 8192);
+            if (v) prefetch_l2(r, bytes);
+        }
+    }
+    pdl_wait();
 
     float ss[BT];
 #pragma unroll
@@ -375,6 +412,8 @@ __global__ void __launch_bounds__(kThreads, 2) gemv_kernel(GemvParams p) {
 
 __global__ void argmax_reduce_kernel(const uint64_t* keys, int nblocks, int BT, int B, int32_t* tokens) {
     __shared__ uint64_t s[256];
+    pdl_trigger();
+    pdl_wait();
     const int b = blockIdx.x;
     uint64_t k = 0;
     for (int i = threadIdx.x; i < nblocks; i += blockDim.x) {
@@ -390,14 +429,41 @@ __global__ void argmax_reduce_kernel(const uint64_t* keys, int nblocks, int BT, 
     if (threadIdx.x == 0 && b < B) tokens[b] = (int32_t)(0xffffffffu - (uint32_t)(s[0] & 0xffffffffu));
 }
 
+// Launch with programmatic stream serialisation when `pdl` (the previous
+// operation on the stream is a kernel of the same chain).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool pdl,
+                     Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = pdl ? at : nullptr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 template <int EPI>
-cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, int* nblocks_out = nullptr) {
+cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, bool pdl, int* nblocks_out = nullptr) {
     int BT = p.B <= 1 ? 1 : p.B <= 2 ? 2 : p.B <= 4 ? 4 : 8;
     int kc_max = (kStageFloats / BT) & ~255;
     bool single = p.K <= kc_max;
     int KC = single ? ((p.K + 255) & ~255) : kc_max;
     size_t smem = (size_t)KC * BT * sizeof(float);
     int blocks = (p.n_units + kWarps - 1) / kWarps;
+    static bool attr_set = false;
+    if (!attr_set) {  // before any occupancy query: the stage is above the 48 KB default
+        int bytes = kStageFloats * (int)sizeof(float);
+        cudaFuncSetAttribute(gemv_kernel<1, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        cudaFuncSetAttribute(gemv_kernel<2, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        cudaFuncSetAttribute(gemv_kernel<4, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        cudaFuncSetAttribute(gemv_kernel<8, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        attr_set = true;
+    }
     if (single) {
         static int per_sm[4] = {0, 0, 0, 0};
         static int sms = 0;
@@ -421,22 +487,13 @@ cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, int* nblocks_out = nullp
     }
     if (blocks < 1) blocks = 1;
     if (nblocks_out) *nblocks_out = blocks;
-    static bool attr_set = false;
-    if (!attr_set) {
-        int bytes = kStageFloats * (int)sizeof(float);
-        cudaFuncSetAttribute(gemv_kernel<1, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-        cudaFuncSetAttribute(gemv_kernel<2, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-        cudaFuncSetAttribute(gemv_kernel<4, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-        cudaFuncSetAttribute(gemv_kernel<8, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-        attr_set = true;
-    }
+
     switch (BT) {
-        case 1: gemv_kernel<1, EPI><<<blocks, kThreads, smem, st>>>(p); break;
-        case 2: gemv_kernel<2, EPI><<<blocks, kThreads, smem, st>>>(p); break;
-        case 4: gemv_kernel<4, EPI><<<blocks, kThreads, smem, st>>>(p); break;
-        default: gemv_kernel<8, EPI><<<blocks, kThreads, smem, st>>>(p); break;
+        case 1: return launch_k(gemv_kernel<1, EPI>, dim3(blocks), dim3(kThreads), smem, st, pdl, p);
+        case 2: return launch_k(gemv_kernel<2, EPI>, dim3(blocks), dim3(kThreads), smem, st, pdl, p);
+        case 4: return launch_k(gemv_kernel<4, EPI>, dim3(blocks), dim3(kThreads), smem, st, pdl, p);
+        default: return launch_k(gemv_kernel<8, EPI>, dim3(blocks), dim3(kThreads), smem, st, pdl, p);
     }
-    return cudaGetLastError();
 }
 
 // ----------------------------------------------------------------------------
@@ -463,6 +520,8 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
     __shared__ float s_m[G], s_l[G];
     __shared__ float s_o[G][D];
 
+    pdl_trigger();
+    pdl_wait();
     const int row = blockIdx.z, kvh = blockIdx.y;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
@@ -499,31 +558,47 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
         for (int t0 = warp * 32; t0 < P; t0 += 64) {
             const int tl = t0 + lane;
             const bool valid = (pg * P + tl) < ctx && tl < P;
+            const int nt = min(32, min(P - t0, ctx - (pg * P + t0)));
+            // every K row (one per lane) and every V slice of the 32 tokens in flight at once
+            uint4 kk[D / 8];
+            const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)(valid ? tl : t0) * D);
+#pragma unroll
+            for (int u = 0; u < D / 8; ++u) kk[u] = valid ? kr[u] : make_uint4(0, 0, 0, 0);
+            uint32_t vv[32][DPL / 2];
+#pragma unroll
+            for (int u = 0; u < 32; ++u) {
+                const uint16_t* vr = Vh + (size_t)(t0 + u) * D + lane * DPL;
+                const bool ok = u < nt;
+                if constexpr (DPL == 4) {
+                    uint2 v2 = ok ? *reinterpret_cast<const uint2*>(vr) : make_uint2(0, 0);
+                    vv[u][0] = v2.x;
+                    vv[u][1] = v2.y;
+                } else {
+                    static_assert(DPL == 2, "head_dim 64 or 128");
+                    vv[u][0] = ok ? *reinterpret_cast<const uint32_t*>(vr) : 0u;
+                }
+            }
             float s[G];
 #pragma unroll
             for (int g = 0; g < G; ++g) s[g] = 0.f;
-            if (valid) {
-                const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)tl * D);
-#pragma unroll 4
-                for (int dd = 0; dd < D / 8; ++dd) {
-                    uint4 kk = kr[dd];
-                    float kf[8] = {bf_lo(kk.x), bf_hi(kk.x), bf_lo(kk.y), bf_hi(kk.y),
-                                   bf_lo(kk.z), bf_hi(kk.z), bf_lo(kk.w), bf_hi(kk.w)};
 #pragma unroll
-                    for (int g = 0; g < G; ++g) {
-                        const float4 qa = *reinterpret_cast<const float4*>(&sq[g][dd * 8]);
-                        const float4 qb = *reinterpret_cast<const float4*>(&sq[g][dd * 8 + 4]);
-                        float a = s[g];
-                        a = fmaf(qa.x, kf[0], a);
-                        a = fmaf(qa.y, kf[1], a);
-                        a = fmaf(qa.z, kf[2], a);
-                        a = fmaf(qa.w, kf[3], a);
-                        a = fmaf(qb.x, kf[4], a);
-                        a = fmaf(qb.y, kf[5], a);
-                        a = fmaf(qb.z, kf[6], a);
-                        a = fmaf(qb.w, kf[7], a);
-                        s[g] = a;
-                    }
+            for (int u = 0; u < D / 8; ++u) {
+                const float kf[8] = {bf_lo(kk[u].x), bf_hi(kk[u].x), bf_lo(kk[u].y), bf_hi(kk[u].y),
+                                     bf_lo(kk[u].z), bf_hi(kk[u].z), bf_lo(kk[u].w), bf_hi(kk[u].w)};
+#pragma unroll
+                for (int g = 0; g < G; ++g) {
+                    const float4 qa = *reinterpret_cast<const float4*>(&sq[g][u * 8]);
+                    const float4 qb = *reinterpret_cast<const float4*>(&sq[g][u * 8 + 4]);
+                    float a = s[g];
+                    a = fmaf(qa.x, kf[0], a);
+                    a = fmaf(qa.y, kf[1], a);
+                    a = fmaf(qa.z, kf[2], a);
+                    a = fmaf(qa.w, kf[3], a);
+                    a = fmaf(qb.x, kf[4], a);
+                    a = fmaf(qb.y, kf[5], a);
+                    a = fmaf(qb.z, kf[6], a);
+                    a = fmaf(qb.w, kf[7], a);
+                    s[g] = a;
                 }
             }
             float pe[G];
@@ -539,25 +614,17 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
                 for (int c = 0; c < DPL; ++c) o[g][c] *= corr;
                 m[g] = mn;
             }
-            const int nt = min(32, min(P - t0, ctx - (pg * P + t0)));
-            for (int tt = 0; tt < nt; ++tt) {
-                const uint16_t* vr = Vh + (size_t)(t0 + tt) * D + lane * DPL;
+#pragma unroll
+            for (int u = 0; u < 32; ++u) {
                 float vf[DPL];
-                if constexpr (DPL == 4) {
-                    uint2 vv = *reinterpret_cast<const uint2*>(vr);
-                    vf[0] = bf_lo(vv.x);
-                    vf[1] = bf_hi(vv.x);
-                    vf[2] = bf_lo(vv.y);
-                    vf[3] = bf_hi(vv.y);
-                } else {
-                    static_assert(DPL == 2, "head_dim 64 or 128");
-                    uint32_t vv = *reinterpret_cast<const uint32_t*>(vr);
-                    vf[0] = bf_lo(vv);
-                    vf[1] = bf_hi(vv);
+#pragma unroll
+                for (int c = 0; c < DPL / 2; ++c) {
+                    vf[2 * c] = bf_lo(vv[u][c]);
+                    vf[2 * c + 1] = bf_hi(vv[u][c]);
                 }
 #pragma unroll
                 for (int g = 0; g < G; ++g) {
-                    float pg_ = __shfl_sync(0xffffffffu, pe[g], tt);
+                    const float pg_ = __shfl_sync(0xffffffffu, pe[g], u);
 #pragma unroll
                     for (int c = 0; c < DPL; ++c) o[g][c] = fmaf(pg_, vf[c], o[g][c]);
                 }
@@ -612,13 +679,17 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
 
 // Combines the per-page partial softmax states of one (row, head).
 __global__ void attn_combine_kernel(AttnParams p, int D) {
+    pdl_trigger();
+    pdl_wait();
     const int h = blockIdx.x, row = blockIdx.y, j = threadIdx.x;
     const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
     const int n = (ctx + p.kv.page_tokens - 1) / p.kv.page_tokens;
     const float* part = p.scratch + ((size_t)row * p.Hq + h) * p.max_chunks * (D + 2);
     float M = -INFINITY;
+#pragma unroll 8
     for (int c = 0; c < n; ++c) M = fmaxf(M, part[(size_t)c * (D + 2) + D]);
     float L = 0.f, acc = 0.f;
+#pragma unroll 8
     for (int c = 0; c < n; ++c) {
         const float* pc = part + (size_t)c * (D + 2);
         float w = (pc[D] == -INFINITY) ? 0.f : expf(pc[D] - M);
@@ -634,24 +705,29 @@ __global__ void attn_combine_kernel(AttnParams p, int D) {
 }
 
 template <int G, int D>
-cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st) {
+cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st, bool pdl) {
     dim3 grid(p.split ? p.max_chunks : 1, p.Hkv, p.B);
-    attn_kernel<G, D><<<grid, 64, 0, st>>>(p);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_k(attn_kernel<G, D>, grid, dim3(64), 0, st, pdl, p);
     if (e != cudaSuccess || !p.split) return e;
-    attn_combine_kernel<<<dim3(p.Hq, p.B), D, 0, st>>>(p, D);
-    return cudaGetLastError();
+    return launch_k(attn_combine_kernel, dim3(p.Hq, p.B), dim3(D), 0, st, pdl, p, D);
 }
 
 // ----------------------------------------------------------------------------
 // Embedding gather and generator
 // ----------------------------------------------------------------------------
 __global__ void embed_kernel(const uint16_t* E, const int32_t* tokens, int H, int V, float* x) {
+    pdl_trigger();
+    pdl_wait();
     const int b = blockIdx.x;
     const int tok = tokens[b];
     const bool ok = tok >= 0 && tok < V;
-    const uint16_t* row = E + (size_t)(ok ? tok : 0) * H;
-    for (int i = threadIdx.x; i < H; i += blockDim.x) x[(size_t)b * H + i] = ok ? bf2f(row[i]) : 0.f;
+    const uint4* row = reinterpret_cast<const uint4*>(E + (size_t)(ok ? tok : 0) * H);
+    float4* out = reinterpret_cast<float4*>(x + (size_t)b * H);
+    for (int i = threadIdx.x; i < H / 8; i += blockDim.x) {  // 8 bf16 per 16-byte load
+        const uint4 v = ok ? row[i] : make_uint4(0, 0, 0, 0);
+        out[2 * i] = make_float4(bf_lo(v.x), bf_hi(v.x), bf_lo(v.y), bf_hi(v.y));
+        out[2 * i + 1] = make_float4(bf_lo(v.z), bf_hi(v.z), bf_lo(v.w), bf_hi(v.w));
+    }
 }
 
 // SplitMix64 (Steele, Lea & Flood 2014) used as a counter-based generator:
@@ -675,6 +751,8 @@ __device__ __forceinline__ uint16_t gen_elem(uint64_t seed, uint32_t tensor_id, 
 }
 
 __global__ void advance_kernel(int32_t* pos, int B) {
+    pdl_trigger();
+    pdl_wait();
     if ((int)threadIdx.x < B) pos[threadIdx.x] += 1;
 }
 
@@ -692,7 +770,7 @@ __global__ void generate_kernel(uint16_t* out, uint64_t n, uint64_t first, uint6
 // ----------------------------------------------------------------------------
 cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
                             int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
-                            const int32_t* row_req, cudaStream_t st) {
+                            const int32_t* row_req, cudaStream_t st, bool pdl) {
     GemvParams p{};
     p.in = x;
     p.g = g;
@@ -706,27 +784,28 @@ cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* w
     p.Hq = Hq;
     p.Hkv = Hkv;
     p.d = d;
-    p.theta = theta;
+    p.rope = rope_freqs(theta, d);
     p.positions = positions;
     p.row_req = row_req;
     p.kv = kv;
-    return launch_gemv<EPI_QKV>(p, st);
+    return launch_gemv<EPI_QKV>(p, st, pdl);
 }
 
-cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st) {
+cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st,
+                              bool pdl) {
     GemvParams p{};
     p.in = in;
     p.w0 = w;
     p.B = B;
     p.K = K;
     p.N = N;
-    p.n_units = (N + 1) / 2;
+    p.n_units = N;
     p.out = x;
-    return launch_gemv<EPI_RESID>(p, st);
+    return launch_gemv<EPI_RESID>(p, st, pdl);
 }
 
 cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,
-                           int F, float eps, float* a, cudaStream_t st) {
+                           int F, float eps, float* a, cudaStream_t st, bool pdl) {
     GemvParams p{};
     p.in = x;
     p.g = g;
@@ -738,7 +817,13 @@ cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg
     p.n_units = F;
     p.eps = eps;
     p.out = a;
-    return launch_gemv<EPI_SWIGLU>(p, st);
+    return launch_gemv<EPI_SWIGLU>(p, st, pdl);
+}
+
+RopeFreqs rope_freqs(float theta, int d) {
+    RopeFreqs f{};
+    for (int i = 0; i < d / 2 && i < 64; ++i) f.inv_freq[i] = pow((double)theta, -2.0 * (double)i / (double)d);
+    return f;
 }
 
 size_t lm_head_scratch_bytes(int B, int V) {
@@ -749,7 +834,7 @@ size_t lm_head_scratch_bytes(int B, int V) {
 }
 
 cudaError_t launch_lm_head(const float* x, const uint16_t* g, const uint16_t* w, int B, int H, int V, float eps,
-                           float* z, float* logits, int32_t* tokens, void* scratch, cudaStream_t st) {
+                           float* z, float* logits, int32_t* tokens, void* scratch, cudaStream_t st, bool pdl) {
     GemvParams p{};
     p.in = x;
     p.g = g;
@@ -763,11 +848,11 @@ cudaError_t launch_lm_head(const float* x, const uint16_t* g, const uint16_t* w,
     p.z = z;
     p.keys = reinterpret_cast<uint64_t*>(scratch);
     int nblocks = 0;
-    cudaError_t e = launch_gemv<EPI_LOGITS>(p, st, &nblocks);
+    cudaError_t e = launch_gemv<EPI_LOGITS>(p, st, pdl, &nblocks);
     if (e != cudaSuccess) return e;
     int BT = B <= 1 ? 1 : B <= 2 ? 2 : B <= 4 ? 4 : 8;
-    argmax_reduce_kernel<<<B, 256, 0, st>>>(p.keys, nblocks, BT, B, tokens);
-    return cudaGetLastError();
+    return launch_k(argmax_reduce_kernel, dim3(B), dim3(256), 0, st, true, (const uint64_t*)p.keys, nblocks, BT, B,
+                    tokens);
 }
 
 size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens) {
@@ -777,7 +862,7 @@ size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_toke
 
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
-                             float* scratch, void* o, bool o_bf16, cudaStream_t st) {
+                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl) {
     AttnParams p{};
     p.q = q;
     p.kv = kv;
@@ -796,31 +881,29 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
     const int G = Hq / Hkv;
     if (d == 128) {
         switch (G) {
-            case 1: return launch_attn_t<1, 128>(p, st);
-            case 2: return launch_attn_t<2, 128>(p, st);
-            case 4: return launch_attn_t<4, 128>(p, st);
-            case 8: return launch_attn_t<8, 128>(p, st);
+            case 1: return launch_attn_t<1, 128>(p, st, pdl);
+            case 2: return launch_attn_t<2, 128>(p, st, pdl);
+            case 4: return launch_attn_t<4, 128>(p, st, pdl);
+            case 8: return launch_attn_t<8, 128>(p, st, pdl);
         }
     } else if (d == 64) {
         switch (G) {
-            case 1: return launch_attn_t<1, 64>(p, st);
-            case 2: return launch_attn_t<2, 64>(p, st);
-            case 4: return launch_attn_t<4, 64>(p, st);
-            case 8: return launch_attn_t<8, 64>(p, st);
+            case 1: return launch_attn_t<1, 64>(p, st, pdl);
+            case 2: return launch_attn_t<2, 64>(p, st, pdl);
+            case 4: return launch_attn_t<4, 64>(p, st, pdl);
+            case 8: return launch_attn_t<8, 64>(p, st, pdl);
         }
     }
     return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_embed(const uint16_t* embed, const int32_t* tokens, int B, int H, int V, float* x,
-                         cudaStream_t st) {
-    embed_kernel<<<B, 256, 0, st>>>(embed, tokens, H, V, x);
-    return cudaGetLastError();
+                         cudaStream_t st, bool pdl) {
+    return launch_k(embed_kernel, dim3(B), dim3(256), 0, st, pdl, embed, tokens, H, V, x);
 }
 
-cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st) {
-    advance_kernel<<<1, 32, 0, st>>>(positions, B);
-    return cudaGetLastError();
+cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st, bool pdl) {
+    return launch_k(advance_kernel, dim3(1), dim3(32), 0, st, pdl, positions, B);
 }
 
 cudaError_t launch_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id, int kind,

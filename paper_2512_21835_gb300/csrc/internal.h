@@ -11,6 +11,22 @@ namespace loip {
 // at byte offset layer * layer_page_bytes sit K [Hkv][page_tokens][d] and then
 // V [Hkv][page_tokens][d], bf16.  page_offsets[row * max_pages + i] is the
 // byte offset of page i of page-table row `row` from `base`.
+// Rotary inverse frequencies theta^(-2i/d), i < d/2, computed in fp64 on the host.
+struct RopeFreqs {
+    double inv_freq[64];
+};
+RopeFreqs rope_freqs(float theta, int d);
+
+// cos/sin of pos * inv_freq: the angle is formed and reduced modulo 2*pi in fp64
+// (two-term Cody-Waite reduction), then sincosf on the reduced angle.
+__device__ __forceinline__ void rope_cos_sin(int pos, double inv_freq, float* c, float* s) {
+    const double a = (double)pos * inv_freq;
+    const double k = rint(a * 0.15915494309189535);  // 1 / (2 pi)
+    double r = fma(-k, 6.283185307179586, a);          // 2 pi, high part
+    r = fma(-k, 2.4492935982947064e-16, r);            // 2 pi - high part
+    sincosf((float)r, s, c);
+}
+
 struct KvView {
     char* base;
     const int64_t* page_offsets;
@@ -24,12 +40,14 @@ struct KvView {
 // activation; every kernel streams its weight matrix exactly once.
 cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
                             int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
-                            const int32_t* row_req, cudaStream_t st);
-cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st);
+                            const int32_t* row_req, cudaStream_t st, bool pdl = false);
+cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st,
+                              bool pdl = false);
 cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,
-                           int F, float eps, float* a, cudaStream_t st);
+                           int F, float eps, float* a, cudaStream_t st, bool pdl = false);
 cudaError_t launch_lm_head(const float* x, const uint16_t* g, const uint16_t* w, int B, int H, int V, float eps,
-                           float* z, float* logits, int32_t* tokens, void* scratch, cudaStream_t st);
+                           float* z, float* logits, int32_t* tokens, void* scratch, cudaStream_t st,
+                           bool pdl = false);
 size_t lm_head_scratch_bytes(int B, int V);
 
 // Grouped-query attention over the paged cache.  Rows b = 0..B-1 attend over
@@ -39,26 +57,29 @@ size_t lm_head_scratch_bytes(int B, int V);
 // combine kernel writes o; otherwise one block per (row, kv head) loops over all
 // pages.  o_bf16: write o as bf16 (prefill) instead of fp32.
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
-                             const int32_t* row_req, int B, int Hq,
-                             int Hkv, int d, int max_ctx, bool split, float* scratch, void* o, bool o_bf16,
-                             cudaStream_t st);
+                             const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
+                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl = false);
 size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens);
 
 cudaError_t launch_embed(const uint16_t* embed, const int32_t* tokens, int B, int H, int V, float* x,
-                         cudaStream_t st);
-cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st);
+                         cudaStream_t st, bool pdl = false);
+cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st, bool pdl = false);
 cudaError_t launch_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id, int kind,
                             cudaStream_t st);
 
-// Prefill (M tokens at once): bf16 x fp32-accumulate GEMMs with fused epilogues.
+// Prefill (M tokens at once).
 cudaError_t launch_rmsnorm_bf16(const float* x, const uint16_t* g, int M, int H, float eps, uint16_t* y,
                                 cudaStream_t st);
-cudaError_t launch_gemm_qkv_rope(const uint16_t* y, const uint16_t* wqkv, int M, int H, int Hq, int Hkv, int d,
-                                 float theta, const int32_t* positions, const int32_t* row_req, float* q, KvView kv,
+// Prefill projections on the tensor cores (tcgen05, TMA), fused epilogues.
+cudaError_t launch_tc_gemm_qkv_rope(const uint16_t* y, const uint16_t* wqkv, int M, int H, int Hq, int Hkv, int d,
+                                    float theta, const int32_t* positions, const int32_t* row_req, float* q,
+                                    KvView kv, cudaStream_t st);
+cudaError_t launch_tc_gemm_resid(const uint16_t* a, const uint16_t* w, int M, int N, int K, float* x,
                                  cudaStream_t st);
-cudaError_t launch_gemm_resid(const uint16_t* a, const uint16_t* w, int M, int N, int K, float* x, cudaStream_t st);
-cudaError_t launch_gemm_swiglu(const uint16_t* y, const uint16_t* wg, const uint16_t* wu, int M, int H, int F,
-                               uint16_t* a, cudaStream_t st);
+cudaError_t launch_tc_gemm_swiglu(const uint16_t* y, const uint16_t* wg, const uint16_t* wu, int M, int H, int F,
+                                  uint16_t* a, cudaStream_t st);
+// First failure code recorded by a tensor-core GEMM launch (0 = none).
+cudaError_t tc_error(int* code);
 cudaError_t launch_gather_rows(const float* x, const int32_t* rows, int n, int H, float* out, cudaStream_t st);
 
 }  // namespace loip

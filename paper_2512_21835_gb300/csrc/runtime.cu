@@ -179,6 +179,10 @@ struct loip_ctx {
     std::vector<cudaEvent_t> event_pool;
     uint64_t copy_seq = 0, compute_seq = 0;
     bool ktiming = false;
+    // true when the last operation enqueued on the compute stream is a kernel
+    // of the decode chain, so the next kernel may use programmatic launch
+    bool chain = false;
+    bool pdl() const { return chain && !ktiming; }
     struct KEv {
         int cls;
         cudaEvent_t a, b;
@@ -378,8 +382,10 @@ struct loip_ctx {
         if (!ktiming) return fn();
         cudaEvent_t a = take_event(), b = take_event();
         cudaEventRecord(a, s);
+        chain = false;
         cudaError_t e = fn();
         cudaEventRecord(b, s);
+        chain = false;
         kernel_events.push_back({cls, a, b});
         return e;
     }
@@ -417,19 +423,20 @@ struct loip_ctx {
         cudaError_t e;
         e = timed(0, s, [&] {
             return launch_qkv_rope(x, g_attn, wqkv, B, H, Hq, Hkv, d, desc.rms_eps, desc.rope_theta, pos_dev, q, kv,
-                                   nullptr, s);
+                                   nullptr, s, pdl());
         });
         if (e != cudaSuccess) return cuda_fail(e, "qkv kernel");
+        chain = true;
         e = timed(1, s, [&] {
             return launch_attention(q, kv, nullptr, pos_dev, nullptr, B, Hq, Hkv, d, cfg.max_ctx, true,
-                                    fixed_ptr<float>(fx.attn_scratch), o, false, s);
+                                    fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl());
         });
         if (e != cudaSuccess) return cuda_fail(e, "attention kernel");
-        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s); });
+        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl()); });
         if (e != cudaSuccess) return cuda_fail(e, "o-proj kernel");
-        e = timed(3, s, [&] { return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s); });
+        e = timed(3, s, [&] { return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s, pdl()); });
         if (e != cudaSuccess) return cuda_fail(e, "gate/up kernel");
-        e = timed(4, s, [&] { return launch_resid_gemv(a, wd, B, H, F, x, s); });
+        e = timed(4, s, [&] { return launch_resid_gemv(a, wd, B, H, F, x, s, pdl()); });
         if (e != cudaSuccess) return cuda_fail(e, "down kernel");
         return LOIP_OK;
     }
@@ -447,15 +454,25 @@ struct loip_ctx {
         const int64_t* pt = fixed_ptr<int64_t>(fx.page_table);
         KvView kv = kv_view(l, pt);
         cudaError_t e;
-        e = launch_rmsnorm_bf16(px, w + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s);
+        e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, w + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s); });
         if (e == cudaSuccess)
-            e = launch_gemm_qkv_rope(py, w + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos, req, pq, kv, s);
+            e = timed(6, s, [&] {
+                return launch_tc_gemm_qkv_rope(py, w + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos, req,
+                                               pq, kv, s);
+            });
         if (e == cudaSuccess)
-            e = launch_attention(pq, kv, nullptr, pos, req, Mc, Hq, Hkv, d, cfg.max_ctx, false, nullptr, po, true, s);
-        if (e == cudaSuccess) e = launch_gemm_resid(po, w + lay.off_wo / 2, Mc, H, qd, px, s);
-        if (e == cudaSuccess) e = launch_rmsnorm_bf16(px, w + lay.off_g_mlp / 2, Mc, H, desc.rms_eps, py, s);
-        if (e == cudaSuccess) e = launch_gemm_swiglu(py, w + lay.off_wg / 2, w + lay.off_wu / 2, Mc, H, F, pa, s);
-        if (e == cudaSuccess) e = launch_gemm_resid(pa, w + lay.off_wd / 2, Mc, H, F, px, s);
+            e = timed(7, s, [&] {
+                return launch_attention(pq, kv, nullptr, pos, req, Mc, Hq, Hkv, d, cfg.max_ctx, false, nullptr, po,
+                                        true, s);
+            });
+        if (e == cudaSuccess) e = timed(8, s, [&] { return launch_tc_gemm_resid(po, w + lay.off_wo / 2, Mc, H, qd, px, s); });
+        if (e == cudaSuccess)
+            e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, w + lay.off_g_mlp / 2, Mc, H, desc.rms_eps, py, s); });
+        if (e == cudaSuccess)
+            e = timed(9, s, [&] {
+                return launch_tc_gemm_swiglu(py, w + lay.off_wg / 2, w + lay.off_wu / 2, Mc, H, F, pa, s);
+            });
+        if (e == cudaSuccess) e = timed(10, s, [&] { return launch_tc_gemm_resid(pa, w + lay.off_wd / 2, Mc, H, F, px, s); });
         if (e != cudaSuccess) return cuda_fail(e, "prefill kernel");
         return LOIP_OK;
     }
@@ -471,6 +488,7 @@ struct loip_ctx {
                     // conventional path: load when needed, compute waits
                     slot = 0;
                     cudaEventRecord(ev_reach, compute);
+                    chain = false;
                     cudaStreamWaitEvent(copy, ev_reach, 0);
                     int rc = enqueue_copy(l, 0, copy);
                     if (rc) return rc;
@@ -481,12 +499,14 @@ struct loip_ctx {
                 }
                 cudaError_t e = cudaStreamWaitEvent(compute, slot_full[slot], 0);
                 if (e != cudaSuccess) return cuda_fail(e, "compute wait");
+                chain = false;
             }
             int rc = fn(l, slot);
             if (rc) return rc;
             if (offloaded[l]) {
                 cudaError_t e = cudaEventRecord(slot_free[slot], compute);
                 if (e != cudaSuccess) return cuda_fail(e, "slot free event");
+                chain = false;
                 if (!naive) {
                     ++compute_seq;
                     rc = issue_next_copy();
@@ -914,7 +934,9 @@ extern "C" int loip_layer_forward(loip_ctx* c, int32_t layer, int32_t slot, floa
         e = cudaStreamWaitEvent(s, c->slot_full[slot], 0);
         if (e != cudaSuccess) return c->cuda_fail(e, "slot wait");
     }
+    c->chain = false;
     rc = c->decode_layer(layer, batch, positions, s, slot);
+    c->chain = false;
     if (rc) return rc;
     if (c->offloaded[layer]) cudaEventRecord(c->slot_free[slot], s);
     e = cudaMemcpyAsync(hidden, x, (size_t)batch * c->H * 4, cudaMemcpyDeviceToDevice, s);
@@ -944,20 +966,24 @@ static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int3
     int32_t* pos = c->fixed_ptr<int32_t>(c->fx.dec_pos);
     cudaError_t e;
     cudaEventRecord(c->ev_step0, s);
+    c->chain = false;
     float* x = c->fixed_ptr<float>(c->fx.x);
-    e = launch_embed(c->fixed_ptr<uint16_t>(c->fx.embed), d_tokens, B, c->H, c->V, x, s);
+    e = launch_embed(c->fixed_ptr<uint16_t>(c->fx.embed), d_tokens, B, c->H, c->V, x, s, false);
     if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
+    c->chain = true;
     rc = c->run_layers([&](int l, int slot) { return c->decode_layer(l, B, pos, s, slot); });
     if (rc) return rc;
     e = c->timed(5, s, [&] {
         return launch_lm_head(x, c->fixed_ptr<uint16_t>(c->fx.g_final), c->fixed_ptr<uint16_t>(c->fx.lm_head), B, c->H,
                               c->V, c->desc.rms_eps, out_hidden ? out_hidden : c->fixed_ptr<float>(c->fx.z),
-                              c->fixed_ptr<float>(c->fx.logits), d_out, c->fixed_ptr<void>(c->fx.lm_scratch), s);
+                              c->fixed_ptr<float>(c->fx.logits), d_out, c->fixed_ptr<void>(c->fx.lm_scratch), s,
+                              c->pdl());
     });
     if (e != cudaSuccess) return c->cuda_fail(e, "lm head kernel");
-    e = launch_advance(pos, B, s);
+    e = launch_advance(pos, B, s, !c->ktiming);
     if (e != cudaSuccess) return c->cuda_fail(e, "position advance");
     cudaEventRecord(c->ev_step1, s);
+    c->chain = false;
     for (int b = 0; b < B; ++b) c->reqs[b].len += 1;
     c->st.steps += 1;
     c->st.tokens += B;
@@ -1092,6 +1118,12 @@ extern "C" int loip_prefill(loip_ctx* c, const int32_t* tokens, const int32_t* p
     cudaEventRecord(c->ev_done, s);
     rc = c->wait_event(c->ev_done);
     if (rc) return rc;
+    c->collect_kernel_times();
+    int tcerr = 0;
+    if (tc_error(&tcerr) != cudaSuccess || tcerr != 0) {
+        c->failed = true;
+        return c->fail(LOIP_ERR_TIMEOUT, "tensor-core GEMM pipeline did not complete (code " + std::to_string(tcerr) + ")");
+    }
     memcpy(out_tokens, hout, (size_t)n_prompts * 4);
     for (int i = 0; i < n_prompts; ++i) c->reqs[i].len = prompt_lens[i];
     c->active_batch = n_prompts;
@@ -1152,7 +1184,7 @@ extern "C" int loip_set_kernel_timing(loip_ctx* c, int32_t enable) {
     int rc = c->sync_all();
     if (rc) return rc;
     c->collect_kernel_times();
-    for (int i = 0; i < 6; ++i) {
+    for (int i = 0; i < 12; ++i) {
         c->st.kernel_ms[i] = 0;
         c->st.kernel_launches[i] = 0;
     }
@@ -1228,6 +1260,20 @@ extern "C" int loip_k_down(const float* a, const uint16_t* wd, int32_t B, int32_
                            void* stream) {
     if (!a || !wd || !x || B < 1 || B > 8 || F % 8 || H < 1 || !al16(wd)) return LOIP_ERR_INVALID;
     return cerr(launch_resid_gemv(a, wd, B, H, F, x, (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_gemm_bf16(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N, int32_t K, float* x,
+                                void* stream) {
+    if (!A || !W || !x || M < 1 || N < 1 || K < 8 || K % 8 || !al16(A) || !al16(W) || !al16(x) || N % 4)
+        return LOIP_ERR_INVALID;
+    cudaError_t e = launch_tc_gemm_resid(A, W, M, N, K, x, (cudaStream_t)stream);
+    return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA;
+}
+
+extern "C" int loip_k_tc_status(void) {
+    int code = 0;
+    if (tc_error(&code) != cudaSuccess) return -1;
+    return code;
 }
 
 extern "C" uint64_t loip_k_lm_head_scratch_bytes(int32_t B, int32_t V) {

@@ -33,3 +33,10 @@ def bf16_bits(seed: int, shape, scale: float = 0.02) -> np.ndarray:
     from fp32 -- any bf16 pattern is a valid input."""
     f = normal_f32(seed, shape, scale)
     return (f.view(np.uint32) >> 16).astype(np.uint16)
+
+
+def batched_prompts(ctx_seed: int, tok_seed: int, batch: int, lo: int, hi: int, vocab: int):
+    """Requests with context lengths uniform in [lo, hi] (seed ctx_seed), each a
+    prompt of uniform token ids (seed tok_seed + request index)."""
+    lens = context_lengths(ctx_seed, batch, lo, hi)
+    return [token_ids(tok_seed + 1000 * (i + 1), int(n), vocab) for i, n in enumerate(lens)]

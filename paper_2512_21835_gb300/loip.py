@@ -55,7 +55,7 @@ class Stats(C.Structure):
                 ("last_step_ms", C.c_double), ("copy_busy_ms", C.c_double), ("compute_ms", C.c_double),
                 ("n_resident", C.c_int32), ("n_offloaded", C.c_int32), ("n_replans", C.c_int32),
                 ("kv_tokens", C.c_uint64), ("kv_bytes", C.c_uint64), ("arena_used", C.c_uint64),
-                ("kernel_ms", C.c_double * 6), ("kernel_launches", C.c_uint64 * 6)]
+                ("kernel_ms", C.c_double * 12), ("kernel_launches", C.c_uint64 * 12)]
 
 
 P, U64, I32, U32, F32, F64, VP = C.c_void_p, C.c_uint64, C.c_int32, C.c_uint32, C.c_float, C.c_double, C.c_void_p
@@ -94,6 +94,8 @@ _SIGS = {
     "loip_k_down": (C.c_int, [P, P, I32, I32, I32, P, P]),
     "loip_k_lm_head": (C.c_int, [P, P, P, I32, I32, I32, F32, P, P, P, P, P]),
     "loip_k_lm_head_scratch_bytes": (C.c_uint64, [I32, I32]),
+    "loip_k_gemm_bf16": (C.c_int, [P, P, I32, I32, I32, P, P]),
+    "loip_k_tc_status": (C.c_int, []),
 }
 
 _lib = None
@@ -352,6 +354,16 @@ def loip_k_gate_up(x, g, wg, wu, eps, a, stream=None):
 def loip_k_down(a, wd, x, stream=None):
     B, F = a.shape
     _check(lib().loip_k_down(_ptr(a), _ptr(wd), B, x.shape[1], F, _ptr(x), _s(stream)))
+
+
+def loip_k_gemm_bf16(A, W, x, stream=None):
+    """x += A W^T on the tensor cores (A [M, K], W [N, K] bf16 as int16 tensors)."""
+    M, K = A.shape
+    _check(lib().loip_k_gemm_bf16(_ptr(A), _ptr(W), M, W.shape[0], K, _ptr(x), _s(stream)))
+
+
+def loip_k_tc_status() -> int:
+    return int(lib().loip_k_tc_status())
 
 
 def loip_k_lm_head_scratch_bytes(B, V) -> int:
