@@ -87,19 +87,18 @@ class Clocks:
 
 
 def link_peak_gbs(torch, nbytes=1 << 30, reps=5):
-    """Live host->device copy peak: pinned source, one cudaMemcpyAsync, best of reps."""
-    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
-    d = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
-    best = 1e9
-    for _ in range(reps):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record()
-        d.copy_(h, non_blocking=True)
-        b.record()
-        b.synchronize()
-        best = min(best, a.elapsed_time(b) / 1e3)
-    del h, d
-    return nbytes / best / 1e9
+    """Live host->device copy peak: the pool's pinned memory, one cudaMemcpyAsync, best of reps."""
+    from paper_2512_21835_gb300 import loip
+    return loip.loip_measure_h2d(nbytes, reps) / 1e9
+
+
+def max_over_ranks(values, device="cpu"):
+    """Elementwise max of per-rank timings (replicas are timed between barriers)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
 
 
 def workload_setup(name):
@@ -196,15 +195,19 @@ def run_ours(args, rank, world):
     torch.cuda.synchronize()
     ctx.synchronize()
     st0 = ctx.stats()
+    step_ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     with Clocks() as clk:
         ev0.record(s)
-        for _ in range(steps):
+        for i in range(steps):
             ctx.decode_step_device(tok, tok2)
             tok, tok2 = tok2, tok
+            step_ev[i].record(s)
         ev1.record(s)
         ctx.synchronize()
         torch.cuda.synchronize()
     dev_s = ev0.elapsed_time(ev1) / 1e3
+    step_ms = [round(ev0.elapsed_time(step_ev[0]), 2)] + [round(step_ev[i - 1].elapsed_time(step_ev[i]), 2)
+                                                          for i in range(1, steps)]
     st1 = ctx.stats()
     # ---- per-kernel durations (CUDA events around every launch, separate pass) ----
     ctx.set_kernel_timing(True)
@@ -228,10 +231,7 @@ def run_ours(args, rank, world):
     ctx.close()
 
     if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([dev_s, e2e_s], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        dev_s, e2e_s = float(t[0]), float(t[1])
+        dev_s, e2e_s = max_over_ranks([dev_s, e2e_s], device="cuda")
 
     tokens = steps * Bsz * world
     n_off = st1["n_offloaded"]
@@ -282,10 +282,17 @@ def run_ours(args, rank, world):
                           "exposed_frac": round(exposed / step_s, 4),
                           "kernel_ms_per_step": {n: round(st["kernel_ms"][i] / steps, 4)
                                                  for i, n in enumerate(KERNEL_NAMES)},
-                          "copy_busy_ms_last": round(st["copy_busy_ms"], 3)},
+                          "copy_GBps_while_copying": round(
+                              (st1["copies_total"] - st0["copies_total"]) * lay["l_size"] /
+                              max(1e-9, (st1["copy_ms_total"] - st0["copy_ms_total"]) / 1e3) / 1e9, 1),
+                          "copy_busy_frac": round((st1["copy_ms_total"] - st0["copy_ms_total"]) / 1e3 / dev_s, 4),
+                          "pool_blob_GBps_min_median": [round(st1["pool_min_GBps"], 1),
+                                                        round(st1["pool_median_GBps"], 1)],
+                          "pool_blobs_moved": st1["pool_replaced"]},
         "e2e": {"value": round(tokens / e2e_s, 4), "unit": "tokens/s", "h2d_bytes_per_step": 4 * Bsz,
                 "d2h_bytes_per_step": 4 * Bsz},
         "gpu_launches": per_step_launches * steps,
+        "step_ms": step_ms,
         "clocks": clk.summary(),
         "setup_s": {"create_and_weights": round(t_load, 1), "prefill": round(t_prefill, 1)},
     }

@@ -98,6 +98,11 @@ typedef struct loip_stats {
      * prefill: 6 qkv GEMM, 7 attention, 8 o-proj GEMM, 9 gate/up GEMM, 10 down GEMM, 11 RMSNorm */
     double kernel_ms[12];
     uint64_t kernel_launches[12];
+    double copy_ms_total;      /* summed duration of every completed layer copy (events) */
+    uint64_t copies_total;     /* number of completed layer copies */
+    double pool_min_GBps;      /* slowest host-pool blob copy when the pool was qualified */
+    double pool_median_GBps;   /* median blob copy rate at qualification */
+    uint64_t pool_replaced;    /* blobs moved to fresh host memory because they copied slowly */
 } loip_stats;
 
 typedef struct loip_ctx loip_ctx;
@@ -223,6 +228,12 @@ int loip_set_kernel_timing(loip_ctx* ctx, int32_t enable);
 /* Waits (with the context deadline) until all work of the context is done. */
 int loip_synchronize(loip_ctx* ctx);
 
+/* Host-link throughput as the layer copies see it: best of `reps` timed
+ * cudaMemcpyAsync of `bytes` (>= 1 MiB) from pinned, huge-page-backed host
+ * memory (the pool's allocator) to device memory on the current device.
+ * Allocates and frees its own buffers.  *out_Bps in bytes per second. */
+int loip_measure_h2d(uint64_t bytes, int32_t reps, double* out_Bps);
+
 /* Device pointer of the compute / copy stream (cudaStream_t). */
 void* loip_compute_stream(loip_ctx* ctx);
 void* loip_copy_stream(loip_ctx* ctx);
@@ -257,10 +268,12 @@ int loip_k_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int
  *   q (fp32 [B, Hq*d]); request b attends over its first ctx_lens[b] cached
  *   positions; page_offsets (dev int64 [B, max_pages]) gives each page's byte
  *   offset from kv_base; a page holds, for layer `layer`, K then V as
- *   [Hkv][page_tokens][d] bf16 at layer * layer_page_bytes inside the page.
- *   Writes o (fp32 [B, Hq*d]).  `scratch` (dev fp32, at least
- *   loip_k_attention_scratch_floats(...) floats) holds the per-chunk partial
- *   softmax states. */
+ *   [Hkv][page_tokens][d] bf16 at layer * layer_page_bytes inside the page
+ *   (page_tokens = 64; q, kv_base 16-byte aligned; max_ctx <= 16384).
+ *   Writes o (fp32 [B, Hq*d]).  `scratch` (dev, at least
+ *   loip_k_attention_scratch_floats(...) floats) holds the per-page partial
+ *   softmax states and per-(request, head) completion counters; it needs no
+ *   initialisation (the call zeroes the counters on `stream`). */
 int loip_k_attention(const float* q, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
                      const int32_t* ctx_lens, int32_t B, int32_t Hq, int32_t Hkv, int32_t d, int32_t page_tokens,
                      int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx, float* scratch, float* o,
@@ -276,16 +289,16 @@ uint64_t loip_k_attention_scratch_floats(int32_t B, int32_t Hq, int32_t d, int32
  * latency-critical path that must not pay the device-wide synchronisation of
  * cudaMalloc/cudaFree.  The paper has no counterpart; this is a library
  * convenience.  Same arguments and result as loip_k_attention without
- * `scratch`: the partial softmax states go to a file-scope device array of
- * LOIP_NOALLOC_SCRATCH_FLOATS floats that every GPU loading the library holds
- * until the process exits.  LOIP_ERR_INVALID when
- * B * Hq * ceil(max_ctx / page_tokens) * (d + 2) exceeds that size.  It
- * allocates nothing (no cudaMalloc, cudaFree or allocating library call).
- * The first call on a device, with that device current, looks up the array's
- * device address (cudaGetSymbolAddress); make that first call before any
- * stream capture.  All calls on a device share the array and it keeps the last
- * call's contents (nothing in it needs to start at zero): calls that overlap on
- * the GPU race. */
+ * `scratch`: the partial softmax states and completion counters go to a
+ * file-scope device array of LOIP_NOALLOC_SCRATCH_FLOATS floats that every GPU
+ * loading the library holds until the process exits.  LOIP_ERR_INVALID when
+ * loip_k_attention_scratch_floats(B, Hq, d, max_ctx, page_tokens) exceeds that
+ * size.  It allocates nothing (no cudaMalloc, cudaFree or allocating library
+ * call).  The first call on a device, with that device current, looks up the
+ * array's device address (cudaGetSymbolAddress); make that first call before
+ * any stream capture.  All calls on a device share the array and it keeps the
+ * last call's contents; each call clears the counters it needs on `stream`
+ * (cudaMemsetAsync) before its kernel: calls that overlap on the GPU race. */
 int loip_k_attention_noalloc(const float* q, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
                              const int32_t* ctx_lens, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
                              int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx, float* o,

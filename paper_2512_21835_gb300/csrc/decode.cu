@@ -25,6 +25,13 @@ namespace {
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
 constexpr int kStageFloats = 16384;  // 64 KB of staged activations per block
+constexpr int kMaxChunks = 256;      // pages per request in split attention (16384 positions)
+#ifndef LOIP_GEMV_MIN_BLOCKS1
+#define LOIP_GEMV_MIN_BLOCKS1 2  // resident blocks per SM the registers are sized for, batch tile 1
+#endif
+#ifndef LOIP_GEMV_JU1
+#define LOIP_GEMV_JU1 4  // 128-bit loads per row and batch at batch tile 1
+#endif
 
 __device__ __forceinline__ uint4 ld_stream(const uint16_t* p) {
     uint4 r;
@@ -189,7 +196,7 @@ __device__ __forceinline__ void load_batch(uint4 (&w)[4][U], const uint16_t* con
 template <int BT, int U, int EPI>
 __device__ __forceinline__ void unit_chunk(float (&acc)[U][BT], const uint16_t* const (&rp)[U], const bool (&rv)[U],
                                            const float* __restrict__ s, int kc0, int kn, int K, int lane) {
-    constexpr int JU = (BT <= 2) ? 4 : 2;
+    constexpr int JU = (BT == 1) ? LOIP_GEMV_JU1 : (BT == 2) ? 4 : 2;
     const int nj = (kn + 255) >> 8;
     uint4 wa[4][U], wb[4][U];
     load_batch<BT, U>(wa, rp, rv, kc0, 0, nj, K, lane, JU);
@@ -276,7 +283,7 @@ __device__ __forceinline__ void unit_epilogue(const GemvParams& p, int unit, flo
 }
 
 template <int BT, int EPI>
-__global__ void __launch_bounds__(kThreads, 2) gemv_kernel(GemvParams p) {
+__global__ void __launch_bounds__(kThreads, BT == 1 ? LOIP_GEMV_MIN_BLOCKS1 : 2) gemv_kernel(GemvParams p) {
     constexpr int U = UnitRows<EPI>::U;
     extern __shared__ __align__(16) float s_stage[];
     __shared__ float s_red[kWarps][BT];
@@ -311,20 +318,50 @@ __global__ void __launch_bounds__(kThreads, 2) gemv_kernel(GemvParams p) {
 #pragma unroll
     for (int b = 0; b < BT; ++b) best[b] = 0;
 
+    // Stages chunk [kc0, kc0 + KC) of every activation row: 16-byte loads, four
+    // per thread issued before any is consumed, so one L2 round trip covers
+    // 4 x 256 x 16 bytes; zeros pad the chunk to a multiple of 256 elements.
     auto stage = [&](int kc0) {
         const int kn = min(KC, K - kc0), kpad = (kn + 255) & ~255;
+        const int n4 = kpad >> 2;
+        constexpr int UN = 4;
 #pragma unroll
         for (int b = 0; b < BT; ++b) {
-            for (int k = tid; k < kpad; k += kThreads) {
-                float v = 0.f;
-                if (k < kn && b < p.B) {
-                    v = p.in[(size_t)b * K + kc0 + k];
+            for (int base = tid; base < n4; base += kThreads * UN) {
+                float4 v[UN];
+                uint2 gv[UN];
+#pragma unroll
+                for (int u = 0; u < UN; ++u) {
+                    const int k = (base + u * kThreads) * 4;
+                    const bool ok = k < kn && b < p.B;
+                    v[u] = ok ? *reinterpret_cast<const float4*>(p.in + (size_t)b * K + kc0 + k)
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
+                    gv[u] = (ok && norm) ? *reinterpret_cast<const uint2*>(p.g + kc0 + k) : make_uint2(0, 0);
+                }
+#pragma unroll
+                for (int u = 0; u < UN; ++u) {
+                    const int k = (base + u * kThreads) * 4;
+                    if (k >= kpad) continue;
+                    float4 w = v[u];
                     if (norm) {
-                        ss[b] = fmaf(v, v, ss[b]);
-                        v *= bf2f(p.g[kc0 + k]);
+                        ss[b] = fmaf(w.x, w.x, ss[b]);
+                        ss[b] = fmaf(w.y, w.y, ss[b]);
+                        ss[b] = fmaf(w.z, w.z, ss[b]);
+                        ss[b] = fmaf(w.w, w.w, ss[b]);
+                        w.x *= bf_lo(gv[u].x);
+                        w.y *= bf_hi(gv[u].x);
+                        w.z *= bf_lo(gv[u].y);
+                        w.w *= bf_hi(gv[u].y);
+                    }
+                    if (BT == 1) {
+                        *reinterpret_cast<float4*>(&s_stage[stage_index<1>(k, 0)]) = w;
+                    } else {
+                        s_stage[stage_index<BT>(k, b)] = w.x;
+                        s_stage[stage_index<BT>(k + 1, b)] = w.y;
+                        s_stage[stage_index<BT>(k + 2, b)] = w.z;
+                        s_stage[stage_index<BT>(k + 3, b)] = w.w;
                     }
                 }
-                s_stage[stage_index<BT>(k, b)] = v;
             }
         }
     };
@@ -465,24 +502,32 @@ cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, bool pdl, int* nblocks_o
         attr_set = true;
     }
     if (single) {
-        static int per_sm[4] = {0, 0, 0, 0};
+        // resident blocks per SM for this stage size (cached per batch tile and size)
+        static int cache_bt[16], cache_smem[16], cache_val[16], cache_n = 0;
         static int sms = 0;
-        int bi = BT == 1 ? 0 : BT == 2 ? 1 : BT == 4 ? 2 : 3;
-        if (per_sm[bi] == 0) {
+        int per_sm = 0;
+        for (int i = 0; i < cache_n; ++i)
+            if (cache_bt[i] == BT && cache_smem[i] == (int)smem) per_sm = cache_val[i];
+        if (per_sm == 0) {
             int dev;
             cudaGetDevice(&dev);
             cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
             int v = 0;
-            size_t sm_bytes = (size_t)kStageFloats * sizeof(float);
             switch (BT) {
-                case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<1, EPI>, kThreads, sm_bytes); break;
-                case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<2, EPI>, kThreads, sm_bytes); break;
-                case 4: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<4, EPI>, kThreads, sm_bytes); break;
-                default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<8, EPI>, kThreads, sm_bytes); break;
+                case 1: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<1, EPI>, kThreads, smem); break;
+                case 2: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<2, EPI>, kThreads, smem); break;
+                case 4: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<4, EPI>, kThreads, smem); break;
+                default: cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, gemv_kernel<8, EPI>, kThreads, smem); break;
             }
-            per_sm[bi] = v < 1 ? 1 : v;
+            per_sm = v < 1 ? 1 : v;
+            if (cache_n < 16) {
+                cache_bt[cache_n] = BT;
+                cache_smem[cache_n] = (int)smem;
+                cache_val[cache_n] = per_sm;
+                ++cache_n;
+            }
         }
-        int cap = per_sm[bi] * sms;
+        int cap = per_sm * sms;
         if (blocks > cap) blocks = cap;
     }
     if (blocks < 1) blocks = 1;
@@ -507,25 +552,48 @@ struct AttnParams {
     const int32_t* row_req;
     int B, Hq, Hkv, max_chunks;
     float scale;
-    float* scratch;  // split: [B][Hq][max_chunks][d + 2]
+    float* scratch;  // split: [B][Hq][max_chunks][d + 2] partial states, then int counters [B][Hq]
+    int* counters;
     void* o;         // [B, Hq*d] fp32 or bf16
     int o_bf16;
     int split;
 };
 
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+                 "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+
+// One block per (request row, kv head, page) in split mode, or per (row, kv
+// head) looping over the pages otherwise.  The page's keys and values (64
+// positions x d, bf16) are staged in shared memory with asynchronous 16-byte
+// copies, all in flight together; key rows are stored with their 16-byte chunks
+// rotated by the row index so that one-row-per-lane reads hit distinct banks.
+// Each of the two warps scores 32 positions for the G query heads of the kv
+// head (online softmax), then accumulates the values with the weights
+// broadcast by shuffles; the two warps merge through shared memory.
 template <int G, int D>
 __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
     constexpr int DPL = D / 32;  // dims per lane in the PV product
+    constexpr int CH = D / 8;    // 16-byte chunks per row
+    __shared__ __align__(16) uint16_t sK[64 * D];
+    __shared__ __align__(16) uint16_t sV[64 * D];
     __shared__ __align__(16) float sq[G][D];
     __shared__ float s_m[G], s_l[G];
     __shared__ float s_o[G][D];
+    __shared__ float s_w[G][kMaxChunks];  // combine weights of the per-page states
+    __shared__ int s_last;
 
     pdl_trigger();
     pdl_wait();
     const int row = blockIdx.z, kvh = blockIdx.y;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
-    const int P = p.kv.page_tokens;
+    const int P = p.kv.page_tokens;  // 64
     const int npages = (ctx + P - 1) / P;
     int pg0, pg1;
     if (p.split) {
@@ -537,9 +605,16 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
         pg1 = npages;
     }
     const int req = p.row_req ? p.row_req[row] : row;
-    for (int i = threadIdx.x; i < G * D; i += 64)
-        sq[i / D][i % D] = p.q[(size_t)row * p.Hq * D + (size_t)kvh * G * D + i];
-    __syncthreads();
+    {
+        const float4* qs = reinterpret_cast<const float4*>(p.q + (size_t)row * p.Hq * D + (size_t)kvh * G * D);
+        constexpr int NQ = G * D / 4 / 64;  // float4 per thread (G * D is a multiple of 256)
+        float4 qv[NQ > 0 ? NQ : 1];
+#pragma unroll
+        for (int u = 0; u < NQ; ++u) qv[u] = qs[tid + u * 64];
+#pragma unroll
+        for (int u = 0; u < NQ; ++u) reinterpret_cast<float4*>(&sq[0][0])[tid + u * 64] = qv[u];
+        if (NQ == 0 && tid < G * D / 4) reinterpret_cast<float4*>(&sq[0][0])[tid] = qs[tid];
+    }
 
     float m[G], l[G], o[G][DPL];
 #pragma unroll
@@ -551,54 +626,50 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
     }
     const int Hkv = p.Hkv;
     for (int pg = pg0; pg < pg1; ++pg) {
+        const int nvalid = min(P, ctx - pg * P);
         const char* page = p.kv.base + p.kv.page_offsets[(int64_t)req * p.kv.max_pages + pg] +
                            (uint64_t)p.kv.layer * p.kv.layer_page_bytes;
         const uint16_t* Kh = reinterpret_cast<const uint16_t*>(page) + (size_t)kvh * P * D;
         const uint16_t* Vh = reinterpret_cast<const uint16_t*>(page) + ((size_t)Hkv + kvh) * P * D;
-        for (int t0 = warp * 32; t0 < P; t0 += 64) {
-            const int tl = t0 + lane;
-            const bool valid = (pg * P + tl) < ctx && tl < P;
-            const int nt = min(32, min(P - t0, ctx - (pg * P + t0)));
-            // every K row (one per lane) and every V slice of the 32 tokens in flight at once
-            uint4 kk[D / 8];
-            const uint4* kr = reinterpret_cast<const uint4*>(Kh + (size_t)(valid ? tl : t0) * D);
-#pragma unroll
-            for (int u = 0; u < D / 8; ++u) kk[u] = valid ? kr[u] : make_uint4(0, 0, 0, 0);
-            uint32_t vv[32][DPL / 2];
-#pragma unroll
-            for (int u = 0; u < 32; ++u) {
-                const uint16_t* vr = Vh + (size_t)(t0 + u) * D + lane * DPL;
-                const bool ok = u < nt;
-                if constexpr (DPL == 4) {
-                    uint2 v2 = ok ? *reinterpret_cast<const uint2*>(vr) : make_uint2(0, 0);
-                    vv[u][0] = v2.x;
-                    vv[u][1] = v2.y;
-                } else {
-                    static_assert(DPL == 2, "head_dim 64 or 128");
-                    vv[u][0] = ok ? *reinterpret_cast<const uint32_t*>(vr) : 0u;
-                }
+        if (pg != pg0) __syncthreads();  // the previous page's rows are no longer read
+        for (int i = tid; i < 64 * CH; i += 64) {
+            const int t = i / CH, c = i - t * CH;
+            if (t < nvalid) {
+                cp_async16(&sK[(t * CH + ((c + t) & (CH - 1))) * 8], Kh + (size_t)t * D + c * 8);
+                cp_async16(&sV[(t * CH + c) * 8], Vh + (size_t)t * D + c * 8);
+            } else {
+                *reinterpret_cast<uint4*>(&sV[(t * CH + c) * 8]) = make_uint4(0, 0, 0, 0);
             }
+        }
+        cp_async_wait_all();
+        __syncthreads();
+        {
+            const int tl = warp * 32 + lane;
+            const bool valid = tl < nvalid;
             float s[G];
 #pragma unroll
             for (int g = 0; g < G; ++g) s[g] = 0.f;
+            if (valid) {
+#pragma unroll 4
+                for (int u = 0; u < CH; ++u) {
+                    const uint4 kk = *reinterpret_cast<const uint4*>(&sK[(tl * CH + ((u + tl) & (CH - 1))) * 8]);
+                    const float kf[8] = {bf_lo(kk.x), bf_hi(kk.x), bf_lo(kk.y), bf_hi(kk.y),
+                                         bf_lo(kk.z), bf_hi(kk.z), bf_lo(kk.w), bf_hi(kk.w)};
 #pragma unroll
-            for (int u = 0; u < D / 8; ++u) {
-                const float kf[8] = {bf_lo(kk[u].x), bf_hi(kk[u].x), bf_lo(kk[u].y), bf_hi(kk[u].y),
-                                     bf_lo(kk[u].z), bf_hi(kk[u].z), bf_lo(kk[u].w), bf_hi(kk[u].w)};
-#pragma unroll
-                for (int g = 0; g < G; ++g) {
-                    const float4 qa = *reinterpret_cast<const float4*>(&sq[g][u * 8]);
-                    const float4 qb = *reinterpret_cast<const float4*>(&sq[g][u * 8 + 4]);
-                    float a = s[g];
-                    a = fmaf(qa.x, kf[0], a);
-                    a = fmaf(qa.y, kf[1], a);
-                    a = fmaf(qa.z, kf[2], a);
-                    a = fmaf(qa.w, kf[3], a);
-                    a = fmaf(qb.x, kf[4], a);
-                    a = fmaf(qb.y, kf[5], a);
-                    a = fmaf(qb.z, kf[6], a);
-                    a = fmaf(qb.w, kf[7], a);
-                    s[g] = a;
+                    for (int g = 0; g < G; ++g) {
+                        const float4 qa = *reinterpret_cast<const float4*>(&sq[g][u * 8]);
+                        const float4 qb = *reinterpret_cast<const float4*>(&sq[g][u * 8 + 4]);
+                        float a = s[g];
+                        a = fmaf(qa.x, kf[0], a);
+                        a = fmaf(qa.y, kf[1], a);
+                        a = fmaf(qa.z, kf[2], a);
+                        a = fmaf(qa.w, kf[3], a);
+                        a = fmaf(qb.x, kf[4], a);
+                        a = fmaf(qb.y, kf[5], a);
+                        a = fmaf(qb.z, kf[6], a);
+                        a = fmaf(qb.w, kf[7], a);
+                        s[g] = a;
+                    }
                 }
             }
             float pe[G];
@@ -614,13 +685,21 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
                 for (int c = 0; c < DPL; ++c) o[g][c] *= corr;
                 m[g] = mn;
             }
-#pragma unroll
-            for (int u = 0; u < 32; ++u) {
+            const int nt = min(32, nvalid - warp * 32);
+            for (int u = 0; u < nt; ++u) {
+                const uint16_t* vr = &sV[(warp * 32 + u) * D + lane * DPL];
                 float vf[DPL];
-#pragma unroll
-                for (int c = 0; c < DPL / 2; ++c) {
-                    vf[2 * c] = bf_lo(vv[u][c]);
-                    vf[2 * c + 1] = bf_hi(vv[u][c]);
+                if constexpr (DPL == 4) {
+                    const uint2 vv = *reinterpret_cast<const uint2*>(vr);
+                    vf[0] = bf_lo(vv.x);
+                    vf[1] = bf_hi(vv.x);
+                    vf[2] = bf_lo(vv.y);
+                    vf[3] = bf_hi(vv.y);
+                } else {
+                    static_assert(DPL == 2, "head_dim 64 or 128");
+                    const uint32_t vv = *reinterpret_cast<const uint32_t*>(vr);
+                    vf[0] = bf_lo(vv);
+                    vf[1] = bf_hi(vv);
                 }
 #pragma unroll
                 for (int g = 0; g < G; ++g) {
@@ -675,41 +754,59 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
             }
         }
     }
-}
-
-// Combines the per-page partial softmax states of one (row, head).
-__global__ void attn_combine_kernel(AttnParams p, int D) {
-    pdl_trigger();
-    pdl_wait();
-    const int h = blockIdx.x, row = blockIdx.y, j = threadIdx.x;
-    const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
-    const int n = (ctx + p.kv.page_tokens - 1) / p.kv.page_tokens;
-    const float* part = p.scratch + ((size_t)row * p.Hq + h) * p.max_chunks * (D + 2);
-    float M = -INFINITY;
-#pragma unroll 8
-    for (int c = 0; c < n; ++c) M = fmaxf(M, part[(size_t)c * (D + 2) + D]);
-    float L = 0.f, acc = 0.f;
-#pragma unroll 8
-    for (int c = 0; c < n; ++c) {
-        const float* pc = part + (size_t)c * (D + 2);
-        float w = (pc[D] == -INFINITY) ? 0.f : expf(pc[D] - M);
-        L += pc[D + 1] * w;
-        acc += pc[j] * w;
+    if (!p.split) return;
+    // The last block of this (row, kv head) to finish combines every page's
+    // state: exp-weighted sum of the partial outputs over the summed weights.
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+        int* cnt = p.counters + (size_t)row * p.Hq + kvh;
+        const int ticket = atomicAdd(cnt, 1);
+        s_last = ticket == npages - 1;
+        if (s_last) atomicExch(cnt, 0);  // every block of the group has arrived: reset for the next launch
     }
-    float v = L > 0.f ? acc / L : 0.f;
-    size_t idx = (size_t)row * p.Hq * D + (size_t)h * D + j;
-    if (p.o_bf16)
-        reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(v);
-    else
-        reinterpret_cast<float*>(p.o)[idx] = v;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    const float* base = p.scratch + ((size_t)row * p.Hq + (size_t)kvh * G) * p.max_chunks * (D + 2);
+    for (int g = warp; g < G; g += 2) {
+        const float* ph = base + (size_t)g * p.max_chunks * (D + 2);
+        float mx = -INFINITY;
+        for (int c = lane; c < npages; c += 32) {
+            const float mc = ph[(size_t)c * (D + 2) + D];
+            s_w[g][c] = mc;
+            mx = fmaxf(mx, mc);
+        }
+        mx = warp_max(mx);
+        float lsum = 0.f;
+        for (int c = lane; c < npages; c += 32) {
+            const float w = (s_w[g][c] == -INFINITY) ? 0.f : expf(s_w[g][c] - mx);
+            s_w[g][c] = w;
+            lsum = fmaf(ph[(size_t)c * (D + 2) + D + 1], w, lsum);
+        }
+        lsum = warp_sum(lsum);
+        const float inv = lsum > 0.f ? 1.0f / lsum : 0.f;
+        for (int c = lane; c < npages; c += 32) s_w[g][c] *= inv;
+    }
+    __syncthreads();
+    for (int e = tid; e < G * D; e += 64) {
+        const int g = e / D, j = e - g * D;
+        const float* ph = base + (size_t)g * p.max_chunks * (D + 2) + j;
+        float acc = 0.f;
+#pragma unroll 8
+        for (int c = 0; c < npages; ++c) acc = fmaf(ph[(size_t)c * (D + 2)], s_w[g][c], acc);
+        const size_t idx = (size_t)row * p.Hq * D + (size_t)(kvh * G + g) * D + j;
+        if (p.o_bf16)
+            reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(acc);
+        else
+            reinterpret_cast<float*>(p.o)[idx] = acc;
+    }
 }
 
 template <int G, int D>
 cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st, bool pdl) {
     dim3 grid(p.split ? p.max_chunks : 1, p.Hkv, p.B);
-    cudaError_t e = launch_k(attn_kernel<G, D>, grid, dim3(64), 0, st, pdl, p);
-    if (e != cudaSuccess || !p.split) return e;
-    return launch_k(attn_combine_kernel, dim3(p.Hq, p.B), dim3(D), 0, st, pdl, p, D);
+    return launch_k(attn_kernel<G, D>, grid, dim3(64), 0, st, pdl, p);
 }
 
 // ----------------------------------------------------------------------------
@@ -855,9 +952,17 @@ cudaError_t launch_lm_head(const float* x, const uint16_t* g, const uint16_t* w,
                     tokens);
 }
 
-size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens) {
+static size_t attention_partial_floats(int B, int Hq, int d, int max_ctx, int page_tokens) {
     size_t chunks = ((size_t)max_ctx + page_tokens - 1) / page_tokens;
-    return (size_t)B * Hq * chunks * (d + 2);
+    return ((size_t)B * Hq * chunks * (d + 2) + 63) / 64 * 64;
+}
+
+size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens) {
+    return attention_partial_floats(B, Hq, d, max_ctx, page_tokens) + (size_t)B * Hq;  // + int counters
+}
+
+int* attention_counters(float* scratch, int B, int Hq, int d, int max_ctx, int page_tokens) {
+    return reinterpret_cast<int*>(scratch + attention_partial_floats(B, Hq, d, max_ctx, page_tokens));
 }
 
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
@@ -873,8 +978,10 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
     p.Hq = Hq;
     p.Hkv = Hkv;
     p.max_chunks = (max_ctx + kv.page_tokens - 1) / kv.page_tokens;
+    if (split && p.max_chunks > kMaxChunks) return cudaErrorInvalidValue;
     p.scale = 1.0f / sqrtf((float)d);
     p.scratch = scratch;
+    p.counters = split ? attention_counters(scratch, B, Hq, d, max_ctx, kv.page_tokens) : nullptr;
     p.o = o;
     p.o_bf16 = o_bf16 ? 1 : 0;
     p.split = split ? 1 : 0;
@@ -911,8 +1018,8 @@ cudaError_t launch_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t 
     if (n == 0) return cudaSuccess;
     uint64_t blocks = (n + 255) / 256;
     if (blocks > 152 * 32) blocks = 152 * 32;
-    generate_kernel<<<(unsigned)blocks, 256, 0, st>>>(out, n, first, seed, tensor_id, kind);
-    return cudaGetLastError();
+    return launch_k(generate_kernel, dim3((unsigned)blocks), dim3(256), 0, st, false, out, n, first, seed, tensor_id,
+                    kind);
 }
 
 }  // namespace loip

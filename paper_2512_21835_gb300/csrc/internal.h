@@ -53,13 +53,18 @@ size_t lm_head_scratch_bytes(int B, int V);
 // Grouped-query attention over the paged cache.  Rows b = 0..B-1 attend over
 // their first ctx_lens[b] positions with query q[b] (ctx_lens NULL: over
 // positions[b] + 1 positions, the causal window of the token at positions[b]).  row_req maps a row to its
-// page-table row (NULL = identity).  split: partial states go to scratch and a
-// combine kernel writes o; otherwise one block per (row, kv head) loops over all
-// pages.  o_bf16: write o as bf16 (prefill) instead of fp32.
+// page-table row (NULL = identity).  split: one block per page writes its
+// partial state to scratch and the last block of each (row, kv head) combines
+// them into o (max_ctx <= 16384); otherwise one block per (row, kv head) loops
+// over all pages.  o_bf16: write o as bf16 (prefill) instead of fp32.
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
                              float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl = false);
 size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens);
+// Split attention keeps one int completion counter per (row, head) after the
+// partial states; they must be zero before a launch and every launch leaves
+// them zero.
+int* attention_counters(float* scratch, int B, int Hq, int d, int max_ctx, int page_tokens);
 
 cudaError_t launch_embed(const uint16_t* embed, const int32_t* tokens, int B, int H, int V, float* x,
                          cudaStream_t st, bool pdl = false);

@@ -55,16 +55,22 @@ extern "C" int loip_k_attention_noalloc(const float* q, const void* kv_base, con
                                         int32_t d, int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes,
                                         int32_t max_ctx, float* o, void* stream) {
     if (!q || !kv_base || !page_offsets || !ctx_lens || !o || B < 1 || Hq < 1 || Hkv < 1 || (d != 64 && d != 128) ||
-        Hq % Hkv || max_ctx < 1 || page_tokens < 1 || (int64_t)max_pages * page_tokens < max_ctx)
+        Hq % Hkv || max_ctx < 1 || page_tokens != 64 || (int64_t)max_pages * page_tokens < max_ctx)
         return LOIP_ERR_INVALID;
-    if (attention_scratch_floats(B, Hq, d, max_ctx, page_tokens) > LOIP_NOALLOC_SCRATCH_FLOATS)
-        return LOIP_ERR_INVALID;  // B * Hq * ceil(max_ctx / page_tokens) * (d + 2) floats do not fit
+    if (attention_scratch_floats(B, Hq, d, max_ctx, page_tokens) > LOIP_NOALLOC_SCRATCH_FLOATS ||
+        (max_ctx + page_tokens - 1) / page_tokens > 256)
+        return LOIP_ERR_INVALID;  // the partial states and counters do not fit
     float* scratch = nullptr;
     if (scratch_for_current_device(&scratch) != cudaSuccess) return LOIP_ERR_CUDA;
-    // Nothing in the scratch has to start at zero: every partial state the
-    // combine step reads is written by the same launch first.
+    // The completion counters behind the partial states must start at zero
+    // (a launch leaves them zero; clearing them here also covers the first call
+    // and any earlier call that was cut short).  The partial states themselves
+    // are written by the same launch before they are read.
     KvView kv{(char*)kv_base, page_offsets, max_pages, page_tokens, layer, layer_page_bytes};
-    cudaError_t e = launch_attention(q, kv, ctx_lens, nullptr, nullptr, B, Hq, Hkv, d, max_ctx, true, scratch, o,
+    cudaError_t e = cudaMemsetAsync(attention_counters(scratch, B, Hq, d, max_ctx, page_tokens), 0,
+                                    (size_t)B * Hq * sizeof(int), (cudaStream_t)stream);
+    if (e != cudaSuccess) return LOIP_ERR_CUDA;
+    e = launch_attention(q, kv, ctx_lens, nullptr, nullptr, B, Hq, Hkv, d, max_ctx, true, scratch, o,
                                      false, (cudaStream_t)stream);
     return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA;
 }

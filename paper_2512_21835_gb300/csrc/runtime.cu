@@ -27,6 +27,7 @@
 #include <vector>
 
 #include "../../include/loip.h"
+#include "hostpool.h"
 #include "internal.h"
 #include "plan.h"
 
@@ -164,8 +165,9 @@ struct loip_ctx {
     std::vector<Request> reqs;
     int max_pages = 0;
     bool pt_dirty = true;
-    // host pool
+    // host pool: blobs of offloaded layers inside pinned huge-page regions
     std::vector<void*> host_layer;
+    std::vector<HostBuf> host_regions;
     int32_t* h_stage = nullptr;  // pinned staging for small transfers
     size_t h_stage_ints = 0;
     int64_t* h_pt = nullptr;     // pinned page-table staging
@@ -202,6 +204,7 @@ struct loip_ctx {
     int cuda_fail(cudaError_t e, const char* what) {
         err = std::string(what) + ": " + cudaGetErrorString(e);
         if (e != cudaErrorNotReady) failed = true;
+        cudaGetLastError();  // a non-sticky error must not surface again in a later, unrelated launch
         return LOIP_ERR_CUDA;
     }
     template <class T>
@@ -525,6 +528,8 @@ struct loip_ctx {
             float ms = 0;
             cudaEventElapsedTime(&ms, pr.first, pr.second);
             busy += ms;
+            st.copy_ms_total += ms;
+            st.copies_total += 1;
             event_pool.push_back(pr.first);
             event_pool.push_back(pr.second);
             copy_events.pop_front();
@@ -568,11 +573,11 @@ struct loip_ctx {
 
     int demote_layer(int l) {
         if (!host_layer[l]) {
-            cudaError_t e = cudaHostAlloc(&host_layer[l], lay.l_size, cudaHostAllocDefault);
-            if (e != cudaSuccess) {
-                host_layer[l] = nullptr;
-                return fail(LOIP_ERR_OOM, "pinned allocation for a demoted layer failed");
-            }
+            HostBuf hb;
+            cudaError_t e = host_buf_alloc(lay.l_size, &hb);
+            if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned allocation for a demoted layer failed");
+            host_regions.push_back(hb);
+            host_layer[l] = hb.ptr;
             e = cudaMemcpy(host_layer[l], block_ptr(layer_block[l]), lay.l_size, cudaMemcpyDeviceToHost);
             if (e != cudaSuccess) return cuda_fail(e, "demote copy");
         }
@@ -582,6 +587,77 @@ struct loip_ctx {
         layer_block[l] = -1;
         offloaded[l] = 1;
         return LOIP_OK;
+    }
+
+    // Times one copy of every offloaded layer's host blob into slot 0 and moves
+    // blobs that copy clearly slower than the pool's median (pages the host
+    // could not back with huge pages copy at a fraction of the link rate) to a
+    // fresh buffer, keeping the slow memory reserved while retrying so it is not
+    // handed back.  At most 3 attempts per blob; the fastest buffer wins.
+    int qualify_host_pool() {
+        if (off_order.empty()) return LOIP_OK;
+        cudaEvent_t a = take_event(), b = take_event();
+        auto rate = [&](const void* src, double* gbps) -> int {
+            cudaEventRecord(a, compute);
+            cudaError_t e = cudaMemcpyAsync(slot_ptr(0), src, lay.l_size, cudaMemcpyHostToDevice, compute);
+            cudaEventRecord(b, compute);
+            if (e == cudaSuccess) e = cudaEventSynchronize(b);
+            float ms = 0;
+            if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, a, b);
+            if (e != cudaSuccess) return cuda_fail(e, "pool qualification copy");
+            *gbps = ms > 0 ? (double)lay.l_size / (ms * 1e-3) / 1e9 : 0.0;
+            return LOIP_OK;
+        };
+        std::vector<double> r(L, 0.0);
+        for (int l : off_order) {
+            int rc = rate(host_layer[l], &r[l]);
+            if (rc) return rc;
+        }
+        std::vector<double> sorted;
+        for (int l : off_order) sorted.push_back(r[l]);
+        std::sort(sorted.begin(), sorted.end());
+        const double median = sorted[sorted.size() / 2];
+        std::vector<HostBuf> spare;  // rejected buffers, released after the search
+        for (int l : off_order) {
+            for (int attempt = 0; attempt < 3 && r[l] < 0.9 * median; ++attempt) {
+                HostBuf hb;
+                if (host_buf_alloc(lay.l_size, &hb) != cudaSuccess) break;
+                double g = 0;
+                int rc = rate(hb.ptr, &g);
+                if (rc) return rc;
+                if (g > r[l]) {
+                    host_regions.push_back(hb);
+                    host_layer[l] = hb.ptr;
+                    r[l] = g;
+                    st.pool_replaced += 1;
+                } else {
+                    spare.push_back(hb);
+                }
+            }
+        }
+        for (auto& hb : spare) host_buf_free(&hb);
+        double mn = 1e30;
+        for (int l : off_order) mn = std::min(mn, r[l]);
+        st.pool_min_GBps = mn;
+        st.pool_median_GBps = median;
+        event_pool.push_back(a);
+        event_pool.push_back(b);
+        return LOIP_OK;
+    }
+
+    // One pinned region for every offloaded layer that has no host copy yet.
+    int ensure_host_pool() {
+        std::vector<int> need;
+        for (int l = 0; l < L; ++l)
+            if (offloaded[l] && !host_layer[l]) need.push_back(l);
+        if (need.empty()) return LOIP_OK;
+        HostBuf b;
+        cudaError_t e = host_buf_alloc(need.size() * lay.l_size, &b);
+        if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
+        host_regions.push_back(b);
+        for (size_t i = 0; i < need.size(); ++i)
+            host_layer[need[i]] = static_cast<char*>(b.ptr) + i * lay.l_size;
+        return qualify_host_pool();
     }
 
     uint64_t arena_used() const {
@@ -623,8 +699,7 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
     if (!ctx) return;
     if (ctx->compute) cudaStreamSynchronize(ctx->compute);
     if (ctx->copy) cudaStreamSynchronize(ctx->copy);
-    for (void* p : ctx->host_layer)
-        if (p) cudaFreeHost(p);
+    for (auto& hb : ctx->host_regions) host_buf_free(&hb);
     if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
     if (ctx->h_pt) cudaFreeHost(ctx->h_pt);
     for (auto e : ctx->slot_full) cudaEventDestroy(e);
@@ -655,6 +730,7 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     }
     loip_config cfg = normalized(cfg_in);
     if (cfg.n_slots < 1 || cfg.n_slots > 3 || cfg.max_batch < 1 || cfg.max_batch > 8 || cfg.max_ctx < 1 ||
+        cfg.max_ctx > 16384 ||
         cfg.page_tokens != 64 || !device_arena || ((uintptr_t)device_arena % kAlign) ||
         arena_bytes < cfg.device_budget_bytes || (cfg.mode != LOIP_MODE_OVERLAP && cfg.mode != LOIP_MODE_NAIVE)) {
         g_create_error = "invalid configuration (slots 1..3, batch 1..8, page 64, arena >= budget, aligned)";
@@ -769,6 +845,16 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
         loip_destroy(c);
         return LOIP_ERR_CUDA;
     }
+    // attention completion counters start at zero (each launch leaves them zero)
+    e = cudaMemsetAsync(c->arena + c->fx.attn_scratch, 0,
+                        attention_scratch_floats(cfg.max_batch, c->Hq, c->d, cfg.max_ctx, cfg.page_tokens) * 4,
+                        c->compute);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->compute);
+    if (e != cudaSuccess) {
+        g_create_error = std::string("CUDA setup failed: ") + cudaGetErrorString(e);
+        loip_destroy(c);
+        return LOIP_ERR_CUDA;
+    }
     c->st.n_resident = c->L - (int)c->off_order.size();
     c->st.n_offloaded = (int)c->off_order.size();
     *out = c;
@@ -834,13 +920,8 @@ extern "C" int loip_load_weights_generated(loip_ctx* c, uint64_t seed) {
             rc = write_layer_generated(c, c->block_ptr(c->layer_block[l]), l, seed);
             if (rc) return rc;
         } else {
-            if (!c->host_layer[l]) {
-                e = cudaHostAlloc(&c->host_layer[l], c->lay.l_size, cudaHostAllocDefault);
-                if (e != cudaSuccess) {
-                    c->host_layer[l] = nullptr;
-                    return c->fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
-                }
-            }
+            rc = c->ensure_host_pool();
+            if (rc) return rc;
             char* tmp = c->slot_ptr(0);
             rc = write_layer_generated(c, tmp, l, seed);
             if (rc) return rc;
@@ -862,18 +943,13 @@ extern "C" int loip_load_layer(loip_ctx* c, int32_t layer, const void* host_blob
         return c->fail(LOIP_ERR_INVALID, "layer index or blob size");
     int rc = c->sync_all();
     if (rc) return rc;
+    rc = c->ensure_host_pool();  // every offloaded layer gets its pool blob before the ring is primed
+    if (rc) return rc;
     cudaError_t e;
     if (c->layer_block[layer] >= 0) {
         e = cudaMemcpy(c->block_ptr(c->layer_block[layer]), host_blob, bytes, cudaMemcpyHostToDevice);
         if (e != cudaSuccess) return c->cuda_fail(e, "layer upload");
     } else {
-        if (!c->host_layer[layer]) {
-            e = cudaHostAlloc(&c->host_layer[layer], bytes, cudaHostAllocDefault);
-            if (e != cudaSuccess) {
-                c->host_layer[layer] = nullptr;
-                return c->fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
-            }
-        }
         memcpy(c->host_layer[layer], host_blob, bytes);
     }
     c->weights_loaded = true;
@@ -1192,6 +1268,38 @@ extern "C" int loip_set_kernel_timing(loip_ctx* c, int32_t enable) {
     return LOIP_OK;
 }
 
+extern "C" int loip_measure_h2d(uint64_t bytes, int32_t reps, double* out_Bps) {
+    if (!out_Bps || bytes < (1u << 20) || reps < 1) return LOIP_ERR_INVALID;
+    HostBuf hb;
+    if (host_buf_alloc(bytes, &hb) != cudaSuccess) return LOIP_ERR_OOM;
+    memset(hb.ptr, 1, bytes);
+    void* d = nullptr;
+    cudaStream_t s = nullptr;
+    cudaEvent_t a = nullptr, b = nullptr;
+    cudaError_t e = cudaMalloc(&d, bytes);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreate(&a);
+    if (e == cudaSuccess) e = cudaEventCreate(&b);
+    double best = 0;
+    for (int r = 0; r < reps + 1 && e == cudaSuccess; ++r) {
+        cudaEventRecord(a, s);
+        e = cudaMemcpyAsync(d, hb.ptr, bytes, cudaMemcpyHostToDevice, s);
+        cudaEventRecord(b, s);
+        if (e == cudaSuccess) e = cudaEventSynchronize(b);
+        float ms = 0;
+        if (e == cudaSuccess && r > 0 && cudaEventElapsedTime(&ms, a, b) == cudaSuccess && ms > 0)
+            best = std::max(best, (double)bytes / (ms * 1e-3));
+    }
+    if (a) cudaEventDestroy(a);
+    if (b) cudaEventDestroy(b);
+    if (s) cudaStreamDestroy(s);
+    if (d) cudaFree(d);
+    host_buf_free(&hb);
+    if (e != cudaSuccess) return LOIP_ERR_CUDA;
+    *out_Bps = best;
+    return LOIP_OK;
+}
+
 extern "C" void* loip_compute_stream(loip_ctx* c) { return c ? (void*)c->compute : nullptr; }
 extern "C" void* loip_copy_stream(loip_ctx* c) { return c ? (void*)c->copy : nullptr; }
 
@@ -1199,7 +1307,11 @@ extern "C" void* loip_copy_stream(loip_ctx* c) { return c ? (void*)c->copy : nul
 // Kernel-level entry points
 // ============================================================================
 static bool al16(const void* p) { return ((uintptr_t)p & 15) == 0; }
-static int cerr(cudaError_t e) { return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA; }
+static int cerr(cudaError_t e) {
+    if (e == cudaSuccess) return LOIP_OK;
+    cudaGetLastError();  // leave no non-sticky error behind for the next call
+    return LOIP_ERR_CUDA;
+}
 
 extern "C" int loip_k_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id,
                                int32_t kind, void* stream) {
@@ -1218,7 +1330,7 @@ extern "C" int loip_k_qkv_rope(const float* x, const uint16_t* g, const uint16_t
                                float* q_out, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
                                int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, void* stream) {
     if (!x || !g || !wqkv || !positions || !q_out || !kv_base || !page_offsets || B < 1 || B > 8 || H % 8 ||
-        (d != 64 && d != 128) || Hq % Hkv || page_tokens < 1 || !al16(wqkv) || !al16(x))
+        (d != 64 && d != 128) || Hq % Hkv || page_tokens < 1 || !al16(wqkv) || !al16(x) || ((uintptr_t)g & 7))
         return LOIP_ERR_INVALID;
     KvView kv{(char*)kv_base, page_offsets, max_pages, page_tokens, layer, layer_page_bytes};
     return cerr(launch_qkv_rope(x, g, wqkv, B, H, Hq, Hkv, d, eps, theta, positions, q_out, kv, nullptr,
@@ -1236,29 +1348,35 @@ extern "C" int loip_k_attention(const float* q, const void* kv_base, const int64
                                 int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx,
                                 float* scratch, float* o, void* stream) {
     if (!q || !kv_base || !page_offsets || !ctx_lens || !scratch || !o || B < 1 || (d != 64 && d != 128) ||
-        Hq % Hkv || max_ctx < 1 || page_tokens < 1 || (int64_t)max_pages * page_tokens < max_ctx)
+        Hq % Hkv || max_ctx < 1 || page_tokens != 64 || (int64_t)max_pages * page_tokens < max_ctx || !al16(q) ||
+        ((uintptr_t)kv_base & 15))
         return LOIP_ERR_INVALID;
+    if ((max_ctx + page_tokens - 1) / page_tokens > 256) return LOIP_ERR_INVALID;
     KvView kv{(char*)kv_base, page_offsets, max_pages, page_tokens, layer, layer_page_bytes};
+    cudaError_t e = cudaMemsetAsync(attention_counters(scratch, B, Hq, d, max_ctx, page_tokens), 0,
+                                    (size_t)B * Hq * sizeof(int), (cudaStream_t)stream);
+    if (e != cudaSuccess) return LOIP_ERR_CUDA;
     return cerr(launch_attention(q, kv, ctx_lens, nullptr, nullptr, B, Hq, Hkv, d, max_ctx, true, scratch, o, false,
                                  (cudaStream_t)stream));
 }
 
 extern "C" int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x,
                             void* stream) {
-    if (!o || !wo || !x || B < 1 || B > 8 || K % 8 || H < 1 || !al16(wo)) return LOIP_ERR_INVALID;
+    if (!o || !wo || !x || B < 1 || B > 8 || K % 8 || H < 1 || !al16(wo) || !al16(o)) return LOIP_ERR_INVALID;
     return cerr(launch_resid_gemv(o, wo, B, H, K, x, (cudaStream_t)stream));
 }
 
 extern "C" int loip_k_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int32_t B,
                               int32_t H, int32_t F, float eps, float* a, void* stream) {
-    if (!x || !g || !wg || !wu || !a || B < 1 || B > 8 || H % 8 || F < 1 || !al16(wg) || !al16(wu))
+    if (!x || !g || !wg || !wu || !a || B < 1 || B > 8 || H % 8 || F < 1 || !al16(wg) || !al16(wu) || !al16(x) ||
+        ((uintptr_t)g & 7))
         return LOIP_ERR_INVALID;
     return cerr(launch_gate_up(x, g, wg, wu, B, H, F, eps, a, (cudaStream_t)stream));
 }
 
 extern "C" int loip_k_down(const float* a, const uint16_t* wd, int32_t B, int32_t H, int32_t F, float* x,
                            void* stream) {
-    if (!a || !wd || !x || B < 1 || B > 8 || F % 8 || H < 1 || !al16(wd)) return LOIP_ERR_INVALID;
+    if (!a || !wd || !x || B < 1 || B > 8 || F % 8 || H < 1 || !al16(wd) || !al16(a)) return LOIP_ERR_INVALID;
     return cerr(launch_resid_gemv(a, wd, B, H, F, x, (cudaStream_t)stream));
 }
 
@@ -1284,7 +1402,8 @@ extern "C" uint64_t loip_k_lm_head_scratch_bytes(int32_t B, int32_t V) {
 extern "C" int loip_k_lm_head(const float* x, const uint16_t* g_final, const uint16_t* lm_head, int32_t B, int32_t H,
                               int32_t V, float eps, float* z, float* logits, int32_t* tokens, void* scratch,
                               void* stream) {
-    if (!x || !g_final || !lm_head || !tokens || !scratch || B < 1 || B > 8 || H % 8 || V < 1 || !al16(lm_head))
+    if (!x || !g_final || !lm_head || !tokens || !scratch || B < 1 || B > 8 || H % 8 || V < 1 || !al16(lm_head) ||
+        !al16(x) || ((uintptr_t)g_final & 7))
         return LOIP_ERR_INVALID;
     return cerr(launch_lm_head(x, g_final, lm_head, B, H, V, eps, z, logits, tokens, scratch, (cudaStream_t)stream));
 }

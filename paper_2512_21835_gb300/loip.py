@@ -55,7 +55,9 @@ class Stats(C.Structure):
                 ("last_step_ms", C.c_double), ("copy_busy_ms", C.c_double), ("compute_ms", C.c_double),
                 ("n_resident", C.c_int32), ("n_offloaded", C.c_int32), ("n_replans", C.c_int32),
                 ("kv_tokens", C.c_uint64), ("kv_bytes", C.c_uint64), ("arena_used", C.c_uint64),
-                ("kernel_ms", C.c_double * 12), ("kernel_launches", C.c_uint64 * 12)]
+                ("kernel_ms", C.c_double * 12), ("kernel_launches", C.c_uint64 * 12),
+                ("copy_ms_total", C.c_double), ("copies_total", C.c_uint64),
+                ("pool_min_GBps", C.c_double), ("pool_median_GBps", C.c_double), ("pool_replaced", C.c_uint64)]
 
 
 P, U64, I32, U32, F32, F64, VP = C.c_void_p, C.c_uint64, C.c_int32, C.c_uint32, C.c_float, C.c_double, C.c_void_p
@@ -81,6 +83,7 @@ _SIGS = {
     "loip_get_stats": (C.c_int, [P, C.POINTER(Stats)]),
     "loip_synchronize": (C.c_int, [P]),
     "loip_set_kernel_timing": (C.c_int, [P, I32]),
+    "loip_measure_h2d": (C.c_int, [U64, I32, C.POINTER(C.c_double)]),
     "loip_compute_stream": (C.c_void_p, [P]),
     "loip_copy_stream": (C.c_void_p, [P]),
     "loip_k_generate": (C.c_int, [P, U64, U64, U64, U32, I32, P]),
@@ -176,6 +179,13 @@ def loip_plan_residency(m: dict, layer_bytes, budget: int, kv_bytes: int, fixed_
 def loip_kv_threshold(left_bytes: int, kv_bytes_per_token: int) -> int:
     out = C.c_uint64()
     _check(lib().loip_kv_threshold(left_bytes, kv_bytes_per_token, C.byref(out)))
+    return out.value
+
+
+def loip_measure_h2d(nbytes: int = 1 << 30, reps: int = 5) -> float:
+    """Host-to-device copy throughput (bytes/s) from the pool's kind of pinned memory."""
+    out = C.c_double()
+    _check(lib().loip_measure_h2d(nbytes, reps, C.byref(out)))
     return out.value
 
 
