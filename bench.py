@@ -229,6 +229,7 @@ def run_ours(args, rank, world):
     st_end = ctx.stats()
     plan_end = ctx.plan()
     ctx.close()
+    link_after = link_peak_gbs(torch)  # contention on the shared host link shows here too
 
     if world > 1:
         dev_s, e2e_s = max_over_ranks([dev_s, e2e_s], device="cuda")
@@ -276,6 +277,7 @@ def run_ours(args, rank, world):
                      "avg_launch_ms": round(gu_ms, 4)},
         "step_roofline": {"bound": "host-link" if link_bytes / link_peak > hbm_bytes / hbm_peak else "hbm",
                           "link_bytes_per_step": link_bytes, "link_peak_GBps": round(link_peak, 1),
+                          "link_peak_after_GBps": round(link_after, 1),
                           "link_achieved_GBps": round(link_bytes / step_s / 1e9, 1),
                           "hbm_bytes_per_step": hbm_bytes, "roofline_step_ms": round(roof_step * 1e3, 3),
                           "frac": round(roof_step / step_s, 4), "exposed_load_ms": round(exposed * 1e3, 3),

@@ -9,6 +9,12 @@ MODELS = {
     # 2 layers, hidden 256, 4 query heads x 64, 2 kv heads, SwiGLU 688, vocab 1024
     "tiny": dict(n_layers=2, hidden=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=688, vocab=1024,
                  rms_eps=1e-5, rope_theta=500000.0),
+    # plain multi-head attention (one kv head per query head)
+    "tiny-mha": dict(n_layers=3, hidden=256, n_heads=4, n_kv_heads=4, head_dim=64, ffn=688, vocab=1024,
+                     rms_eps=1e-5, rope_theta=10000.0),
+    # the paper's 13B model shape (LLaMA2-13B: MHA, vocabulary 32000, rotary base 10000)
+    "llama2-13b": dict(n_layers=40, hidden=5120, n_heads=40, n_kv_heads=40, head_dim=128, ffn=13824, vocab=32000,
+                       rms_eps=1e-5, rope_theta=10000.0),
     "llama3-8b": dict(n_layers=32, hidden=4096, n_heads=32, n_kv_heads=8, head_dim=128, ffn=14336, vocab=128256,
                       rms_eps=1e-5, rope_theta=500000.0),
     "llama3-70b": dict(n_layers=80, hidden=8192, n_heads=64, n_kv_heads=8, head_dim=128, ffn=28672, vocab=128256,
@@ -23,6 +29,7 @@ CONTEXT_SEED = 2
 WORKLOADS = {
     "tiny-decode": dict(model="tiny", batch=1, prompt=32, decode=16, budget=None, n_slots=2),
     "8b-decode": dict(model="llama3-8b", batch=1, prompt=512, decode=128, budget=None, n_slots=2),
+    "13b-decode": dict(model="llama2-13b", batch=1, prompt=512, decode=128, budget=None, n_slots=2),
     "70b-offload-decode": dict(model="llama3-70b", batch=1, prompt=1024, decode=64, budget=60_000_000_000,
                                n_slots=2),
     "70b-offload-prefill": dict(model="llama3-70b", batch=4, prompt=512, decode=0, budget=60_000_000_000,

@@ -180,12 +180,11 @@ __device__ __forceinline__ void fma_block(float (&acc)[U][BT], const uint4 (&w)[
 // Accumulates the unit's rows over staged chunk [kc0, kc0 + kn).  Two register
 // batches of JU 128-bit loads per row alternate, so the next batch is in flight
 // while the current one is consumed.
-template <int BT, int U>
-__device__ __forceinline__ void load_batch(uint4 (&w)[4][U], const uint16_t* const (&rp)[U], const bool (&rv)[U],
-                                           int kc0, int j0, int nj, int K, int lane, int JU) {
+template <int BT, int U, int JU>
+__device__ __forceinline__ void load_batch(uint4 (&w)[JU][U], const uint16_t* const (&rp)[U], const bool (&rv)[U],
+                                           int kc0, int j0, int nj, int K, int lane) {
 #pragma unroll
-    for (int jj = 0; jj < 4; ++jj) {
-        if (jj >= JU) break;
+    for (int jj = 0; jj < JU; ++jj) {
         const int k = kc0 + (j0 + jj) * 256 + lane * 8;
         const bool ok = (j0 + jj < nj) && (k < K);
 #pragma unroll
@@ -193,19 +192,26 @@ __device__ __forceinline__ void load_batch(uint4 (&w)[4][U], const uint16_t* con
     }
 }
 
+// Loads per row and batch: a warp keeps about 2 x 8 x 16 bytes per lane in
+// flight whatever its unit's row count.
+template <int BT, int U>
+struct Batch {
+    static constexpr int JU = (BT == 1) ? (U == 1 ? 2 * LOIP_GEMV_JU1 : LOIP_GEMV_JU1) : (BT == 2) ? 4 : 2;
+};
+
 template <int BT, int U, int EPI>
 __device__ __forceinline__ void unit_chunk(float (&acc)[U][BT], const uint16_t* const (&rp)[U], const bool (&rv)[U],
                                            const float* __restrict__ s, int kc0, int kn, int K, int lane) {
-    constexpr int JU = (BT == 1) ? LOIP_GEMV_JU1 : (BT == 2) ? 4 : 2;
+    constexpr int JU = Batch<BT, U>::JU;
     const int nj = (kn + 255) >> 8;
-    uint4 wa[4][U], wb[4][U];
-    load_batch<BT, U>(wa, rp, rv, kc0, 0, nj, K, lane, JU);
+    uint4 wa[JU][U], wb[JU][U];
+    load_batch<BT, U, JU>(wa, rp, rv, kc0, 0, nj, K, lane);
     for (int j0 = 0; j0 < nj; j0 += 2 * JU) {
-        load_batch<BT, U>(wb, rp, rv, kc0, j0 + JU, nj, K, lane, JU);
+        load_batch<BT, U, JU>(wb, rp, rv, kc0, j0 + JU, nj, K, lane);
 #pragma unroll
         for (int jj = 0; jj < JU; ++jj)
             if (j0 + jj < nj) fma_block<BT, U>(acc, wa[jj], s, j0 + jj, lane);
-        load_batch<BT, U>(wa, rp, rv, kc0, j0 + 2 * JU, nj, K, lane, JU);
+        load_batch<BT, U, JU>(wa, rp, rv, kc0, j0 + 2 * JU, nj, K, lane);
 #pragma unroll
         for (int jj = 0; jj < JU; ++jj)
             if (j0 + JU + jj < nj) fma_block<BT, U>(acc, wb[jj], s, j0 + JU + jj, lane);
@@ -298,14 +304,14 @@ __global__ void __launch_bounds__(kThreads, BT == 1 ? LOIP_GEMV_MIN_BLOCKS1 : 2)
     const bool norm = p.g != nullptr;
 
     // weights never depend on the previous kernel: start pulling this warp's
-    // first rows into L2 before waiting for the activations
+    // first rows (up to 32 KB each) into L2 before waiting for the activations
     pdl_trigger();
     {
         const int u0 = blockIdx.x * kWarps + warp;
         if (lane < U && u0 < p.n_units) {
             bool v;
             const uint16_t* r = unit_row<EPI>(p, u0, lane, v);
-            const uint32_t bytes = (uint32_t)min(K * 2, 8192);
+            const uint32_t bytes = (uint32_t)min(K * 2, 32768);
             if (v) prefetch_l2(r, bytes);
         }
     }
@@ -447,6 +453,193 @@ __global__ void __launch_bounds__(kThreads, BT == 1 ? LOIP_GEMV_MIN_BLOCKS1 : 2)
     }
 }
 
+// ----------------------------------------------------------------------------
+// Batch-1 block-tile GEMV.  A block owns kTileRows weight rows; its warps split
+// K, so every 128-bit load of the tile is issued within one or two batches per
+// warp (double-buffered), and the activation slice a warp needs comes straight
+// from L1/L2 (no staging barrier).  Partial sums are reduced in a fixed order
+// (lanes, then warps) so results do not depend on scheduling.  Row units as in
+// the persistent kernel: QKV and SwiGLU tiles hold 4 row pairs.
+// ----------------------------------------------------------------------------
+constexpr int kTileWarps = 8;
+constexpr int kTileRows = 8;
+
+template <int EPI>
+__device__ __forceinline__ const uint16_t* tile_row(const GemvParams& p, int tile, int r, bool& valid) {
+    if (EPI == EPI_QKV) {
+        const int half = p.d >> 1;
+        const int pair = tile * (kTileRows / 2) + (r & 3);
+        const int h = pair / half, i = pair - h * half;
+        valid = pair < p.n_units;
+        return p.w0 + (size_t)(h * p.d + i + (r >> 2) * half) * p.K;
+    } else if (EPI == EPI_SWIGLU) {
+        const int j = tile * (kTileRows / 2) + (r & 3);
+        valid = j < p.n_units;
+        return ((r >> 2) ? p.w1 : p.w0) + (size_t)j * p.K;
+    } else {
+        const int row = tile * kTileRows + r;
+        valid = row < p.N;
+        return p.w0 + (size_t)row * p.K;
+    }
+}
+
+__device__ __forceinline__ void tile_load(uint4 (&w)[kTileRows], const uint16_t* const (&rp)[kTileRows],
+                                          const bool (&rv)[kTileRows], int j, int j_end, int K, int lane) {
+    const int k = j * 256 + lane * 8;
+    const bool ok = j < j_end && k < K;
+#pragma unroll
+    for (int r = 0; r < kTileRows; ++r) w[r] = (ok && rv[r]) ? ld_stream(rp[r] + k) : make_uint4(0, 0, 0, 0);
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParams p) {
+    constexpr int R = kTileRows;
+    __shared__ float s_part[kTileWarps][R];
+    __shared__ float s_ss[kTileWarps];
+    __shared__ float s_val[R];
+    __shared__ float s_inv;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int tile = blockIdx.x, K = p.K;
+    const int nj = (K + 255) >> 8;
+    const int njw = (nj + kTileWarps - 1) / kTileWarps;
+    const int j_begin = warp * njw, j_end = min(nj, j_begin + njw);
+    const bool norm = p.g != nullptr;
+    const uint16_t* rp[R];
+    bool rv[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) rp[r] = tile_row<EPI>(p, tile, r, rv[r]);
+
+    pdl_trigger();
+    uint4 wa[R], wb[R];
+    tile_load(wa, rp, rv, j_begin, j_end, K, lane);  // weights do not depend on the previous kernel
+    pdl_wait();
+
+    float acc[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) acc[r] = 0.f;
+    float ss = 0.f;
+    auto consume = [&](const uint4 (&w)[R], int j) {
+        const int k = j * 256 + lane * 8;
+        if (j >= j_end || k >= K) return;
+        const float4 xa = *reinterpret_cast<const float4*>(p.in + k);
+        const float4 xb = *reinterpret_cast<const float4*>(p.in + k + 4);
+        float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+        if (norm) {
+            const uint4 gv = *reinterpret_cast<const uint4*>(p.g + k);
+            const float gf[8] = {bf_lo(gv.x), bf_hi(gv.x), bf_lo(gv.y), bf_hi(gv.y),
+                                 bf_lo(gv.z), bf_hi(gv.z), bf_lo(gv.w), bf_hi(gv.w)};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                ss = fmaf(xv[e], xv[e], ss);
+                xv[e] *= gf[e];
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            float a = acc[r];
+            a = fmaf(bf_lo(w[r].x), xv[0], a);
+            a = fmaf(bf_hi(w[r].x), xv[1], a);
+            a = fmaf(bf_lo(w[r].y), xv[2], a);
+            a = fmaf(bf_hi(w[r].y), xv[3], a);
+            a = fmaf(bf_lo(w[r].z), xv[4], a);
+            a = fmaf(bf_hi(w[r].z), xv[5], a);
+            a = fmaf(bf_lo(w[r].w), xv[6], a);
+            a = fmaf(bf_hi(w[r].w), xv[7], a);
+            acc[r] = a;
+        }
+    };
+    for (int j = j_begin; j < j_end; j += 2) {
+        tile_load(wb, rp, rv, j + 1, j_end, K, lane);
+        consume(wa, j);
+        tile_load(wa, rp, rv, j + 2, j_end, K, lane);
+        consume(wb, j + 1);
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const float v = warp_sum(acc[r]);
+        if (lane == 0) s_part[warp][r] = v;
+    }
+    if (norm) {
+        const float v = warp_sum(ss);
+        if (lane == 0) s_ss[warp] = v;
+    }
+    __syncthreads();
+    if (tid < R) {
+        float t = 0.f;
+        for (int w = 0; w < kTileWarps; ++w) t += s_part[w][tid];
+        s_val[tid] = t;
+    }
+    if (tid == 32) {
+        float t = 0.f;
+        if (norm)
+            for (int w = 0; w < kTileWarps; ++w) t += s_ss[w];
+        s_inv = norm ? 1.0f / sqrtf(t / (float)K + p.eps) : 1.0f;
+    }
+    __syncthreads();
+    const float inv = s_inv;
+    if (EPI == EPI_QKV) {
+        if (tid < R / 2) {
+            const int half = p.d >> 1;
+            const int pair = tile * (R / 2) + tid;
+            if (pair < p.n_units) {
+                const int h = pair / half, i = pair - h * half;
+                float v0 = s_val[tid] * inv, v1 = s_val[tid + R / 2] * inv;
+                const int pos = p.positions[0];
+                if (h < p.Hq + p.Hkv) {
+                    float cf, sf;
+                    rope_cos_sin(pos, p.rope.inv_freq[i], &cf, &sf);
+                    const float r0 = v0 * cf - v1 * sf, r1 = v1 * cf + v0 * sf;
+                    v0 = r0;
+                    v1 = r1;
+                }
+                if (h < p.Hq) {
+                    float* q = p.out + (size_t)h * p.d;
+                    q[i] = v0;
+                    q[i + half] = v1;
+                } else {
+                    const int req = p.row_req ? p.row_req[0] : 0;
+                    const bool is_v = h >= p.Hq + p.Hkv;
+                    const int kh = h - p.Hq - (is_v ? p.Hkv : 0);
+                    uint16_t* row = reinterpret_cast<uint16_t*>(kv_row(p.kv, req, pos, is_v ? 1 : 0, kh, p.Hkv, p.d));
+                    row[i] = f2bf(v0);
+                    row[i + half] = f2bf(v1);
+                }
+            }
+        }
+    } else if (EPI == EPI_SWIGLU) {
+        if (tid < R / 2) {
+            const int j = tile * (R / 2) + tid;
+            if (j < p.n_units) {
+                const float gt = s_val[tid] * inv, ut = s_val[tid + R / 2] * inv;
+                p.out[j] = gt / (1.0f + expf(-gt)) * ut;
+            }
+        }
+    } else if (EPI == EPI_RESID) {
+        if (tid < R) {
+            const int row = tile * R + tid;
+            if (row < p.N) p.out[row] += s_val[tid];
+        }
+    } else {  // EPI_LOGITS
+        if (tid < R) {
+            const int row = tile * R + tid;
+            if (row < p.N && p.out) p.out[row] = s_val[tid] * inv;
+        }
+        if (tid == 0) {
+            uint64_t best = 0;
+            for (int r = 0; r < R; ++r) {
+                const int row = tile * R + r;
+                if (row < p.N) {
+                    const uint64_t key = argmax_key(s_val[r] * inv, (uint32_t)row);
+                    best = key > best ? key : best;
+                }
+            }
+            p.keys[tile] = best;
+        }
+        if (tile == 0 && p.z)
+            for (int k = tid; k < K; k += kTileWarps * 32) p.z[k] = p.in[k] * inv * bf2f(p.g[k]);
+    }
+}
+
 __global__ void argmax_reduce_kernel(const uint64_t* keys, int nblocks, int BT, int B, int32_t* tokens) {
     __shared__ uint64_t s[256];
     pdl_trigger();
@@ -486,6 +679,18 @@ cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
 
 template <int EPI>
 cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, bool pdl, int* nblocks_out = nullptr) {
+    // Batch 1: matrices with few rows (QKV, O-proj, down) keep too few units per
+    // warp for the persistent kernel to ramp up; the block-tile kernel issues a
+    // whole tile at once.  Row-rich ones (gate/up, LM head) stream better
+    // persistent.
+    const int rows = (EPI == EPI_SWIGLU) ? 2 * p.n_units : p.N;
+    if (p.B == 1 && rows <= 16384) {
+        const int per_tile = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? kTileRows / 2 : kTileRows;
+        const int units = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? p.n_units : p.N;
+        const int tiles = (units + per_tile - 1) / per_tile;
+        if (nblocks_out) *nblocks_out = tiles;
+        return launch_k(gemv_tile_kernel<EPI>, dim3(tiles), dim3(kTileWarps * 32), 0, st, pdl, p);
+    }
     int BT = p.B <= 1 ? 1 : p.B <= 2 ? 2 : p.B <= 4 ? 4 : 8;
     int kc_max = (kStageFloats / BT) & ~255;
     bool single = p.K <= kc_max;
@@ -585,7 +790,6 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
     __shared__ __align__(16) float sq[G][D];
     __shared__ float s_m[G], s_l[G];
     __shared__ float s_o[G][D];
-    __shared__ float s_w[G][kMaxChunks];  // combine weights of the per-page states
     __shared__ int s_last;
 
     pdl_trigger();
@@ -769,37 +973,64 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
     if (!s_last) return;
     __threadfence();
     const float* base = p.scratch + ((size_t)row * p.Hq + (size_t)kvh * G) * p.max_chunks * (D + 2);
+    const size_t hstride = (size_t)p.max_chunks * (D + 2);
+    // the staging buffers are dead: combine weights and denominators reuse them
+    static_assert(G * kMaxChunks * sizeof(float) <= sizeof(sK), "combine weights fit the key stage");
+    float(*s_w)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sK[0]);
+    float(*s_lw)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sV[0]);
+    // (m, l) of every (head, page) in one round trip; weights reduced in shared memory
+    for (int i = tid; i < G * npages; i += 64) {
+        const int g = i / npages, c = i - g * npages;
+        const float* pc = base + g * hstride + (size_t)c * (D + 2);
+        s_w[g][c] = pc[D];
+        s_lw[g][c] = pc[D + 1];
+    }
+    __syncthreads();
     for (int g = warp; g < G; g += 2) {
-        const float* ph = base + (size_t)g * p.max_chunks * (D + 2);
         float mx = -INFINITY;
-        for (int c = lane; c < npages; c += 32) {
-            const float mc = ph[(size_t)c * (D + 2) + D];
-            s_w[g][c] = mc;
-            mx = fmaxf(mx, mc);
-        }
+        for (int c = lane; c < npages; c += 32) mx = fmaxf(mx, s_w[g][c]);
         mx = warp_max(mx);
         float lsum = 0.f;
         for (int c = lane; c < npages; c += 32) {
             const float w = (s_w[g][c] == -INFINITY) ? 0.f : expf(s_w[g][c] - mx);
             s_w[g][c] = w;
-            lsum = fmaf(ph[(size_t)c * (D + 2) + D + 1], w, lsum);
+            lsum = fmaf(s_lw[g][c], w, lsum);
         }
         lsum = warp_sum(lsum);
         const float inv = lsum > 0.f ? 1.0f / lsum : 0.f;
         for (int c = lane; c < npages; c += 32) s_w[g][c] *= inv;
     }
     __syncthreads();
-    for (int e = tid; e < G * D; e += 64) {
-        const int g = e / D, j = e - g * D;
-        const float* ph = base + (size_t)g * p.max_chunks * (D + 2) + j;
-        float acc = 0.f;
-#pragma unroll 8
-        for (int c = 0; c < npages; ++c) acc = fmaf(ph[(size_t)c * (D + 2)], s_w[g][c], acc);
+    // chunks outer, this thread's outputs inner: 4 x NOUT loads in flight
+    constexpr int NOUT = G * D / 64;
+    float acc[NOUT];
+#pragma unroll
+    for (int k = 0; k < NOUT; ++k) acc[k] = 0.f;
+    for (int c0 = 0; c0 < npages; c0 += 4) {
+        float v[4][NOUT];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int k = 0; k < NOUT; ++k) {
+                const int e = tid + 64 * k, g = e / D, j = e - g * D;
+                v[u][k] = (c0 + u < npages) ? base[g * hstride + (size_t)(c0 + u) * (D + 2) + j] : 0.f;
+            }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int k = 0; k < NOUT; ++k) {
+                const int g = (tid + 64 * k) / D;
+                if (c0 + u < npages) acc[k] = fmaf(v[u][k], s_w[g][c0 + u], acc[k]);
+            }
+    }
+#pragma unroll
+    for (int k = 0; k < NOUT; ++k) {
+        const int e = tid + 64 * k, g = e / D, j = e - g * D;
         const size_t idx = (size_t)row * p.Hq * D + (size_t)(kvh * G + g) * D + j;
         if (p.o_bf16)
-            reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(acc);
+            reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(acc[k]);
         else
-            reinterpret_cast<float*>(p.o)[idx] = acc;
+            reinterpret_cast<float*>(p.o)[idx] = acc[k];
     }
 }
 

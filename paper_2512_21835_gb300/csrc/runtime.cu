@@ -1330,7 +1330,7 @@ extern "C" int loip_k_qkv_rope(const float* x, const uint16_t* g, const uint16_t
                                float* q_out, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
                                int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, void* stream) {
     if (!x || !g || !wqkv || !positions || !q_out || !kv_base || !page_offsets || B < 1 || B > 8 || H % 8 ||
-        (d != 64 && d != 128) || Hq % Hkv || page_tokens < 1 || !al16(wqkv) || !al16(x) || ((uintptr_t)g & 7))
+        (d != 64 && d != 128) || Hq % Hkv || page_tokens < 1 || !al16(wqkv) || !al16(x) || !al16(g))
         return LOIP_ERR_INVALID;
     KvView kv{(char*)kv_base, page_offsets, max_pages, page_tokens, layer, layer_page_bytes};
     return cerr(launch_qkv_rope(x, g, wqkv, B, H, Hq, Hkv, d, eps, theta, positions, q_out, kv, nullptr,
@@ -1369,7 +1369,7 @@ extern "C" int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32
 extern "C" int loip_k_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int32_t B,
                               int32_t H, int32_t F, float eps, float* a, void* stream) {
     if (!x || !g || !wg || !wu || !a || B < 1 || B > 8 || H % 8 || F < 1 || !al16(wg) || !al16(wu) || !al16(x) ||
-        ((uintptr_t)g & 7))
+        !al16(g))
         return LOIP_ERR_INVALID;
     return cerr(launch_gate_up(x, g, wg, wu, B, H, F, eps, a, (cudaStream_t)stream));
 }
@@ -1403,7 +1403,7 @@ extern "C" int loip_k_lm_head(const float* x, const uint16_t* g_final, const uin
                               int32_t V, float eps, float* z, float* logits, int32_t* tokens, void* scratch,
                               void* stream) {
     if (!x || !g_final || !lm_head || !tokens || !scratch || B < 1 || B > 8 || H % 8 || V < 1 || !al16(lm_head) ||
-        !al16(x) || ((uintptr_t)g_final & 7))
+        !al16(x) || !al16(g_final))
         return LOIP_ERR_INVALID;
     return cerr(launch_lm_head(x, g_final, lm_head, B, H, V, eps, z, logits, tokens, scratch, (cudaStream_t)stream));
 }

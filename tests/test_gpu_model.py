@@ -145,3 +145,18 @@ def test_kv_growth_demotes_layers(torch, L, orc):
     assert st["arena_used"] <= budget
     assert np.array_equal(np.array(toks), base[0])
     assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
+
+
+def test_multi_head_model_matches_oracle(torch, L, orc):
+    """LLaMA2-style plain multi-head attention (G = 1), two of three layers streamed through one slot."""
+    m = configs.MODELS["tiny-mha"]
+    prompt = inputs.token_ids(71, 40, m["vocab"])
+    P = 24
+    ref = _oracle(orc, m, prompt[:P], prompt[P:])
+    cont = [[t] for t in prompt[P:]]
+    toks, hids, plan, _ = _run(L, torch, m, [prompt[:P]], cont, dict(max_batch=1, max_ctx=64, n_slots=1), 1)
+    assert plan["n_offloaded"] == 2
+    for i in range(len(toks)):
+        t = P - 1 + i
+        _check_hidden(hids[i][0], ref["hidden"][t])
+        assert int(toks[i][0]) == int(ref["argmax"][t])
