@@ -63,43 +63,66 @@ class _Desc(C.Structure):
 _lib = None
 
 
+def _bind(L):
+    """Declares the C signatures on a loaded oracle library."""
+    L.orc_splitmix64.restype = C.c_uint64
+    L.orc_splitmix64.argtypes = [C.c_uint64, C.c_uint64]
+    L.orc_gen_elem.restype = C.c_uint16
+    L.orc_gen_elem.argtypes = [C.c_uint64, C.c_uint32, C.c_uint64, C.c_int]
+    L.orc_gen_tensor.restype = None
+    L.orc_gen_tensor.argtypes = [C.c_uint64, C.c_uint32, C.c_uint64, C.c_uint64, C.c_int, C.c_void_p]
+    L.orc_f32_to_bf16.restype = C.c_uint16
+    L.orc_f32_to_bf16.argtypes = [C.c_float]
+    L.orc_bf16_to_f32.restype = C.c_float
+    L.orc_bf16_to_f32.argtypes = [C.c_uint16]
+    L.orc_round_bf16.restype = C.c_double
+    L.orc_round_bf16.argtypes = [C.c_double]
+    L.orc_rmsnorm.restype = None
+    L.orc_rmsnorm.argtypes = [C.c_void_p, C.POINTER(_Tensor), C.c_int, C.c_double, C.c_void_p]
+    L.orc_gemv.restype = None
+    L.orc_gemv.argtypes = [C.POINTER(_Tensor), C.c_int64, C.c_void_p, C.c_int64, C.c_void_p, C.c_void_p]
+    L.orc_rope.restype = None
+    L.orc_rope.argtypes = [C.c_void_p, C.c_int, C.c_int64, C.c_double]
+    L.orc_silu.restype = C.c_double
+    L.orc_silu.argtypes = [C.c_double]
+    L.orc_attention.restype = None
+    L.orc_attention.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64, C.c_int, C.c_int, C.c_int,
+                                C.c_void_p, C.c_void_p]
+    L.orc_tensor_id.restype = C.c_uint32
+    L.orc_tensor_id.argtypes = [C.c_int, C.c_int]
+    L.orc_generated_tensors.restype = None
+    L.orc_generated_tensors.argtypes = [C.POINTER(_Desc), C.c_uint64, C.POINTER(_Tensor)]
+    L.orc_forward.restype = C.c_int
+    L.orc_forward.argtypes = [C.POINTER(_Desc), C.POINTER(_Tensor), C.c_void_p, C.c_int64, C.c_int64, C.c_int,
+                              C.c_int, C.c_void_p, C.c_void_p, C.c_void_p]
+    L.orc_num_threads.restype = C.c_int
+    return L
+
+
 def lib():
     global _lib
     if _lib is None:
-        _lib = C.CDLL(build())
-        L = _lib
-        L.orc_splitmix64.restype = C.c_uint64
-        L.orc_splitmix64.argtypes = [C.c_uint64, C.c_uint64]
-        L.orc_gen_elem.restype = C.c_uint16
-        L.orc_gen_elem.argtypes = [C.c_uint64, C.c_uint32, C.c_uint64, C.c_int]
-        L.orc_gen_tensor.restype = None
-        L.orc_gen_tensor.argtypes = [C.c_uint64, C.c_uint32, C.c_uint64, C.c_uint64, C.c_int, C.c_void_p]
-        L.orc_f32_to_bf16.restype = C.c_uint16
-        L.orc_f32_to_bf16.argtypes = [C.c_float]
-        L.orc_bf16_to_f32.restype = C.c_float
-        L.orc_bf16_to_f32.argtypes = [C.c_uint16]
-        L.orc_round_bf16.restype = C.c_double
-        L.orc_round_bf16.argtypes = [C.c_double]
-        L.orc_rmsnorm.restype = None
-        L.orc_rmsnorm.argtypes = [C.c_void_p, C.POINTER(_Tensor), C.c_int, C.c_double, C.c_void_p]
-        L.orc_gemv.restype = None
-        L.orc_gemv.argtypes = [C.POINTER(_Tensor), C.c_int64, C.c_void_p, C.c_int64, C.c_void_p, C.c_void_p]
-        L.orc_rope.restype = None
-        L.orc_rope.argtypes = [C.c_void_p, C.c_int, C.c_int64, C.c_double]
-        L.orc_silu.restype = C.c_double
-        L.orc_silu.argtypes = [C.c_double]
-        L.orc_attention.restype = None
-        L.orc_attention.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64, C.c_int, C.c_int, C.c_int,
-                                    C.c_void_p, C.c_void_p]
-        L.orc_tensor_id.restype = C.c_uint32
-        L.orc_tensor_id.argtypes = [C.c_int, C.c_int]
-        L.orc_generated_tensors.restype = None
-        L.orc_generated_tensors.argtypes = [C.POINTER(_Desc), C.c_uint64, C.POINTER(_Tensor)]
-        L.orc_forward.restype = C.c_int
-        L.orc_forward.argtypes = [C.POINTER(_Desc), C.POINTER(_Tensor), C.c_void_p, C.c_int64, C.c_int64, C.c_int,
-                                  C.c_int, C.c_void_p, C.c_void_p, C.c_void_p]
-        L.orc_num_threads.restype = C.c_int
+        _lib = _bind(C.CDLL(build()))
     return _lib
+
+
+class use_library:
+    """Context manager: route every oracle call through another build of
+    oracle.c (the pin tests use it to check that planted mistakes are caught)."""
+
+    def __init__(self, path: str):
+        self.path = path
+
+    def __enter__(self):
+        global _lib
+        self.saved = lib()
+        _lib = _bind(C.CDLL(self.path))
+        return _lib
+
+    def __exit__(self, *exc):
+        global _lib
+        _lib = self.saved
+        return False
 
 
 def _ptr(a: np.ndarray) -> int:

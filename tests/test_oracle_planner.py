@@ -75,3 +75,50 @@ def test_plan_and_threshold():
     # Eq. 6 reading: tokens until the KV cache exhausts what is left
     assert P.kv_threshold_tokens(1000, 100, 100, 6, 2, 10) == 10
     assert P.kv_threshold_tokens(1000, 100, 100, 8, 2, 10) == 0
+
+
+def _max_resident_run(mask):
+    """Longest cyclic run of resident layers (brute force over start points)."""
+    L = len(mask)
+    if not any(mask):
+        return L
+    best = 0
+    for s in range(L):
+        run = 0
+        while run < L and not mask[(s + run) % L]:
+            run += 1
+        best = max(best, run)
+    return best
+
+
+def test_demote_one_hand_cases():
+    # nothing offloaded: the last layer goes first (where m = 1 even spacing puts it)
+    assert P.demote_one([False] * 8) == ([False] * 7 + [True], 7)
+    # L = 8: 7 -> 3 (middle of 0..6) -> 5 (first of two runs of 3, 4..6) -> 1
+    mask, order = [False] * 8, []
+    for _ in range(4):
+        mask, v = P.demote_one(mask)
+        order.append(v)
+    assert order == [7, 3, 5, 1]
+    assert mask == [False, True] * 4
+    # even-length run: the lower middle (L = 5: after 4, run 0..3 -> layer 1)
+    assert P.demote_one(P.demote_one([False] * 5)[0])[1] == 1
+    # the run may wrap around the end of the layer order: offloaded {2}, run 3,4,0,1 -> layer 4
+    assert P.demote_one([False, False, True, False, False]) == ([False, False, True, False, True], 4)
+    # everything offloaded: no victim
+    assert P.demote_one([True] * 3) == ([True] * 3, None)
+
+
+def test_demote_one_minimises_longest_resident_run_brute_force():
+    import random
+    rng = random.Random(5)
+    for _ in range(300):
+        L = rng.randint(2, 24)
+        mask = [rng.random() < 0.3 for _ in range(L)]
+        if all(mask):
+            continue
+        new, v = P.demote_one(mask)
+        assert not mask[v] and new[v] and sum(new) == sum(mask) + 1
+        assert all(new[i] == mask[i] for i in range(L) if i != v)
+        best = min(_max_resident_run(mask[:i] + [True] + mask[i + 1:]) for i in range(L) if not mask[i])
+        assert _max_resident_run(new) == best
