@@ -5,17 +5,22 @@ of which the ones that do not fit the 60 GB device budget stream from pinned
 host memory through the slot ring, final norm, LM head, argmax) for one batch.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+                    [--mode overlap|direct|naive]
 
 Prints one JSON line (rank 0).  `value` is timed on the device with CUDA events
 on the compute stream, tokens fed back on the device; `e2e` is the same
 metric through loip_decode_step with host token buffers (host<->device copies
 inside the timed region).  `--impl reference` times the CPU oracle (the plain
 fp64 definition of the decoder) on the host cores on a bounded sample.
+`--mode direct` runs the decode steps with the offloaded layers read in place
+from the pinned pool (zero-copy) instead of streamed through the slots;
+`--mode naive` is the conventional load-then-compute path.
 Multi-GPU: independent replicas (the path does not shard), one per rank.
 """
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -33,6 +38,25 @@ from paper_2512_21835_gb300 import configs, inputs  # noqa: E402
 
 METRIC = "decode tokens/s, 70B-shaped bf16 w/ offload; HBM & host-link GB/s vs peak"
 KERNEL_NAMES = ["qkv_rope", "attention", "o_proj", "gate_up", "down", "lm_head"]
+MODES = {"overlap": 0, "naive": 1, "direct": 2}
+
+# DRAM bytes (read + write) per launch of the gate/up SwiGLU GEMV at batch 1,
+# from an ncu capture of the kernel microbenchmark on the model's shape
+# (profiles/gemv_traffic.md has the commands and figures).  They describe the
+# kernel source they were taken on: when the decode kernels' source no longer
+# has this hash the figure is reported as null.
+GATE_UP_TRAFFIC = {"llama3-70b": 939_846_656, "llama3-8b": 235_065_856}
+GATE_UP_TRAFFIC_SRC = "8a6e3c9ff5b7d7c56c075510a220df0f29e88defef9726a21d874449af555503"
+
+
+def gate_up_traffic(model, batch):
+    src = os.path.join(ROOT, "paper_2512_21835_gb300", "csrc", "decode.cu")
+    if batch != 1 or GATE_UP_TRAFFIC.get(model) is None:
+        return None
+    with open(src, "rb") as f:
+        if hashlib.sha256(f.read()).hexdigest() != GATE_UP_TRAFFIC_SRC:
+            return None
+    return GATE_UP_TRAFFIC[model]
 
 
 def measured_peaks():
@@ -128,6 +152,8 @@ def run_ours(args, rank, world):
     w, m = workload_setup(args.workload)
     hbm_peak, tc_peak, peak_kind = measured_peaks()
     link_peak = link_peak_gbs(torch)
+    mode = MODES[args.mode]
+    direct_peak = loip.loip_measure_direct_read(1 << 30, 5) / 1e9 if mode == MODES["direct"] else None
     lay = loip.loip_layer_layout(m)
     prompts = make_prompts(w, m)
     Bsz = len(prompts)
@@ -142,7 +168,7 @@ def run_ours(args, rank, world):
     max_prefill = sum(lens) if prefill_mode else min(4096, sum(lens))
     cfg = loip.config(budget=budget, n_slots=w["n_slots"], max_batch=Bsz, max_ctx=max_ctx,
                       max_prefill_tokens=max_prefill, link_Bps=link_peak * 1e9, hbm_Bps=hbm_peak * 1e9,
-                      kv_reserve_bytes=kv_reserve)
+                      kv_reserve_bytes=kv_reserve, mode=mode)
     t0 = time.time()
     ctx = loip.Context(m, cfg)
     plan = ctx.plan()
@@ -246,11 +272,14 @@ def run_ours(args, rank, world):
     mean_ctx = float(np.mean(lens)) + warm + steps / 2
     kv_bytes = int(mean_ctx * 2 * m["n_kv_heads"] * m["head_dim"] * 2 * m["n_layers"] * Bsz)
     hbm_bytes = m["n_layers"] * lay["l_size"] + m["vocab"] * m["hidden"] * 2 + kv_bytes
-    roof_step = max(hbm_bytes / (hbm_peak * 1e9), link_bytes / (link_peak * 1e9))
+    # direct access: the offloaded bytes cross the link as kernel reads, whose
+    # ceiling is the measured direct-read rate, not the copy engine's
+    link_roof = direct_peak if direct_peak else link_peak
+    roof_step = max(hbm_bytes / (hbm_peak * 1e9), link_bytes / (link_roof * 1e9))
     kernel_sum_ms = sum(st["kernel_ms"][:6]) / steps
-    t_copy_only = link_bytes / (link_peak * 1e9)
+    t_copy_only = link_bytes / (link_roof * 1e9)
     exposed = max(0.0, step_s - max(kernel_sum_ms / 1e3, t_copy_only))
-    per_step_launches = 1 + m["n_layers"] * 6 + 2 + 1
+    per_step_launches = 1 + m["n_layers"] * 5 + 2 + 1  # embed, 5 per layer, LM head + argmax, advance
     line = {
         "metric": METRIC,
         "value": round(tokens / dev_s, 4),
@@ -266,17 +295,20 @@ def run_ours(args, rank, world):
         "data": "synthetic: SplitMix64 bf16 weights N(0,0.02^2), uniform token ids",
         "config": {"workload": args.workload, "model": w["model"] + "-shaped", "layers": m["n_layers"],
                    "global_batch": Bsz * world, "context": lens if len(set(lens)) > 1 else lens[0],
-                   "budget_bytes": budget, "slots": w["n_slots"], "resident_layers": st1["n_resident"],
+                   "budget_bytes": budget, "slots": 1 if args.mode == "naive" else w["n_slots"], "mode": args.mode,
+                   "resident_layers": st1["n_resident"],
                    "offloaded_layers": n_off, "offloaded_at_start": n_off0,
                    "offloaded_at_end": plan_end["n_offloaded"], "replans": st_end["n_replans"],
                    "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2: every step reads all weights (> 10 GB)"},
         "roofline": {"bound": "hbm", "kernel": "gate_up (RMSNorm+SwiGLU GEMV)", "achieved": round(gu_gbs, 1),
                      "peak": hbm_peak, "unit": "GB/s", "frac": round(gu_gbs / hbm_peak, 4),
-                     "peak_kind": peak_kind, "traffic": None, "bytes_per_launch": gu_bytes,
+                     "peak_kind": peak_kind, "traffic": gate_up_traffic(w["model"], Bsz),
+                     "bytes_per_launch": gu_bytes,
                      "avg_launch_ms": round(gu_ms, 4)},
-        "step_roofline": {"bound": "host-link" if link_bytes / link_peak > hbm_bytes / hbm_peak else "hbm",
+        "step_roofline": {"bound": ("host-link" if link_bytes / link_roof > hbm_bytes / hbm_peak else "hbm"),
                           "link_bytes_per_step": link_bytes, "link_peak_GBps": round(link_peak, 1),
+                          "direct_read_peak_GBps": round(direct_peak, 1) if direct_peak else None,
                           "link_peak_after_GBps": round(link_after, 1),
                           "link_achieved_GBps": round(link_bytes / step_s / 1e9, 1),
                           "hbm_bytes_per_step": hbm_bytes, "roofline_step_ms": round(roof_step * 1e3, 3),
@@ -397,6 +429,7 @@ def main():
     ap.add_argument("--workload", default="70b-offload-decode", choices=sorted(configs.WORKLOADS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mode", default="overlap", choices=sorted(MODES))
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

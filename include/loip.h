@@ -43,7 +43,16 @@ enum {
     LOIP_ERR_STATE = 6       /* call not valid in the context's current state */
 };
 
-enum { LOIP_MODE_OVERLAP = 0, LOIP_MODE_NAIVE = 1 };
+/* OVERLAP: offloaded layers stream into the device slots on the copy stream
+ *   while earlier layers compute (Sec. III-C).
+ * NAIVE: the conventional path the paper measures against (Sec. II-B): one
+ *   slot, each load issued when its layer is reached, compute waits for it.
+ * DIRECT: decode steps read the offloaded layers' weights in place from the
+ *   pinned host pool through its device mapping (zero-copy over the host link;
+ *   the counterpart of the paper's UMA-aware loading, Sec. III-C, on a
+ *   discrete-memory GPU).  Prefill, loip_stream_layer and loip_layer_forward
+ *   keep using the slots, so the plan still reserves them. */
+enum { LOIP_MODE_OVERLAP = 0, LOIP_MODE_NAIVE = 1, LOIP_MODE_DIRECT = 2 };
 
 typedef struct loip_model_desc {
     int32_t n_layers, hidden, n_heads, n_kv_heads, head_dim, ffn, vocab;
@@ -58,7 +67,7 @@ typedef struct loip_config {
     int32_t max_batch;            /* largest decode batch (<= 8) */
     int32_t max_ctx;              /* largest context per request, tokens */
     int32_t use_graphs;           /* capture decode steps as CUDA graphs */
-    int32_t mode;                 /* LOIP_MODE_OVERLAP or LOIP_MODE_NAIVE */
+    int32_t mode;                 /* LOIP_MODE_OVERLAP, LOIP_MODE_NAIVE or LOIP_MODE_DIRECT */
     uint32_t timeout_ms;          /* deadline of every host wait (0 = 600000) */
     double hbm_Bps;               /* bandwidths used by the planner's step model */
     double link_Bps;
@@ -233,6 +242,14 @@ int loip_synchronize(loip_ctx* ctx);
  * memory (the pool's allocator) to device memory on the current device.
  * Allocates and frees its own buffers.  *out_Bps in bytes per second. */
 int loip_measure_h2d(uint64_t bytes, int32_t reps, double* out_Bps);
+
+/* Host-link throughput as direct-access kernels see it: best of `reps` timed
+ * launches of a kernel that streams `bytes` (>= 1 MiB, a multiple of 16) with
+ * 128-bit loads from a pinned, mapped host buffer (the pool's allocator), one
+ * block per SM x 4.  Allocates and frees its own buffers.  *out_Bps in bytes
+ * per second.  The paper has no counterpart; it is the roofline of
+ * LOIP_MODE_DIRECT decode. */
+int loip_measure_direct_read(uint64_t bytes, int32_t reps, double* out_Bps);
 
 /* Device pointer of the compute / copy stream (cudaStream_t). */
 void* loip_compute_stream(loip_ctx* ctx);

@@ -101,6 +101,7 @@ struct GemvParams {
     const int32_t* row_req;
     KvView kv;
     RopeFreqs rope;
+    int w_host;  // weights are read in place from mapped host memory: no L2 prefetch of them
 };
 
 // rows handled per warp unit, by epilogue
@@ -308,7 +309,7 @@ __global__ void __launch_bounds__(kThreads, BT == 1 ? LOIP_GEMV_MIN_BLOCKS1 : 2)
     pdl_trigger();
     {
         const int u0 = blockIdx.x * kWarps + warp;
-        if (lane < U && u0 < p.n_units) {
+        if (!p.w_host && lane < U && u0 < p.n_units) {
             bool v;
             const uint16_t* r = unit_row<EPI>(p, u0, lane, v);
             const uint32_t bytes = (uint32_t)min(K * 2, 32768);
@@ -1091,6 +1092,34 @@ __global__ void generate_kernel(uint16_t* out, uint64_t n, uint64_t first, uint6
     for (; i < n; i += stride) out[i] = gen_elem(seed, tensor_id, first + i, kind);
 }
 
+// 128-bit streaming reads of n16 vectors, four in flight per thread; one
+// xor-fold per block keeps every load live.
+__global__ void __launch_bounds__(256) read_stream_kernel(const uint4* src, uint64_t n16, uint32_t* sink) {
+    __shared__ uint32_t s_x[8];
+    uint32_t x = 0;
+    const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+    uint64_t i = blockIdx.x * (uint64_t)blockDim.x + threadIdx.x;
+    for (; i + 3 * stride < n16; i += 4 * stride) {
+        uint4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) v[u] = ld_stream(reinterpret_cast<const uint16_t*>(src + i + u * stride));
+#pragma unroll
+        for (int u = 0; u < 4; ++u) x ^= v[u].x ^ v[u].y ^ v[u].z ^ v[u].w;
+    }
+    for (; i < n16; i += stride) {
+        const uint4 v = ld_stream(reinterpret_cast<const uint16_t*>(src + i));
+        x ^= v.x ^ v.y ^ v.z ^ v.w;
+    }
+    for (int o = 16; o; o >>= 1) x ^= __shfl_xor_sync(0xffffffffu, x, o);
+    if ((threadIdx.x & 31) == 0) s_x[threadIdx.x >> 5] = x;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t t = 0;
+        for (int w = 0; w < 8; ++w) t ^= s_x[w];
+        sink[blockIdx.x] = t;
+    }
+}
+
 }  // namespace
 
 // ----------------------------------------------------------------------------
@@ -1098,8 +1127,9 @@ __global__ void generate_kernel(uint16_t* out, uint64_t n, uint64_t first, uint6
 // ----------------------------------------------------------------------------
 cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
                             int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
-                            const int32_t* row_req, cudaStream_t st, bool pdl) {
+                            const int32_t* row_req, cudaStream_t st, bool pdl, bool w_host) {
     GemvParams p{};
+    p.w_host = w_host;
     p.in = x;
     p.g = g;
     p.w0 = wqkv;
@@ -1120,8 +1150,9 @@ cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* w
 }
 
 cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st,
-                              bool pdl) {
+                              bool pdl, bool w_host) {
     GemvParams p{};
+    p.w_host = w_host;
     p.in = in;
     p.w0 = w;
     p.B = B;
@@ -1133,8 +1164,9 @@ cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, 
 }
 
 cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,
-                           int F, float eps, float* a, cudaStream_t st, bool pdl) {
+                           int F, float eps, float* a, cudaStream_t st, bool pdl, bool w_host) {
     GemvParams p{};
+    p.w_host = w_host;
     p.in = x;
     p.g = g;
     p.w0 = wg;
@@ -1238,6 +1270,11 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
 cudaError_t launch_embed(const uint16_t* embed, const int32_t* tokens, int B, int H, int V, float* x,
                          cudaStream_t st, bool pdl) {
     return launch_k(embed_kernel, dim3(B), dim3(256), 0, st, pdl, embed, tokens, H, V, x);
+}
+
+cudaError_t launch_read_stream(const void* src, uint64_t bytes, int blocks, uint32_t* sink, cudaStream_t st) {
+    return launch_k(read_stream_kernel, dim3(blocks), dim3(256), 0, st, false, reinterpret_cast<const uint4*>(src),
+                    bytes / 16, sink);
 }
 
 cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st, bool pdl) {

@@ -11,7 +11,8 @@
 // so a buffer is an anonymous mapping aligned to the huge-page size, advised
 // MADV_HUGEPAGE, written through once in address order (which also faults its
 // pages in), then registered with cudaHostRegister; cudaHostAlloc is the
-// fallback when that fails.
+// fallback when that fails.  Every buffer is registered mapped, so kernels can
+// also read it in place through its device address (direct-access decode).
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -37,6 +38,18 @@ static size_t huge_page_bytes() {
     return hp;
 }
 
+// Device address of the buffer on the current device (nullptr when the driver
+// cannot map it; direct-access users check for that).
+static void map_device(HostBuf* b) {
+    void* d = nullptr;
+    if (cudaHostGetDevicePointer(&d, b->ptr, 0) == cudaSuccess) {
+        b->dev = d;
+    } else {
+        cudaGetLastError();
+        b->dev = nullptr;
+    }
+}
+
 cudaError_t host_buf_alloc(size_t bytes, HostBuf* out) {
     *out = HostBuf{};
     if (bytes == 0) return cudaSuccess;
@@ -44,10 +57,11 @@ cudaError_t host_buf_alloc(size_t bytes, HostBuf* out) {
     static const char* mode = getenv("LOIP_HOST_POOL");
     if (mode && strcmp(mode, "hostalloc") == 0) {
         void* q = nullptr;
-        cudaError_t e = cudaHostAlloc(&q, bytes, cudaHostAllocDefault);
+        cudaError_t e = cudaHostAlloc(&q, bytes, cudaHostAllocPortable | cudaHostAllocMapped);
         if (e != cudaSuccess) return e;
         out->ptr = q;
         out->bytes = bytes;
+        map_device(out);
         return cudaSuccess;
     }
     const size_t hp = huge_page_bytes();
@@ -57,23 +71,25 @@ cudaError_t host_buf_alloc(size_t bytes, HostBuf* out) {
         char* p = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(base) + hp - 1) / hp * hp);
         madvise(p, bytes, MADV_HUGEPAGE);
         memset(p, 0, bytes);
-        if (cudaHostRegister(p, bytes, cudaHostRegisterDefault) == cudaSuccess) {
+        if (cudaHostRegister(p, bytes, cudaHostRegisterPortable | cudaHostRegisterMapped) == cudaSuccess) {
             out->base = base;
             out->map_bytes = map_bytes;
             out->ptr = p;
             out->bytes = bytes;
             out->mapped = true;
+            map_device(out);
             return cudaSuccess;
         }
         cudaGetLastError();  // clear the failed registration
         munmap(base, map_bytes);
     }
     void* q = nullptr;
-    cudaError_t e = cudaHostAlloc(&q, bytes, cudaHostAllocDefault);
+    cudaError_t e = cudaHostAlloc(&q, bytes, cudaHostAllocPortable | cudaHostAllocMapped);
     if (e != cudaSuccess) return e;
     out->ptr = q;
     out->bytes = bytes;
     out->mapped = false;
+    map_device(out);
     return cudaSuccess;
 }
 

@@ -10,6 +10,7 @@ struct HostBuf {
     void* ptr = nullptr;   // usable, registered pointer
     size_t bytes = 0;
     bool mapped = false;   // mmap + cudaHostRegister (else cudaHostAlloc)
+    void* dev = nullptr;   // device address of ptr (registered mapped), or nullptr
 };
 cudaError_t host_buf_alloc(size_t bytes, HostBuf* out);
 void host_buf_free(HostBuf* b);

@@ -37,14 +37,20 @@ struct KvView {
 };
 
 // Weight-stationary matrix-vector family (decode).  B = batch rows of the fp32
-// activation; every kernel streams its weight matrix exactly once.
+// activation; every kernel streams its weight matrix exactly once.  w_host: the
+// weight pointer is the device address of mapped host memory (direct access
+// over the host link); the kernels then skip their L2 prefetch of it.
 cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
                             int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
-                            const int32_t* row_req, cudaStream_t st, bool pdl = false);
+                            const int32_t* row_req, cudaStream_t st, bool pdl = false, bool w_host = false);
 cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st,
-                              bool pdl = false);
+                              bool pdl = false, bool w_host = false);
 cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,
-                           int F, float eps, float* a, cudaStream_t st, bool pdl = false);
+                           int F, float eps, float* a, cudaStream_t st, bool pdl = false, bool w_host = false);
+// Streams `bytes` (a multiple of 16) from `src` with 128-bit loads over `blocks`
+// blocks and writes one xor-fold per block to sink[blocks] (so no load is
+// dropped).  Used to measure how fast kernels read mapped host memory.
+cudaError_t launch_read_stream(const void* src, uint64_t bytes, int blocks, uint32_t* sink, cudaStream_t st);
 cudaError_t launch_lm_head(const float* x, const uint16_t* g, const uint16_t* w, int B, int H, int V, float eps,
                            float* z, float* logits, int32_t* tokens, void* scratch, cudaStream_t st,
                            bool pdl = false);

@@ -409,7 +409,35 @@ struct loip_ctx {
     // ---- one decoder layer ---------------------------------------------------
     // Decode-time layer on rows 0..B-1 of the fixed activations.
     int decode_layer(int l, int B, const int32_t* pos_dev, cudaStream_t s, int slot) {
-        const uint16_t* w = layer_weights(l, slot);
+        return decode_layer_w(l, B, pos_dev, s, layer_weights(l, slot), false);
+    }
+
+    // Device address of offloaded layer l's host blob (mapped pinned memory).
+    const uint16_t* host_direct(int l) {
+        const char* h = static_cast<const char*>(host_layer[l]);
+        if (!h) return nullptr;
+        for (const HostBuf& r : host_regions) {
+            const char* p = static_cast<const char*>(r.ptr);
+            if (r.dev && h >= p && h + lay.l_size <= p + r.bytes)
+                return reinterpret_cast<const uint16_t*>(static_cast<const char*>(r.dev) + (h - p));
+        }
+        return nullptr;
+    }
+
+    // Decode over every layer with the offloaded ones read in place from host
+    // memory: no slots, no copy stream.
+    int run_layers_direct(int B, const int32_t* pos_dev, cudaStream_t s) {
+        for (int l = 0; l < L; ++l) {
+            const bool off = layer_block[l] < 0;
+            const uint16_t* w = off ? host_direct(l) : layer_weights(l, -1);
+            if (!w) return fail(LOIP_ERR_STATE, "offloaded layer has no device-mapped host copy");
+            int rc = decode_layer_w(l, B, pos_dev, s, w, off);
+            if (rc) return rc;
+        }
+        return LOIP_OK;
+    }
+
+    int decode_layer_w(int l, int B, const int32_t* pos_dev, cudaStream_t s, const uint16_t* w, bool w_host) {
         const uint16_t* g_attn = w + lay.off_g_attn / 2;
         const uint16_t* wqkv = w + lay.off_wqkv / 2;
         const uint16_t* wo = w + lay.off_wo / 2;
@@ -426,7 +454,7 @@ struct loip_ctx {
         cudaError_t e;
         e = timed(0, s, [&] {
             return launch_qkv_rope(x, g_attn, wqkv, B, H, Hq, Hkv, d, desc.rms_eps, desc.rope_theta, pos_dev, q, kv,
-                                   nullptr, s, pdl());
+                                   nullptr, s, pdl(), w_host);
         });
         if (e != cudaSuccess) return cuda_fail(e, "qkv kernel");
         chain = true;
@@ -435,11 +463,13 @@ struct loip_ctx {
                                     fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl());
         });
         if (e != cudaSuccess) return cuda_fail(e, "attention kernel");
-        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl()); });
+        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl(), w_host); });
         if (e != cudaSuccess) return cuda_fail(e, "o-proj kernel");
-        e = timed(3, s, [&] { return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s, pdl()); });
+        e = timed(3, s, [&] {
+            return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s, pdl(), w_host);
+        });
         if (e != cudaSuccess) return cuda_fail(e, "gate/up kernel");
-        e = timed(4, s, [&] { return launch_resid_gemv(a, wd, B, H, F, x, s, pdl()); });
+        e = timed(4, s, [&] { return launch_resid_gemv(a, wd, B, H, F, x, s, pdl(), w_host); });
         if (e != cudaSuccess) return cuda_fail(e, "down kernel");
         return LOIP_OK;
     }
@@ -732,7 +762,8 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     if (cfg.n_slots < 1 || cfg.n_slots > 3 || cfg.max_batch < 1 || cfg.max_batch > 8 || cfg.max_ctx < 1 ||
         cfg.max_ctx > 16384 ||
         cfg.page_tokens != 64 || !device_arena || ((uintptr_t)device_arena % kAlign) ||
-        arena_bytes < cfg.device_budget_bytes || (cfg.mode != LOIP_MODE_OVERLAP && cfg.mode != LOIP_MODE_NAIVE)) {
+        arena_bytes < cfg.device_budget_bytes ||
+        (cfg.mode != LOIP_MODE_OVERLAP && cfg.mode != LOIP_MODE_NAIVE && cfg.mode != LOIP_MODE_DIRECT)) {
         g_create_error = "invalid configuration (slots 1..3, batch 1..8, page 64, arena >= budget, aligned)";
         return LOIP_ERR_INVALID;
     }
@@ -1047,7 +1078,10 @@ static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int3
     e = launch_embed(c->fixed_ptr<uint16_t>(c->fx.embed), d_tokens, B, c->H, c->V, x, s, false);
     if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
     c->chain = true;
-    rc = c->run_layers([&](int l, int slot) { return c->decode_layer(l, B, pos, s, slot); });
+    if (c->cfg.mode == LOIP_MODE_DIRECT)
+        rc = c->run_layers_direct(B, pos, s);
+    else
+        rc = c->run_layers([&](int l, int slot) { return c->decode_layer(l, B, pos, s, slot); });
     if (rc) return rc;
     e = c->timed(5, s, [&] {
         return launch_lm_head(x, c->fixed_ptr<uint16_t>(c->fx.g_final), c->fixed_ptr<uint16_t>(c->fx.lm_head), B, c->H,
@@ -1296,6 +1330,49 @@ extern "C" int loip_measure_h2d(uint64_t bytes, int32_t reps, double* out_Bps) {
     if (d) cudaFree(d);
     host_buf_free(&hb);
     if (e != cudaSuccess) return LOIP_ERR_CUDA;
+    *out_Bps = best;
+    return LOIP_OK;
+}
+
+extern "C" int loip_measure_direct_read(uint64_t bytes, int32_t reps, double* out_Bps) {
+    if (!out_Bps || bytes < (1u << 20) || (bytes & 15) || reps < 1) return LOIP_ERR_INVALID;
+    HostBuf hb;
+    if (host_buf_alloc(bytes, &hb) != cudaSuccess) return LOIP_ERR_OOM;
+    if (!hb.dev) {
+        host_buf_free(&hb);
+        return LOIP_ERR_CUDA;
+    }
+    memset(hb.ptr, 1, bytes);
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int blocks = std::max(1, sms) * 4;
+    uint32_t* sink = nullptr;
+    cudaStream_t s = nullptr;
+    cudaEvent_t a = nullptr, b = nullptr;
+    cudaError_t e = cudaMalloc(&sink, (size_t)blocks * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreate(&a);
+    if (e == cudaSuccess) e = cudaEventCreate(&b);
+    double best = 0;
+    for (int r = 0; r < reps + 1 && e == cudaSuccess; ++r) {
+        cudaEventRecord(a, s);
+        e = launch_read_stream(hb.dev, bytes, blocks, sink, s);
+        cudaEventRecord(b, s);
+        if (e == cudaSuccess) e = cudaEventSynchronize(b);
+        float ms = 0;
+        if (e == cudaSuccess && r > 0 && cudaEventElapsedTime(&ms, a, b) == cudaSuccess && ms > 0)
+            best = std::max(best, (double)bytes / (ms * 1e-3));
+    }
+    if (a) cudaEventDestroy(a);
+    if (b) cudaEventDestroy(b);
+    if (s) cudaStreamDestroy(s);
+    if (sink) cudaFree(sink);
+    host_buf_free(&hb);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return LOIP_ERR_CUDA;
+    }
     *out_Bps = best;
     return LOIP_OK;
 }

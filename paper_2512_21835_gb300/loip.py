@@ -16,7 +16,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libloip.so")
 
 OK, ERR_INVALID, ERR_OOM, ERR_INFEASIBLE, ERR_CUDA, ERR_TIMEOUT, ERR_STATE = range(7)
-MODE_OVERLAP, MODE_NAIVE = 0, 1
+MODE_OVERLAP, MODE_NAIVE, MODE_DIRECT = 0, 1, 2
 _NAMES = {1: "INVALID", 2: "OOM", 3: "INFEASIBLE", 4: "CUDA", 5: "TIMEOUT", 6: "STATE"}
 
 
@@ -84,6 +84,7 @@ _SIGS = {
     "loip_synchronize": (C.c_int, [P]),
     "loip_set_kernel_timing": (C.c_int, [P, I32]),
     "loip_measure_h2d": (C.c_int, [U64, I32, C.POINTER(C.c_double)]),
+    "loip_measure_direct_read": (C.c_int, [U64, I32, C.POINTER(C.c_double)]),
     "loip_compute_stream": (C.c_void_p, [P]),
     "loip_copy_stream": (C.c_void_p, [P]),
     "loip_k_generate": (C.c_int, [P, U64, U64, U64, U32, I32, P]),
@@ -186,6 +187,13 @@ def loip_measure_h2d(nbytes: int = 1 << 30, reps: int = 5) -> float:
     """Host-to-device copy throughput (bytes/s) from the pool's kind of pinned memory."""
     out = C.c_double()
     _check(lib().loip_measure_h2d(nbytes, reps, C.byref(out)))
+    return out.value
+
+
+def loip_measure_direct_read(nbytes: int = 1 << 30, reps: int = 5) -> float:
+    """Throughput (bytes/s) of a kernel streaming mapped pinned host memory."""
+    out = C.c_double()
+    _check(lib().loip_measure_direct_read(nbytes, reps, C.byref(out)))
     return out.value
 
 

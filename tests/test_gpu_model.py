@@ -86,7 +86,8 @@ def test_tiny_prefill_decode_matches_oracle(torch, L, orc):
     assert exempt == 0
 
 
-@pytest.mark.parametrize("resident,K,mode", [(6, 2, 0), (3, 2, 0), (0, 1, 0), (2, 3, 0), (1, 2, 0), (4, 1, 1)])
+@pytest.mark.parametrize("resident,K,mode", [(6, 2, 0), (3, 2, 0), (0, 1, 0), (2, 3, 0), (1, 2, 0), (4, 1, 1),
+                                             (2, 2, 2), (0, 1, 2)])
 def test_offload_is_bitwise_lossless(torch, L, orc, resident, K, mode):
     prompts = [inputs.token_ids(7, 20, TINY6["vocab"]), inputs.token_ids(8, 9, TINY6["vocab"])]
     cont = [[int(a), int(b)] for a, b in zip(inputs.token_ids(9, 6, 1024), inputs.token_ids(10, 6, 1024))]
@@ -160,3 +161,30 @@ def test_multi_head_model_matches_oracle(torch, L, orc):
         t = P - 1 + i
         _check_hidden(hids[i][0], ref["hidden"][t])
         assert int(toks[i][0]) == int(ref["argmax"][t])
+
+
+def test_direct_access_decode_copies_nothing(torch, L, orc):
+    """LOIP_MODE_DIRECT: decode steps read the offloaded layers in place from the
+    host pool (no weight copies after the prefill's) and stay bit-identical to
+    the all-resident run."""
+    m = TINY6
+    prompts = [inputs.token_ids(51, 30, m["vocab"])]
+    cont = [[int(t)] for t in inputs.token_ids(52, 8, m["vocab"])]
+    base = _run(L, torch, m, prompts, cont, dict(max_batch=1, max_ctx=64), 6)
+    kw = dict(max_batch=1, max_ctx=64, n_slots=2, mode=L.MODE_DIRECT)
+    ctx = L.Context(m, L.config(budget=_budget(L, m, kw, 2), **kw))
+    assert ctx.plan()["n_offloaded"] == 4
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    hid = torch.empty(1, m["hidden"], dtype=torch.float32, device="cuda")
+    toks = [ctx.prefill(prompts, out_hidden=hid)]
+    hids = [hid.cpu().numpy().copy()]
+    ctx.synchronize()
+    after_prefill = ctx.stats()["h2d_weight_bytes"]
+    for step in cont:
+        toks.append(ctx.decode_step(step, out_hidden=hid))
+        hids.append(hid.cpu().numpy().copy())
+    ctx.synchronize()
+    assert ctx.stats()["h2d_weight_bytes"] == after_prefill
+    ctx.close()
+    assert np.array_equal(np.array(toks), base[0])
+    assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
