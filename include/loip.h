@@ -66,7 +66,9 @@ typedef struct loip_config {
     int32_t page_tokens;          /* KV page size in tokens (64) */
     int32_t max_batch;            /* largest decode batch (<= 8) */
     int32_t max_ctx;              /* largest context per request, tokens */
-    int32_t use_graphs;           /* capture decode steps as CUDA graphs */
+    int32_t per_op_kernels;       /* 0: at batch 1, each run of consecutive resident layers is
+                                   * computed by one persistent kernel (grid barriers between
+                                   * the phases of a layer); 1: one kernel launch per operation */
     int32_t mode;                 /* LOIP_MODE_OVERLAP, LOIP_MODE_NAIVE or LOIP_MODE_DIRECT */
     uint32_t timeout_ms;          /* deadline of every host wait (0 = 600000) */
     double hbm_Bps;               /* bandwidths used by the planner's step model */
@@ -104,9 +106,11 @@ typedef struct loip_stats {
     uint64_t arena_used;       /* device arena bytes in use */
     /* per kernel class, accumulated while kernel timing is on (loip_set_kernel_timing):
      * decode: 0 qkv+rope, 1 attention (+combine), 2 o-proj, 3 gate/up, 4 down, 5 lm head (+argmax);
-     * prefill: 6 qkv GEMM, 7 attention, 8 o-proj GEMM, 9 gate/up GEMM, 10 down GEMM, 11 RMSNorm */
-    double kernel_ms[12];
-    uint64_t kernel_launches[12];
+     * prefill: 6 qkv GEMM, 7 attention, 8 o-proj GEMM, 9 gate/up GEMM, 10 down GEMM, 11 RMSNorm;
+     * 12 persistent layer run (decode at batch 1, a run of resident layers in one launch);
+     * 13-15 unused */
+    double kernel_ms[16];
+    uint64_t kernel_launches[16];
     double copy_ms_total;      /* summed duration of every completed layer copy (events) */
     uint64_t copies_total;     /* number of completed layer copies */
     double pool_min_GBps;      /* slowest host-pool blob copy when the pool was qualified */

@@ -492,15 +492,49 @@ __device__ __forceinline__ void tile_load(uint4 (&w)[kTileRows], const uint16_t*
     for (int r = 0; r < kTileRows; ++r) w[r] = (ok && rv[r]) ? ld_stream(rp[r] + k) : make_uint4(0, 0, 0, 0);
 }
 
+// Issues the first batch of tile `tile`'s weight loads into w (this warp's
+// first 256-column slice of every row).
 template <int EPI>
-__global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParams p) {
+__device__ __forceinline__ void tile_first_load(const GemvParams& p, int tile, uint4 (&w)[kTileRows]) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nj = (p.K + 255) >> 8, njw = (nj + kTileWarps - 1) / kTileWarps;
+    const int j_begin = warp * njw, j_end = min(nj, j_begin + njw);
+    const uint16_t* rp[kTileRows];
+    bool rv[kTileRows];
+#pragma unroll
+    for (int r = 0; r < kTileRows; ++r) rp[r] = tile_row<EPI>(p, tile, r, rv[r]);
+    tile_load(w, rp, rv, j_begin, j_end, p.K, lane);
+}
+
+struct TileShared {
+    float part[kTileWarps][kTileRows];
+    float ss[kTileWarps];
+    float val[kTileRows];
+    float inv;
+};
+
+// Activation loads.  CG: through L2 only -- the persistent layer-run kernel
+// rewrites activations between its phases and L1 is not coherent across SMs.
+template <bool CG>
+__device__ __forceinline__ float4 ld_act4(const float* p) {
+    if (CG) return __ldcg(reinterpret_cast<const float4*>(p));
+    return *reinterpret_cast<const float4*>(p);
+}
+template <bool CG>
+__device__ __forceinline__ float ld_act(const float* p) {
+    return CG ? __ldcg(p) : *p;
+}
+
+// One tile of the batch-1 block-tile GEMV.  wa holds the first batch of the
+// tile's loads (tile_first_load).  When next >= 0, the first batch of tile
+// `next` is issued into wa as soon as this tile's loads are consumed, so its
+// weights stream during this tile's reduction and epilogue.
+template <int EPI, bool CG>
+__device__ __forceinline__ void tile_gemv(const GemvParams& p, int tile, int next, uint4 (&wa)[kTileRows],
+                                          TileShared& sm) {
     constexpr int R = kTileRows;
-    __shared__ float s_part[kTileWarps][R];
-    __shared__ float s_ss[kTileWarps];
-    __shared__ float s_val[R];
-    __shared__ float s_inv;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int tile = blockIdx.x, K = p.K;
+    const int K = p.K;
     const int nj = (K + 255) >> 8;
     const int njw = (nj + kTileWarps - 1) / kTileWarps;
     const int j_begin = warp * njw, j_end = min(nj, j_begin + njw);
@@ -510,11 +544,7 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParam
 #pragma unroll
     for (int r = 0; r < R; ++r) rp[r] = tile_row<EPI>(p, tile, r, rv[r]);
 
-    pdl_trigger();
-    uint4 wa[R], wb[R];
-    tile_load(wa, rp, rv, j_begin, j_end, K, lane);  // weights do not depend on the previous kernel
-    pdl_wait();
-
+    uint4 wb[R];
     float acc[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) acc[r] = 0.f;
@@ -522,8 +552,8 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParam
     auto consume = [&](const uint4 (&w)[R], int j) {
         const int k = j * 256 + lane * 8;
         if (j >= j_end || k >= K) return;
-        const float4 xa = *reinterpret_cast<const float4*>(p.in + k);
-        const float4 xb = *reinterpret_cast<const float4*>(p.in + k + 4);
+        const float4 xa = ld_act4<CG>(p.in + k);
+        const float4 xb = ld_act4<CG>(p.in + k + 4);
         float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
         if (norm) {
             const uint4 gv = *reinterpret_cast<const uint4*>(p.g + k);
@@ -555,36 +585,37 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParam
         tile_load(wa, rp, rv, j + 2, j_end, K, lane);
         consume(wb, j + 1);
     }
+    if (next >= 0) tile_first_load<EPI>(p, next, wa);
 #pragma unroll
     for (int r = 0; r < R; ++r) {
         const float v = warp_sum(acc[r]);
-        if (lane == 0) s_part[warp][r] = v;
+        if (lane == 0) sm.part[warp][r] = v;
     }
     if (norm) {
         const float v = warp_sum(ss);
-        if (lane == 0) s_ss[warp] = v;
+        if (lane == 0) sm.ss[warp] = v;
     }
     __syncthreads();
     if (tid < R) {
         float t = 0.f;
-        for (int w = 0; w < kTileWarps; ++w) t += s_part[w][tid];
-        s_val[tid] = t;
+        for (int w = 0; w < kTileWarps; ++w) t += sm.part[w][tid];
+        sm.val[tid] = t;
     }
     if (tid == 32) {
         float t = 0.f;
         if (norm)
-            for (int w = 0; w < kTileWarps; ++w) t += s_ss[w];
-        s_inv = norm ? 1.0f / sqrtf(t / (float)K + p.eps) : 1.0f;
+            for (int w = 0; w < kTileWarps; ++w) t += sm.ss[w];
+        sm.inv = norm ? 1.0f / sqrtf(t / (float)K + p.eps) : 1.0f;
     }
     __syncthreads();
-    const float inv = s_inv;
+    const float inv = sm.inv;
     if (EPI == EPI_QKV) {
         if (tid < R / 2) {
             const int half = p.d >> 1;
             const int pair = tile * (R / 2) + tid;
             if (pair < p.n_units) {
                 const int h = pair / half, i = pair - h * half;
-                float v0 = s_val[tid] * inv, v1 = s_val[tid + R / 2] * inv;
+                float v0 = sm.val[tid] * inv, v1 = sm.val[tid + R / 2] * inv;
                 const int pos = p.positions[0];
                 if (h < p.Hq + p.Hkv) {
                     float cf, sf;
@@ -611,26 +642,26 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParam
         if (tid < R / 2) {
             const int j = tile * (R / 2) + tid;
             if (j < p.n_units) {
-                const float gt = s_val[tid] * inv, ut = s_val[tid + R / 2] * inv;
+                const float gt = sm.val[tid] * inv, ut = sm.val[tid + R / 2] * inv;
                 p.out[j] = gt / (1.0f + expf(-gt)) * ut;
             }
         }
     } else if (EPI == EPI_RESID) {
         if (tid < R) {
             const int row = tile * R + tid;
-            if (row < p.N) p.out[row] += s_val[tid];
+            if (row < p.N) p.out[row] = ld_act<CG>(p.out + row) + sm.val[tid];
         }
     } else {  // EPI_LOGITS
         if (tid < R) {
             const int row = tile * R + tid;
-            if (row < p.N && p.out) p.out[row] = s_val[tid] * inv;
+            if (row < p.N && p.out) p.out[row] = sm.val[tid] * inv;
         }
         if (tid == 0) {
             uint64_t best = 0;
             for (int r = 0; r < R; ++r) {
                 const int row = tile * R + r;
                 if (row < p.N) {
-                    const uint64_t key = argmax_key(s_val[r] * inv, (uint32_t)row);
+                    const uint64_t key = argmax_key(sm.val[r] * inv, (uint32_t)row);
                     best = key > best ? key : best;
                 }
             }
@@ -639,6 +670,17 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParam
         if (tile == 0 && p.z)
             for (int k = tid; k < K; k += kTileWarps * 32) p.z[k] = p.in[k] * inv * bf2f(p.g[k]);
     }
+    __syncthreads();  // the shared partials are reused by the block's next tile
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParams p) {
+    __shared__ TileShared sm;
+    pdl_trigger();
+    uint4 wa[kTileRows];
+    tile_first_load<EPI>(p, blockIdx.x, wa);  // weights do not depend on the previous kernel
+    pdl_wait();
+    tile_gemv<EPI, false>(p, blockIdx.x, -1, wa, sm);
 }
 
 __global__ void argmax_reduce_kernel(const uint64_t* keys, int nblocks, int BT, int B, int32_t* tokens) {
@@ -774,35 +816,44 @@ __device__ __forceinline__ void cp_async_wait_all() {
     asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
 }
 
-// One block per (request row, kv head, page) in split mode, or per (row, kv
-// head) looping over the pages otherwise.  The page's keys and values (64
-// positions x d, bf16) are staged in shared memory with asynchronous 16-byte
-// copies, all in flight together; key rows are stored with their 16-byte chunks
-// rotated by the row index so that one-row-per-lane reads hit distinct banks.
-// Each of the two warps scores 32 positions for the G query heads of the kv
-// head (online softmax), then accumulates the values with the weights
-// broadcast by shuffles; the two warps merge through shared memory.
 template <int G, int D>
-__global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
+struct AttnSmem {
+    alignas(16) uint16_t sK[64 * D];
+    alignas(16) uint16_t sV[64 * D];
+    alignas(16) float sq[G][D];
+    float s_m[G], s_l[G];
+    float s_o[G][D];
+    int s_last;
+};
+
+// Barrier among the 64 threads of one attention group (barrier 0 with 64
+// threads is the whole block of the standalone kernel; the layer-run kernel
+// gives each warp pair a barrier of its own).
+__device__ __forceinline__ void group_sync(int bar_id) { asm volatile("bar.sync %0, 64;" ::"r"(bar_id) : "memory"); }
+
+// Attention of one (request row, kv head) over pages [pg0, pg1) by a group of
+// two warps (tid 0..63).  The page's keys and values (64 positions x d, bf16)
+// are staged in shared memory with asynchronous 16-byte copies, all in flight
+// together; key rows are stored with their 16-byte chunks rotated by the row
+// index so that one-row-per-lane reads hit distinct banks.  Each warp scores 32
+// positions for the G query heads of the kv head (online softmax), then
+// accumulates the values with the weights broadcast by shuffles; the two warps
+// merge through shared memory.  Split mode (one group per page, `chunk` = page):
+// the partial state goes to scratch and the last group of this (row, kv head)
+// to finish combines every page's state.  CG: activations and partial states
+// are read through L2 only (the layer-run kernel reuses their addresses).
+template <int G, int D, bool CG>
+__device__ __forceinline__ void attn_group(const AttnParams& p, int row, int kvh, int chunk, AttnSmem<G, D>& sm,
+                                           int tid, int bar_id) {
     constexpr int DPL = D / 32;  // dims per lane in the PV product
     constexpr int CH = D / 8;    // 16-byte chunks per row
-    __shared__ __align__(16) uint16_t sK[64 * D];
-    __shared__ __align__(16) uint16_t sV[64 * D];
-    __shared__ __align__(16) float sq[G][D];
-    __shared__ float s_m[G], s_l[G];
-    __shared__ float s_o[G][D];
-    __shared__ int s_last;
-
-    pdl_trigger();
-    pdl_wait();
-    const int row = blockIdx.z, kvh = blockIdx.y;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int lane = tid & 31, warp = tid >> 5;
     const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
     const int P = p.kv.page_tokens;  // 64
     const int npages = (ctx + P - 1) / P;
     int pg0, pg1;
     if (p.split) {
-        pg0 = blockIdx.x;
+        pg0 = chunk;
         pg1 = pg0 + 1;
         if (pg0 >= npages) return;
     } else {
@@ -811,14 +862,14 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
     }
     const int req = p.row_req ? p.row_req[row] : row;
     {
-        const float4* qs = reinterpret_cast<const float4*>(p.q + (size_t)row * p.Hq * D + (size_t)kvh * G * D);
+        const float* qs = p.q + (size_t)row * p.Hq * D + (size_t)kvh * G * D;
         constexpr int NQ = G * D / 4 / 64;  // float4 per thread (G * D is a multiple of 256)
         float4 qv[NQ > 0 ? NQ : 1];
 #pragma unroll
-        for (int u = 0; u < NQ; ++u) qv[u] = qs[tid + u * 64];
+        for (int u = 0; u < NQ; ++u) qv[u] = ld_act4<CG>(qs + 4 * (tid + u * 64));
 #pragma unroll
-        for (int u = 0; u < NQ; ++u) reinterpret_cast<float4*>(&sq[0][0])[tid + u * 64] = qv[u];
-        if (NQ == 0 && tid < G * D / 4) reinterpret_cast<float4*>(&sq[0][0])[tid] = qs[tid];
+        for (int u = 0; u < NQ; ++u) reinterpret_cast<float4*>(&sm.sq[0][0])[tid + u * 64] = qv[u];
+        if (NQ == 0 && tid < G * D / 4) reinterpret_cast<float4*>(&sm.sq[0][0])[tid] = ld_act4<CG>(qs + 4 * tid);
     }
 
     float m[G], l[G], o[G][DPL];
@@ -836,35 +887,35 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
                            (uint64_t)p.kv.layer * p.kv.layer_page_bytes;
         const uint16_t* Kh = reinterpret_cast<const uint16_t*>(page) + (size_t)kvh * P * D;
         const uint16_t* Vh = reinterpret_cast<const uint16_t*>(page) + ((size_t)Hkv + kvh) * P * D;
-        if (pg != pg0) __syncthreads();  // the previous page's rows are no longer read
+        if (pg != pg0) group_sync(bar_id);  // the previous page's rows are no longer read
         for (int i = tid; i < 64 * CH; i += 64) {
             const int t = i / CH, c = i - t * CH;
             if (t < nvalid) {
-                cp_async16(&sK[(t * CH + ((c + t) & (CH - 1))) * 8], Kh + (size_t)t * D + c * 8);
-                cp_async16(&sV[(t * CH + c) * 8], Vh + (size_t)t * D + c * 8);
+                cp_async16(&sm.sK[(t * CH + ((c + t) & (CH - 1))) * 8], Kh + (size_t)t * D + c * 8);
+                cp_async16(&sm.sV[(t * CH + c) * 8], Vh + (size_t)t * D + c * 8);
             } else {
-                *reinterpret_cast<uint4*>(&sV[(t * CH + c) * 8]) = make_uint4(0, 0, 0, 0);
+                *reinterpret_cast<uint4*>(&sm.sV[(t * CH + c) * 8]) = make_uint4(0, 0, 0, 0);
             }
         }
         cp_async_wait_all();
-        __syncthreads();
+        group_sync(bar_id);
         {
             const int tl = warp * 32 + lane;
             const bool valid = tl < nvalid;
-            float s[G];
+            float sc[G];
 #pragma unroll
-            for (int g = 0; g < G; ++g) s[g] = 0.f;
+            for (int g = 0; g < G; ++g) sc[g] = 0.f;
             if (valid) {
 #pragma unroll 4
                 for (int u = 0; u < CH; ++u) {
-                    const uint4 kk = *reinterpret_cast<const uint4*>(&sK[(tl * CH + ((u + tl) & (CH - 1))) * 8]);
+                    const uint4 kk = *reinterpret_cast<const uint4*>(&sm.sK[(tl * CH + ((u + tl) & (CH - 1))) * 8]);
                     const float kf[8] = {bf_lo(kk.x), bf_hi(kk.x), bf_lo(kk.y), bf_hi(kk.y),
                                          bf_lo(kk.z), bf_hi(kk.z), bf_lo(kk.w), bf_hi(kk.w)};
 #pragma unroll
                     for (int g = 0; g < G; ++g) {
-                        const float4 qa = *reinterpret_cast<const float4*>(&sq[g][u * 8]);
-                        const float4 qb = *reinterpret_cast<const float4*>(&sq[g][u * 8 + 4]);
-                        float a = s[g];
+                        const float4 qa = *reinterpret_cast<const float4*>(&sm.sq[g][u * 8]);
+                        const float4 qb = *reinterpret_cast<const float4*>(&sm.sq[g][u * 8 + 4]);
+                        float a = sc[g];
                         a = fmaf(qa.x, kf[0], a);
                         a = fmaf(qa.y, kf[1], a);
                         a = fmaf(qa.z, kf[2], a);
@@ -873,14 +924,14 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
                         a = fmaf(qb.y, kf[5], a);
                         a = fmaf(qb.z, kf[6], a);
                         a = fmaf(qb.w, kf[7], a);
-                        s[g] = a;
+                        sc[g] = a;
                     }
                 }
             }
             float pe[G];
 #pragma unroll
             for (int g = 0; g < G; ++g) {
-                float sv = valid ? s[g] * p.scale : -INFINITY;
+                float sv = valid ? sc[g] * p.scale : -INFINITY;
                 float mx = warp_max(sv);
                 float mn = fmaxf(m[g], mx);
                 float corr = (m[g] == -INFINITY) ? 0.f : expf(m[g] - mn);
@@ -892,7 +943,7 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
             }
             const int nt = min(32, nvalid - warp * 32);
             for (int u = 0; u < nt; ++u) {
-                const uint16_t* vr = &sV[(warp * 32 + u) * D + lane * DPL];
+                const uint16_t* vr = &sm.sV[(warp * 32 + u) * D + lane * DPL];
                 float vf[DPL];
                 if constexpr (DPL == 4) {
                     const uint2 vv = *reinterpret_cast<const uint2*>(vr);
@@ -920,27 +971,27 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
 #pragma unroll
         for (int g = 0; g < G; ++g) {
             if (lane == 0) {
-                s_m[g] = m[g];
-                s_l[g] = l[g];
+                sm.s_m[g] = m[g];
+                sm.s_l[g] = l[g];
             }
 #pragma unroll
-            for (int c = 0; c < DPL; ++c) s_o[g][lane * DPL + c] = o[g][c];
+            for (int c = 0; c < DPL; ++c) sm.s_o[g][lane * DPL + c] = o[g][c];
         }
     }
-    __syncthreads();
+    group_sync(bar_id);
     if (warp == 0) {
 #pragma unroll
         for (int g = 0; g < G; ++g) {
-            float m1 = s_m[g], l1 = s_l[g];
+            float m1 = sm.s_m[g], l1 = sm.s_l[g];
             float mn = fmaxf(m[g], m1);
             float c0 = (m[g] == -INFINITY) ? 0.f : expf(m[g] - mn);
             float c1 = (m1 == -INFINITY) ? 0.f : expf(m1 - mn);
             float lt = l[g] * c0 + l1 * c1;
             const int h = kvh * G + g;
             if (p.split) {
-                float* part = p.scratch + (((size_t)row * p.Hq + h) * p.max_chunks + blockIdx.x) * (D + 2);
+                float* part = p.scratch + (((size_t)row * p.Hq + h) * p.max_chunks + chunk) * (D + 2);
 #pragma unroll
-                for (int c = 0; c < DPL; ++c) part[lane * DPL + c] = o[g][c] * c0 + s_o[g][lane * DPL + c] * c1;
+                for (int c = 0; c < DPL; ++c) part[lane * DPL + c] = o[g][c] * c0 + sm.s_o[g][lane * DPL + c] * c1;
                 if (lane == 0) {
                     part[D] = mn;
                     part[D + 1] = lt;
@@ -949,7 +1000,7 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
                 float invl = lt > 0.f ? 1.0f / lt : 0.f;
 #pragma unroll
                 for (int c = 0; c < DPL; ++c) {
-                    float v = (o[g][c] * c0 + s_o[g][lane * DPL + c] * c1) * invl;
+                    float v = (o[g][c] * c0 + sm.s_o[g][lane * DPL + c] * c1) * invl;
                     size_t idx = (size_t)row * p.Hq * D + (size_t)h * D + lane * DPL + c;
                     if (p.o_bf16)
                         reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(v);
@@ -960,33 +1011,33 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
         }
     }
     if (!p.split) return;
-    // The last block of this (row, kv head) to finish combines every page's
+    // The last group of this (row, kv head) to finish combines every page's
     // state: exp-weighted sum of the partial outputs over the summed weights.
     __threadfence();
-    __syncthreads();
+    group_sync(bar_id);
     if (tid == 0) {
         int* cnt = p.counters + (size_t)row * p.Hq + kvh;
         const int ticket = atomicAdd(cnt, 1);
-        s_last = ticket == npages - 1;
-        if (s_last) atomicExch(cnt, 0);  // every block of the group has arrived: reset for the next launch
+        sm.s_last = ticket == npages - 1;
+        if (sm.s_last) atomicExch(cnt, 0);  // every group has arrived: reset for the next launch
     }
-    __syncthreads();
-    if (!s_last) return;
+    group_sync(bar_id);
+    if (!sm.s_last) return;
     __threadfence();
     const float* base = p.scratch + ((size_t)row * p.Hq + (size_t)kvh * G) * p.max_chunks * (D + 2);
     const size_t hstride = (size_t)p.max_chunks * (D + 2);
     // the staging buffers are dead: combine weights and denominators reuse them
-    static_assert(G * kMaxChunks * sizeof(float) <= sizeof(sK), "combine weights fit the key stage");
-    float(*s_w)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sK[0]);
-    float(*s_lw)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sV[0]);
+    static_assert(G * kMaxChunks * sizeof(float) <= sizeof(sm.sK), "combine weights fit the key stage");
+    float(*s_w)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sm.sK[0]);
+    float(*s_lw)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sm.sV[0]);
     // (m, l) of every (head, page) in one round trip; weights reduced in shared memory
     for (int i = tid; i < G * npages; i += 64) {
         const int g = i / npages, c = i - g * npages;
         const float* pc = base + g * hstride + (size_t)c * (D + 2);
-        s_w[g][c] = pc[D];
-        s_lw[g][c] = pc[D + 1];
+        s_w[g][c] = ld_act<CG>(pc + D);
+        s_lw[g][c] = ld_act<CG>(pc + D + 1);
     }
-    __syncthreads();
+    group_sync(bar_id);
     for (int g = warp; g < G; g += 2) {
         float mx = -INFINITY;
         for (int c = lane; c < npages; c += 32) mx = fmaxf(mx, s_w[g][c]);
@@ -1001,7 +1052,7 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
         const float inv = lsum > 0.f ? 1.0f / lsum : 0.f;
         for (int c = lane; c < npages; c += 32) s_w[g][c] *= inv;
     }
-    __syncthreads();
+    group_sync(bar_id);
     // chunks outer, this thread's outputs inner: 4 x NOUT loads in flight
     constexpr int NOUT = G * D / 64;
     float acc[NOUT];
@@ -1014,7 +1065,7 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
 #pragma unroll
             for (int k = 0; k < NOUT; ++k) {
                 const int e = tid + 64 * k, g = e / D, j = e - g * D;
-                v[u][k] = (c0 + u < npages) ? base[g * hstride + (size_t)(c0 + u) * (D + 2) + j] : 0.f;
+                v[u][k] = (c0 + u < npages) ? ld_act<CG>(base + g * hstride + (size_t)(c0 + u) * (D + 2) + j) : 0.f;
             }
 #pragma unroll
         for (int u = 0; u < 4; ++u)
@@ -1035,10 +1086,291 @@ __global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
     }
 }
 
+// One block of two warps per (request row, kv head, page) in split mode, or per
+// (row, kv head) looping over the pages otherwise.
+template <int G, int D>
+__global__ void __launch_bounds__(64) attn_kernel(AttnParams p) {
+    __shared__ AttnSmem<G, D> sm;
+    pdl_trigger();
+    pdl_wait();
+    attn_group<G, D, false>(p, blockIdx.z, blockIdx.y, blockIdx.x, sm, threadIdx.x, 0);
+}
+
 template <int G, int D>
 cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st, bool pdl) {
     dim3 grid(p.split ? p.max_chunks : 1, p.Hkv, p.B);
     return launch_k(attn_kernel<G, D>, grid, dim3(64), 0, st, pdl, p);
+}
+
+// ----------------------------------------------------------------------------
+// Persistent layer run (batch 1)
+// ----------------------------------------------------------------------------
+// The per-operation kernels of a batch-1 decode layer stream 34-235 MB each;
+// every kernel boundary costs a ramp-up and a tail in which HBM idles, and
+// attention leaves it idle altogether.  One cooperative launch keeps 2 blocks
+// per SM resident through a run of resident layers: each phase hands out its
+// tiles round-robin, grid barriers separate dependent phases, and before each
+// barrier a block prefetches into L2 the first weight tile it will own in the
+// next phase (weights never depend on activations), so the next phase starts on
+// L2 hits.  During attention, the warps that hold no attention work prefetch
+// the O-projection tiles.  Activations are read through L2 (ld.global.cg).
+struct RunParams {
+    const char* base[kMaxRunLayers];
+    int n_layers, layer0;
+    uint64_t off_g_attn, off_wqkv, off_wo, off_g_mlp, off_wg, off_wu, off_wd;
+    int H, Hq, Hkv, d, F;
+    float eps;
+    float *x, *q, *o, *a;
+    const int32_t* positions;
+    KvView kv;
+    float* scratch;
+    int* counters;
+    int max_chunks;
+    unsigned* sync;
+    RopeFreqs rope;
+};
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Grid-wide barrier: every block arrives once per barrier on a monotonic
+// counter.  The wait is bounded (1 s); a block that gives up sets the error
+// word, and a block that sees the error word stops waiting, so every block
+// leaves the kernel instead of hanging.  Returns false on error.
+__device__ __forceinline__ bool grid_sync(unsigned* sync, unsigned& nsync, int* s_flag) {
+    __syncthreads();
+    ++nsync;
+    if (threadIdx.x == 0) {
+        __threadfence();
+        atomicAdd(&sync[0], 1u);
+        const unsigned target = nsync * gridDim.x;
+        const uint64_t t0 = globaltimer_ns();
+        int bad = 0;
+        while (ld_acquire_u32(&sync[0]) < target) {
+            if (*(volatile unsigned*)&sync[1]) {
+                bad = 1;
+                break;
+            }
+            if (globaltimer_ns() - t0 > 1000000000ull) {
+                atomicCAS(&sync[1], 0u, 1u);
+                bad = 1;
+                break;
+            }
+        }
+        __threadfence();
+        *s_flag = bad;
+    }
+    __syncthreads();
+    return *s_flag == 0;
+}
+
+// L2 prefetch of the weight rows of one tile (lanes 0..7 of the calling warp),
+// in pieces of at most 32 KB.
+template <int EPI>
+__device__ __forceinline__ void prefetch_tile(const GemvParams& p, int tile, int lane) {
+    if (lane < kTileRows) {
+        bool v;
+        const uint16_t* r = tile_row<EPI>(p, tile, lane, v);
+        if (v) {
+            const uint32_t bytes = (uint32_t)p.K * 2u;  // a multiple of 16 (K % 8 == 0)
+            for (uint32_t off = 0; off < bytes; off += 32768u)
+                prefetch_l2(reinterpret_cast<const char*>(r) + off, min(32768u, bytes - off));
+        }
+    }
+}
+
+template <int EPI>
+__device__ __forceinline__ int tile_count(const GemvParams& p) {
+    return (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? (p.n_units + kTileRows / 2 - 1) / (kTileRows / 2)
+                                                 : (p.N + kTileRows - 1) / kTileRows;
+}
+
+// This block's tiles of one phase, the next tile's first loads issued while the
+// current one reduces.
+template <int EPI>
+__device__ __forceinline__ void run_tiles(const GemvParams& p, TileShared& tsm) {
+    const int ntiles = tile_count<EPI>(p);
+    int t = blockIdx.x;
+    if (t >= ntiles) return;
+    uint4 wa[kTileRows];
+    tile_first_load<EPI>(p, t, wa);
+    while (t < ntiles) {
+        const int nxt = t + gridDim.x;
+        tile_gemv<EPI, true>(p, t, nxt < ntiles ? nxt : -1, wa, tsm);
+        t = nxt;
+    }
+}
+
+enum { PH_QKV = 0, PH_O = 1, PH_GU = 2, PH_D = 3 };
+
+template <int G, int D>
+__global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParams rp) {
+    extern __shared__ __align__(16) unsigned char run_smem[];
+    AttnSmem<G, D>* asm2 = reinterpret_cast<AttnSmem<G, D>*>(run_smem);  // one per attention group
+    __shared__ GemvParams s_gp[4];
+    __shared__ AttnParams s_ap;
+    __shared__ TileShared tsm;
+    __shared__ int s_flag;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int qd = rp.Hq * rp.d, nqkv = (rp.Hq + 2 * rp.Hkv) * rp.d;
+    // weight pointers of phase `ph` for layer `li` of the run
+    auto set_layer = [&](int ph, int li) {
+        const char* w = rp.base[li];
+        GemvParams& g = s_gp[ph];
+        if (ph == PH_QKV) {
+            g.g = reinterpret_cast<const uint16_t*>(w + rp.off_g_attn);
+            g.w0 = reinterpret_cast<const uint16_t*>(w + rp.off_wqkv);
+            g.kv.layer = rp.layer0 + li;
+        } else if (ph == PH_O) {
+            g.w0 = reinterpret_cast<const uint16_t*>(w + rp.off_wo);
+        } else if (ph == PH_GU) {
+            g.g = reinterpret_cast<const uint16_t*>(w + rp.off_g_mlp);
+            g.w0 = reinterpret_cast<const uint16_t*>(w + rp.off_wg);
+            g.w1 = reinterpret_cast<const uint16_t*>(w + rp.off_wu);
+        } else {
+            g.w0 = reinterpret_cast<const uint16_t*>(w + rp.off_wd);
+        }
+    };
+    if (tid == 0) {
+        for (int ph = 0; ph < 4; ++ph) {
+            GemvParams g{};
+            g.B = 1;
+            g.eps = rp.eps;
+            s_gp[ph] = g;
+        }
+        GemvParams& q = s_gp[PH_QKV];
+        q.in = rp.x;
+        q.K = rp.H;
+        q.N = nqkv;
+        q.n_units = nqkv / 2;
+        q.out = rp.q;
+        q.Hq = rp.Hq;
+        q.Hkv = rp.Hkv;
+        q.d = rp.d;
+        q.positions = rp.positions;
+        q.kv = rp.kv;
+        q.rope = rp.rope;
+        GemvParams& o = s_gp[PH_O];
+        o.in = rp.o;
+        o.K = qd;
+        o.N = rp.H;
+        o.n_units = rp.H;
+        o.out = rp.x;
+        GemvParams& gu = s_gp[PH_GU];
+        gu.in = rp.x;
+        gu.K = rp.H;
+        gu.N = rp.F;
+        gu.n_units = rp.F;
+        gu.out = rp.a;
+        GemvParams& dn = s_gp[PH_D];
+        dn.in = rp.a;
+        dn.K = rp.F;
+        dn.N = rp.H;
+        dn.n_units = rp.H;
+        dn.out = rp.x;
+        for (int ph = 0; ph < 4; ++ph) set_layer(ph, 0);
+        AttnParams a{};
+        a.q = rp.q;
+        a.kv = rp.kv;
+        a.positions = rp.positions;
+        a.B = 1;
+        a.Hq = rp.Hq;
+        a.Hkv = rp.Hkv;
+        a.max_chunks = rp.max_chunks;
+        a.scale = 1.0f / sqrtf((float)D);
+        a.scratch = rp.scratch;
+        a.counters = rp.counters;
+        a.o = rp.o;
+        a.split = 1;
+        s_ap = a;
+    }
+    __syncthreads();
+    if (warp == 0) prefetch_tile<EPI_QKV>(s_gp[PH_QKV], blockIdx.x, lane);
+    const int ctx = rp.positions[0] + 1;
+    const int npages = (ctx + rp.kv.page_tokens - 1) / rp.kv.page_tokens;
+    const int items = rp.Hkv * npages;
+    unsigned nsync = 0;
+    for (int li = 0; li < rp.n_layers; ++li) {
+        // ---- RMSNorm + QKV + RoPE + KV append
+        run_tiles<EPI_QKV>(s_gp[PH_QKV], tsm);
+        if (tid == 0) {
+            s_ap.kv.layer = rp.layer0 + li;
+            if (li + 1 < rp.n_layers) set_layer(PH_QKV, li + 1);
+        }
+        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        // ---- split attention (groups = warp pairs 0-1 and 2-3); warps 4-7
+        //      prefetch this block's O-projection tiles meanwhile
+        if (warp < 4) {
+            const int grp = warp >> 1;
+            for (int i = blockIdx.x + grp * gridDim.x; i < items; i += 2 * gridDim.x)
+                attn_group<G, D, true>(s_ap, 0, i / npages, i % npages, asm2[grp], tid & 63, 1 + grp);
+        } else {
+            const GemvParams& o = s_gp[PH_O];
+            const int nt = tile_count<EPI_RESID>(o);
+            const int k = warp - 4;  // tiles blockIdx + k * grid, at most 48 MB over the grid
+            const uint64_t tile_bytes = (uint64_t)kTileRows * o.K * 2;
+            const uint64_t kfit = (48ull << 20) / (tile_bytes * gridDim.x);
+            const int kmax = kfit < 1 ? 1 : (int)kfit;
+            for (int kk = k; kk < kmax && blockIdx.x + kk * gridDim.x < nt; kk += 4)
+                prefetch_tile<EPI_RESID>(o, blockIdx.x + kk * gridDim.x, lane);
+        }
+        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        // ---- O-projection + residual
+        run_tiles<EPI_RESID>(s_gp[PH_O], tsm);
+        if (warp == 0) prefetch_tile<EPI_SWIGLU>(s_gp[PH_GU], blockIdx.x, lane);
+        if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_O, li + 1);
+        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        // ---- RMSNorm + gate/up SwiGLU
+        run_tiles<EPI_SWIGLU>(s_gp[PH_GU], tsm);
+        if (warp == 0) prefetch_tile<EPI_RESID>(s_gp[PH_D], blockIdx.x, lane);
+        if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_GU, li + 1);
+        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        // ---- down + residual
+        run_tiles<EPI_RESID>(s_gp[PH_D], tsm);
+        if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_D, li + 1);
+        __syncthreads();
+        if (warp == 0 && li + 1 < rp.n_layers) prefetch_tile<EPI_QKV>(s_gp[PH_QKV], blockIdx.x, lane);
+        if (li + 1 < rp.n_layers && !grid_sync(rp.sync, nsync, &s_flag)) return;
+    }
+}
+
+template <int G, int D>
+cudaError_t launch_run_t(const RunParams& rp, cudaStream_t st) {
+    const size_t smem = 2 * sizeof(AttnSmem<G, D>);
+    static bool attr = false;
+    static int grid = 0;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(decode_run_kernel<G, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+        int dev = 0, sms = 0, per_sm = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_run_kernel<G, D>, kTileWarps * 32, smem);
+        if (e != cudaSuccess) return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        grid = sms * (per_sm < 2 ? per_sm : 2);
+        attr = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kTileWarps * 32);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeCooperative;  // all blocks co-resident: the grid barriers cannot deadlock
+    at[0].val.cooperative = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decode_run_kernel<G, D>, rp);
 }
 
 // ----------------------------------------------------------------------------
@@ -1230,7 +1562,7 @@ int* attention_counters(float* scratch, int B, int Hq, int d, int max_ctx, int p
 
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
-                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl) {
+                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl, int scratch_rows) {
     AttnParams p{};
     p.q = q;
     p.kv = kv;
@@ -1244,7 +1576,8 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
     if (split && p.max_chunks > kMaxChunks) return cudaErrorInvalidValue;
     p.scale = 1.0f / sqrtf((float)d);
     p.scratch = scratch;
-    p.counters = split ? attention_counters(scratch, B, Hq, d, max_ctx, kv.page_tokens) : nullptr;
+    if (scratch_rows < B) scratch_rows = B;
+    p.counters = split ? attention_counters(scratch, scratch_rows, Hq, d, max_ctx, kv.page_tokens) : nullptr;
     p.o = o;
     p.o_bf16 = o_bf16 ? 1 : 0;
     p.split = split ? 1 : 0;
@@ -1262,6 +1595,65 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
             case 2: return launch_attn_t<2, 64>(p, st, pdl);
             case 4: return launch_attn_t<4, 64>(p, st, pdl);
             case 8: return launch_attn_t<8, 64>(p, st, pdl);
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+bool decode_run_supported(int Hq, int Hkv, int d) {
+    const int G = Hkv > 0 ? Hq / Hkv : 0;
+    return (d == 64 || d == 128) && (G == 1 || G == 2 || G == 4 || G == 8) && Hq == G * Hkv;
+}
+
+cudaError_t launch_decode_run(const DecodeRunArgs& a, cudaStream_t st) {
+    if (a.n_layers < 1 || a.n_layers > kMaxRunLayers || !decode_run_supported(a.Hq, a.Hkv, a.d) || !a.sync)
+        return cudaErrorInvalidValue;
+    RunParams rp{};
+    for (int i = 0; i < a.n_layers; ++i) rp.base[i] = a.base[i];
+    rp.n_layers = a.n_layers;
+    rp.layer0 = a.layer0;
+    rp.off_g_attn = a.off_g_attn;
+    rp.off_wqkv = a.off_wqkv;
+    rp.off_wo = a.off_wo;
+    rp.off_g_mlp = a.off_g_mlp;
+    rp.off_wg = a.off_wg;
+    rp.off_wu = a.off_wu;
+    rp.off_wd = a.off_wd;
+    rp.H = a.H;
+    rp.Hq = a.Hq;
+    rp.Hkv = a.Hkv;
+    rp.d = a.d;
+    rp.F = a.F;
+    rp.eps = a.eps;
+    rp.x = a.x;
+    rp.q = a.q;
+    rp.o = a.o;
+    rp.a = a.a;
+    rp.positions = a.positions;
+    rp.kv = a.kv;
+    rp.scratch = a.attn_scratch;
+    rp.max_chunks = (a.max_ctx + a.kv.page_tokens - 1) / a.kv.page_tokens;
+    if (rp.max_chunks > kMaxChunks) return cudaErrorInvalidValue;
+    rp.counters = attention_counters(a.attn_scratch, a.scratch_rows < 1 ? 1 : a.scratch_rows, a.Hq, a.d, a.max_ctx,
+                                     a.kv.page_tokens);
+    rp.sync = a.sync;
+    rp.rope = rope_freqs(a.theta, a.d);
+    cudaError_t e = cudaMemsetAsync(a.sync, 0, sizeof(unsigned), st);  // barrier counter only
+    if (e != cudaSuccess) return e;
+    const int G = a.Hq / a.Hkv;
+    if (a.d == 128) {
+        switch (G) {
+            case 1: return launch_run_t<1, 128>(rp, st);
+            case 2: return launch_run_t<2, 128>(rp, st);
+            case 4: return launch_run_t<4, 128>(rp, st);
+            case 8: return launch_run_t<8, 128>(rp, st);
+        }
+    } else {
+        switch (G) {
+            case 1: return launch_run_t<1, 64>(rp, st);
+            case 2: return launch_run_t<2, 64>(rp, st);
+            case 4: return launch_run_t<4, 64>(rp, st);
+            case 8: return launch_run_t<8, 64>(rp, st);
         }
     }
     return cudaErrorInvalidValue;

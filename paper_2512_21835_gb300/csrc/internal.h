@@ -63,14 +63,44 @@ size_t lm_head_scratch_bytes(int B, int V);
 // partial state to scratch and the last block of each (row, kv head) combines
 // them into o (max_ctx <= 16384); otherwise one block per (row, kv head) loops
 // over all pages.  o_bf16: write o as bf16 (prefill) instead of fp32.
+// scratch_rows: the batch the scratch was sized for (attention_scratch_floats);
+// the completion counters sit after that many rows of partial states, so the
+// same scratch serves every batch up to it (0 = B).
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
-                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl = false);
+                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl = false,
+                             int scratch_rows = 0);
 size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens);
 // Split attention keeps one int completion counter per (row, head) after the
 // partial states; they must be zero before a launch and every launch leaves
 // them zero.
 int* attention_counters(float* scratch, int B, int Hq, int d, int max_ctx, int page_tokens);
+
+// Persistent layer run (batch 1).  One cooperative launch computes decoder
+// layers layer0 .. layer0 + n_layers - 1 (all resident in device memory) for
+// the single row of x: for each layer, the QKV + RoPE + KV-append tiles, the
+// split attention, the O-projection, the gate/up SwiGLU and the down tiles,
+// separated by grid-wide barriers.  Blocks stay resident for the whole run and
+// prefetch the next phase's first weight tiles into L2 before each barrier.
+// Same arithmetic per output as the batch-1 kernels above.  sync[0] is the
+// barrier counter (zeroed by the launcher on the stream), sync[1] an error word
+// set to 1 when a barrier wait passes its 1 s bound (every block then leaves).
+constexpr int kMaxRunLayers = 128;
+struct DecodeRunArgs {
+    const char* base[kMaxRunLayers];  // device address of each layer's blob
+    int n_layers, layer0;
+    uint64_t off_g_attn, off_wqkv, off_wo, off_g_mlp, off_wg, off_wu, off_wd;  // blob byte offsets
+    int H, Hq, Hkv, d, F;
+    float eps, theta;
+    float *x, *q, *o, *a;            // [H], [Hq d], [Hq d], [F] fp32
+    const int32_t* positions;        // [1]: position of the token
+    KvView kv;                       // layer field ignored
+    float* attn_scratch;             // attention_scratch_floats(scratch_rows, Hq, d, max_ctx, page_tokens)
+    int scratch_rows, max_ctx;
+    unsigned* sync;                  // [2]
+};
+bool decode_run_supported(int Hq, int Hkv, int d);
+cudaError_t launch_decode_run(const DecodeRunArgs& a, cudaStream_t st);
 
 cudaError_t launch_embed(const uint16_t* embed, const int32_t* tokens, int B, int H, int V, float* x,
                          cudaStream_t st, bool pdl = false);

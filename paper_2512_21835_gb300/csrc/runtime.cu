@@ -49,7 +49,7 @@ struct Request {
 
 struct Fixed {  // offsets inside the fixed region
     uint64_t embed, lm_head, g_final, x, q, o, a, z, logits, attn_scratch, lm_scratch;
-    uint64_t tokens, out_tokens, positions, ctx_lens, row_req, page_table, last_rows, dec_pos;
+    uint64_t tokens, out_tokens, positions, ctx_lens, row_req, page_table, last_rows, dec_pos, run_sync;
     uint64_t px, py, pq, po, pa;
     uint64_t total;
 };
@@ -131,6 +131,7 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     f.last_rows = take(B * 4);
     f.dec_pos = take(B * 4);
     f.page_table = take(B * max_pages * 8);
+    f.run_sync = take(16);
     f.px = take(Mp * H * 4);
     f.py = take(Mp * H * 2);
     f.pq = take(Mp * qd * 4);
@@ -168,7 +169,8 @@ struct loip_ctx {
     // host pool: blobs of offloaded layers inside pinned huge-page regions
     std::vector<void*> host_layer;
     std::vector<HostBuf> host_regions;
-    int32_t* h_stage = nullptr;  // pinned staging for small transfers
+    int32_t* h_stage = nullptr;  // pinned staging for small transfers (last word: layer-run error)
+    bool run_launched = false;   // a layer-run kernel has been enqueued (its error word is checked)
     size_t h_stage_ints = 0;
     int64_t* h_pt = nullptr;     // pinned page-table staging
     // streams and events
@@ -239,6 +241,17 @@ struct loip_ctx {
             }
             std::this_thread::yield();
         }
+    }
+
+    // After a host sync point: a layer-run kernel whose grid barrier timed out
+    // left its error word set; the context cannot continue.
+    int check_run_error() {
+        if (!run_launched) return LOIP_OK;
+        if (h_stage[h_stage_ints - 1] != 0) {
+            failed = true;
+            return fail(LOIP_ERR_TIMEOUT, "a grid barrier of the persistent layer-run kernel timed out");
+        }
+        return LOIP_OK;
     }
 
     int sync_all() {
@@ -429,6 +442,14 @@ struct loip_ctx {
     int run_layers_direct(int B, const int32_t* pos_dev, cudaStream_t s) {
         for (int l = 0; l < L; ++l) {
             const bool off = layer_block[l] < 0;
+            if (!off && fuse_runs(B)) {
+                int e = l;
+                while (e < L && layer_block[e] >= 0) ++e;
+                int rc = decode_run(l, e, pos_dev, s);
+                if (rc) return rc;
+                l = e - 1;
+                continue;
+            }
             const uint16_t* w = off ? host_direct(l) : layer_weights(l, -1);
             if (!w) return fail(LOIP_ERR_STATE, "offloaded layer has no device-mapped host copy");
             int rc = decode_layer_w(l, B, pos_dev, s, w, off);
@@ -460,7 +481,7 @@ struct loip_ctx {
         chain = true;
         e = timed(1, s, [&] {
             return launch_attention(q, kv, nullptr, pos_dev, nullptr, B, Hq, Hkv, d, cfg.max_ctx, true,
-                                    fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl());
+                                    fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl(), cfg.max_batch);
         });
         if (e != cudaSuccess) return cuda_fail(e, "attention kernel");
         e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl(), w_host); });
@@ -510,11 +531,69 @@ struct loip_ctx {
         return LOIP_OK;
     }
 
+    // Layers l0 .. l1-1 (resident) of a batch-1 decode step in one persistent
+    // launch.
+    int decode_run(int l0, int l1, const int32_t* pos_dev, cudaStream_t s) {
+        for (int b0 = l0; b0 < l1; b0 += kMaxRunLayers) {
+            const int b1 = std::min(l1, b0 + kMaxRunLayers);
+            DecodeRunArgs a{};
+            for (int l = b0; l < b1; ++l) a.base[l - b0] = reinterpret_cast<const char*>(layer_weights(l, -1));
+            a.n_layers = b1 - b0;
+            a.layer0 = b0;
+            a.off_g_attn = lay.off_g_attn;
+            a.off_wqkv = lay.off_wqkv;
+            a.off_wo = lay.off_wo;
+            a.off_g_mlp = lay.off_g_mlp;
+            a.off_wg = lay.off_wg;
+            a.off_wu = lay.off_wu;
+            a.off_wd = lay.off_wd;
+            a.H = H;
+            a.Hq = Hq;
+            a.Hkv = Hkv;
+            a.d = d;
+            a.F = F;
+            a.eps = desc.rms_eps;
+            a.theta = desc.rope_theta;
+            a.x = fixed_ptr<float>(fx.x);
+            a.q = fixed_ptr<float>(fx.q);
+            a.o = fixed_ptr<float>(fx.o);
+            a.a = fixed_ptr<float>(fx.a);
+            a.positions = pos_dev;
+            a.kv = kv_view(0, fixed_ptr<int64_t>(fx.page_table));
+            a.attn_scratch = fixed_ptr<float>(fx.attn_scratch);
+            a.scratch_rows = cfg.max_batch;
+            a.max_ctx = cfg.max_ctx;
+            a.sync = fixed_ptr<unsigned>(fx.run_sync);
+            chain = false;
+            cudaError_t e = timed(12, s, [&] { return launch_decode_run(a, s); });
+            chain = false;
+            if (e != cudaSuccess) return cuda_fail(e, "layer-run kernel");
+            run_launched = true;
+        }
+        return LOIP_OK;
+    }
+
+    // Whether a batch-B decode step computes its runs of resident layers with
+    // the persistent layer-run kernel.
+    bool fuse_runs(int B) const {
+        return B == 1 && !cfg.per_op_kernels && decode_run_supported(Hq, Hkv, d) && cfg.max_ctx <= 64 * 256;
+    }
+
     // Runs all layers once (decode or prefill pass) with the streaming ring.
+    // run_pos != nullptr: batch-1 decode; runs of resident layers go to the
+    // persistent layer-run kernel.
     template <class LayerFn>
-    int run_layers(LayerFn&& fn) {
+    int run_layers(LayerFn&& fn, const int32_t* run_pos = nullptr) {
         const bool naive = cfg.mode == LOIP_MODE_NAIVE;
         for (int l = 0; l < L; ++l) {
+            if (run_pos && !offloaded[l]) {
+                int e = l;
+                while (e < L && !offloaded[e]) ++e;
+                int rc = decode_run(l, e, run_pos, compute);
+                if (rc) return rc;
+                l = e - 1;
+                continue;
+            }
             int slot = -1;
             if (offloaded[l]) {
                 if (naive) {
@@ -880,6 +959,8 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     e = cudaMemsetAsync(c->arena + c->fx.attn_scratch, 0,
                         attention_scratch_floats(cfg.max_batch, c->Hq, c->d, cfg.max_ctx, cfg.page_tokens) * 4,
                         c->compute);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->arena + c->fx.run_sync, 0, 16, c->compute);
+    c->h_stage[c->h_stage_ints - 1] = 0;
     if (e == cudaSuccess) e = cudaStreamSynchronize(c->compute);
     if (e != cudaSuccess) {
         g_create_error = std::string("CUDA setup failed: ") + cudaGetErrorString(e);
@@ -1081,7 +1162,8 @@ static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int3
     if (c->cfg.mode == LOIP_MODE_DIRECT)
         rc = c->run_layers_direct(B, pos, s);
     else
-        rc = c->run_layers([&](int l, int slot) { return c->decode_layer(l, B, pos, s, slot); });
+        rc = c->run_layers([&](int l, int slot) { return c->decode_layer(l, B, pos, s, slot); },
+                           c->fuse_runs(B) ? pos : nullptr);
     if (rc) return rc;
     e = c->timed(5, s, [&] {
         return launch_lm_head(x, c->fixed_ptr<uint16_t>(c->fx.g_final), c->fixed_ptr<uint16_t>(c->fx.lm_head), B, c->H,
@@ -1092,6 +1174,11 @@ static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int3
     if (e != cudaSuccess) return c->cuda_fail(e, "lm head kernel");
     e = launch_advance(pos, B, s, !c->ktiming);
     if (e != cudaSuccess) return c->cuda_fail(e, "position advance");
+    if (c->run_launched) {  // the layer runs' barrier error word, checked at the next host sync point
+        e = cudaMemcpyAsync(c->h_stage + c->h_stage_ints - 1, c->fixed_ptr<unsigned>(c->fx.run_sync) + 1, 4,
+                            cudaMemcpyDeviceToHost, s);
+        if (e != cudaSuccess) return c->cuda_fail(e, "error word download");
+    }
     cudaEventRecord(c->ev_step1, s);
     c->chain = false;
     for (int b = 0; b < B; ++b) c->reqs[b].len += 1;
@@ -1125,6 +1212,8 @@ extern "C" int loip_decode_step(loip_ctx* c, const int32_t* tokens, int32_t batc
     e = cudaEventRecord(c->ev_done, c->compute);
     if (e != cudaSuccess) return c->cuda_fail(e, "event record");
     rc = c->wait_event(c->ev_done);
+    if (rc) return rc;
+    rc = c->check_run_error();
     if (rc) return rc;
     memcpy(out_tokens, hout, (size_t)batch * 4);
     c->collect_kernel_times();
@@ -1284,6 +1373,7 @@ extern "C" int loip_get_stats(const loip_ctx* c, loip_stats* out) {
 extern "C" int loip_synchronize(loip_ctx* c) {
     if (!c) return LOIP_ERR_INVALID;
     int rc = c->sync_all();
+    if (rc == LOIP_OK) rc = c->check_run_error();
     c->collect_copy_time();
     c->collect_kernel_times();
     return rc;
@@ -1294,7 +1384,7 @@ extern "C" int loip_set_kernel_timing(loip_ctx* c, int32_t enable) {
     int rc = c->sync_all();
     if (rc) return rc;
     c->collect_kernel_times();
-    for (int i = 0; i < 12; ++i) {
+    for (int i = 0; i < 16; ++i) {
         c->st.kernel_ms[i] = 0;
         c->st.kernel_launches[i] = 0;
     }

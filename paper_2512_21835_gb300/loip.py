@@ -34,7 +34,7 @@ class ModelDesc(C.Structure):
 
 class Config(C.Structure):
     _fields_ = [("device_budget_bytes", C.c_uint64), ("n_slots", C.c_int32), ("page_tokens", C.c_int32),
-                ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("use_graphs", C.c_int32), ("mode", C.c_int32),
+                ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("per_op_kernels", C.c_int32), ("mode", C.c_int32),
                 ("timeout_ms", C.c_uint32), ("hbm_Bps", C.c_double), ("link_Bps", C.c_double),
                 ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32)]
 
@@ -55,7 +55,7 @@ class Stats(C.Structure):
                 ("last_step_ms", C.c_double), ("copy_busy_ms", C.c_double), ("compute_ms", C.c_double),
                 ("n_resident", C.c_int32), ("n_offloaded", C.c_int32), ("n_replans", C.c_int32),
                 ("kv_tokens", C.c_uint64), ("kv_bytes", C.c_uint64), ("arena_used", C.c_uint64),
-                ("kernel_ms", C.c_double * 12), ("kernel_launches", C.c_uint64 * 12),
+                ("kernel_ms", C.c_double * 16), ("kernel_launches", C.c_uint64 * 16),
                 ("copy_ms_total", C.c_double), ("copies_total", C.c_uint64),
                 ("pool_min_GBps", C.c_double), ("pool_median_GBps", C.c_double), ("pool_replaced", C.c_uint64)]
 
@@ -150,8 +150,8 @@ def model_desc(m: dict) -> ModelDesc:
 
 def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 2048, mode: int = MODE_OVERLAP,
            timeout_ms: int = 0, hbm_Bps: float = 6.7e12, link_Bps: float = 2.1e11, kv_reserve_bytes: int = 0,
-           max_prefill_tokens: int = 512, page_tokens: int = 64, use_graphs: int = 0) -> Config:
-    return Config(budget, n_slots, page_tokens, max_batch, max_ctx, use_graphs, mode, timeout_ms, hbm_Bps, link_Bps,
+           max_prefill_tokens: int = 512, page_tokens: int = 64, per_op_kernels: int = 0) -> Config:
+    return Config(budget, n_slots, page_tokens, max_batch, max_ctx, per_op_kernels, mode, timeout_ms, hbm_Bps, link_Bps,
                   kv_reserve_bytes, max_prefill_tokens)
 
 

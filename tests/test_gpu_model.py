@@ -188,3 +188,92 @@ def test_direct_access_decode_copies_nothing(torch, L, orc):
     ctx.close()
     assert np.array_equal(np.array(toks), base[0])
     assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
+
+
+def _decode_with_timing(L, torch, m, prompt, cont, cfg_kw, resident_layers):
+    """Prefill then decode with kernel timing on; returns tokens, hidden states and stats."""
+    budget = _budget(L, m, cfg_kw, resident_layers)
+    ctx = L.Context(m, L.config(budget=budget, **cfg_kw))
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    hid = torch.empty(1, m["hidden"], dtype=torch.float32, device="cuda")
+    toks = [ctx.prefill([prompt], out_hidden=hid)]
+    hids = [hid.cpu().numpy().copy()]
+    ctx.set_kernel_timing(True)
+    for step in cont:
+        toks.append(ctx.decode_step(step, out_hidden=hid))
+        hids.append(hid.cpu().numpy().copy())
+    ctx.synchronize()
+    st = ctx.stats()
+    ctx.close()
+    return np.array(toks), np.array(hids), st
+
+
+RUN_CLASS = 12  # kernel-timing class of the persistent layer-run kernel
+
+
+@pytest.mark.parametrize("resident,K,mode", [(6, 2, 0), (3, 2, 0), (1, 1, 0), (2, 2, 2)])
+def test_layer_run_kernel_matches_per_op_kernels(torch, L, orc, resident, K, mode):
+    """Batch-1 decode through the persistent layer-run kernel (runs of resident
+    layers in one launch) equals the per-operation kernels bit for bit: at this
+    shape both use the block-tile GEMV for every projection and the same
+    attention groups."""
+    m = TINY6
+    prompt = inputs.token_ids(61, 70, m["vocab"])
+    cont = [[int(t)] for t in inputs.token_ids(62, 10, m["vocab"])]
+    kw = dict(max_batch=1, max_ctx=128, n_slots=K, mode=mode)
+    fused = _decode_with_timing(L, torch, m, prompt, cont, kw, resident)
+    per_op = _decode_with_timing(L, torch, m, prompt, cont, dict(kw, per_op_kernels=1), resident)
+    assert fused[2]["kernel_launches"][RUN_CLASS] > 0
+    assert per_op[2]["kernel_launches"][RUN_CLASS] == 0
+    assert np.array_equal(fused[0], per_op[0])
+    assert np.array_equal(fused[1].view(np.uint32), per_op[1].view(np.uint32))
+
+
+def test_layer_run_kernel_matches_oracle_llama3_heads(torch, L, orc):
+    """The layer-run kernel at LLaMA-3 head geometry (head_dim 128, 4 query heads
+    per kv head), prompt crossing a KV page boundary, against the oracle."""
+    m = dict(n_layers=3, hidden=512, n_heads=8, n_kv_heads=2, head_dim=128, ffn=1408, vocab=2048,
+             rms_eps=1e-5, rope_theta=500000.0)
+    prompt = inputs.token_ids(81, 78, m["vocab"])
+    P = 70
+    ref = _oracle(orc, m, prompt[:P], prompt[P:])
+    cont = [[int(t)] for t in prompt[P:]]
+    toks, hids, st = _decode_with_timing(L, torch, m, prompt[:P], cont, dict(max_batch=1, max_ctx=128), 3)
+    assert st["kernel_launches"][RUN_CLASS] == len(cont)
+    for i in range(len(toks)):
+        t = P - 1 + i
+        _check_hidden(hids[i][0], ref["hidden"][t])
+        assert int(toks[i][0]) == int(ref["argmax"][t])
+
+
+def test_mixed_batch_sizes_share_attention_scratch(torch, L, orc):
+    """Decode steps at batch 2, then 1, then 2 again on one context: the split
+    attention's completion counters sit at a fixed place in the scratch, so a
+    larger batch's partial states never overwrite a smaller batch's counters."""
+    m = TINY6
+    prompts = [inputs.token_ids(91, 40, m["vocab"]), inputs.token_ids(92, 40, m["vocab"])]
+    kw = dict(max_batch=2, max_ctx=128, n_slots=2)
+    ctx = L.Context(m, L.config(budget=_budget(L, m, kw, 6), **kw))
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    first = ctx.prefill(prompts)
+    hid = torch.empty(2, m["hidden"], dtype=torch.float32, device="cuda")
+    seq0 = list(prompts[0])
+    seq0.append(int(first[0]))
+    feed = [int(first[0]), int(first[1])]
+    hids0 = []
+    for B in (2, 1, 1, 2, 2):
+        out = ctx.decode_step(feed[:B], out_hidden=hid)
+        hids0.append(hid[0].cpu().numpy().copy())
+        feed = [int(out[0]), int(out[1]) if B == 2 else feed[1]]
+        seq0.append(int(out[0]))
+    ctx.close()
+    # request 0 alone, same tokens, batch 1 throughout (its own context)
+    kw1 = dict(max_batch=1, max_ctx=128, n_slots=2)
+    ctx = L.Context(m, L.config(budget=_budget(L, m, kw1, 6), **kw1))
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    ctx.prefill([prompts[0]])
+    h1 = torch.empty(1, m["hidden"], dtype=torch.float32, device="cuda")
+    for i in range(5):
+        ctx.decode_step([seq0[40 + i]], out_hidden=h1)
+        _check_hidden(h1[0].cpu().numpy(), hids0[i])
+    ctx.close()
