@@ -169,7 +169,7 @@ def run_ours(args, rank, world):
     max_prefill = sum(lens) if prefill_mode else min(4096, sum(lens))
     cfg = loip.config(budget=budget, n_slots=w["n_slots"], max_batch=Bsz, max_ctx=max_ctx,
                       max_prefill_tokens=max_prefill, link_Bps=link_peak * 1e9, hbm_Bps=hbm_peak * 1e9,
-                      kv_reserve_bytes=kv_reserve, mode=mode, per_op_kernels=1 if args.per_op_kernels else 0)
+                      kv_reserve_bytes=kv_reserve, mode=mode, layer_run_kernel=1 if args.layer_run_kernel else 0)
     t0 = time.time()
     ctx = loip.Context(m, cfg)
     plan = ctx.plan()
@@ -311,7 +311,7 @@ def run_ours(args, rank, world):
         "config": {"workload": args.workload, "model": w["model"] + "-shaped", "layers": m["n_layers"],
                    "global_batch": Bsz * world, "context": lens if len(set(lens)) > 1 else lens[0],
                    "budget_bytes": budget, "slots": 1 if args.mode == "naive" else w["n_slots"], "mode": args.mode,
-                   "layer_kernels": "per-op" if args.per_op_kernels else "persistent runs at batch 1",
+                   "layer_kernels": "persistent runs at batch 1" if args.layer_run_kernel else "per-op",
                    "resident_layers": st1["n_resident"],
                    "offloaded_layers": n_off, "offloaded_at_start": n_off0,
                    "offloaded_at_end": plan_end["n_offloaded"], "replans": st_end["n_replans"],
@@ -447,8 +447,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--mode", default="overlap", choices=sorted(MODES))
-    ap.add_argument("--per-op-kernels", action="store_true",
-                    help="one launch per operation instead of the persistent layer-run kernel at batch 1")
+    ap.add_argument("--layer-run-kernel", action="store_true",
+                    help="batch 1: compute runs of resident layers with the persistent layer-run kernel")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -66,9 +66,10 @@ typedef struct loip_config {
     int32_t page_tokens;          /* KV page size in tokens (64) */
     int32_t max_batch;            /* largest decode batch (<= 8) */
     int32_t max_ctx;              /* largest context per request, tokens */
-    int32_t per_op_kernels;       /* 0: at batch 1, each run of consecutive resident layers is
-                                   * computed by one persistent kernel (grid barriers between
-                                   * the phases of a layer); 1: one kernel launch per operation */
+    int32_t layer_run_kernel;     /* 0: one kernel launch per operation (default, fastest as
+                                   * measured); 1: at batch 1, each run of consecutive resident
+                                   * layers is computed by one persistent cooperative kernel
+                                   * (grid barriers between the phases of a layer) */
     int32_t mode;                 /* LOIP_MODE_OVERLAP, LOIP_MODE_NAIVE or LOIP_MODE_DIRECT */
     uint32_t timeout_ms;          /* deadline of every host wait (0 = 600000) */
     double hbm_Bps;               /* bandwidths used by the planner's step model */

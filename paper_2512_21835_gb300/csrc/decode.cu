@@ -529,9 +529,9 @@ __device__ __forceinline__ float ld_act(const float* p) {
 // tile's loads (tile_first_load).  When next >= 0, the first batch of tile
 // `next` is issued into wa as soon as this tile's loads are consumed, so its
 // weights stream during this tile's reduction and epilogue.
-template <int EPI, bool CG>
+template <int EPI, bool CG, bool STAGED = false>
 __device__ __forceinline__ void tile_gemv(const GemvParams& p, int tile, int next, uint4 (&wa)[kTileRows],
-                                          TileShared& sm) {
+                                          TileShared& sm, const float* sx = nullptr, float inv_staged = 1.f) {
     constexpr int R = kTileRows;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int K = p.K;
@@ -552,10 +552,10 @@ __device__ __forceinline__ void tile_gemv(const GemvParams& p, int tile, int nex
     auto consume = [&](const uint4 (&w)[R], int j) {
         const int k = j * 256 + lane * 8;
         if (j >= j_end || k >= K) return;
-        const float4 xa = ld_act4<CG>(p.in + k);
-        const float4 xb = ld_act4<CG>(p.in + k + 4);
+        const float4 xa = STAGED ? *reinterpret_cast<const float4*>(sx + k) : ld_act4<CG>(p.in + k);
+        const float4 xb = STAGED ? *reinterpret_cast<const float4*>(sx + k + 4) : ld_act4<CG>(p.in + k + 4);
         float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
-        if (norm) {
+        if (norm && !STAGED) {  // staged inputs already carry the gain
             const uint4 gv = *reinterpret_cast<const uint4*>(p.g + k);
             const float gf[8] = {bf_lo(gv.x), bf_hi(gv.x), bf_lo(gv.y), bf_hi(gv.y),
                                  bf_lo(gv.z), bf_hi(gv.z), bf_lo(gv.w), bf_hi(gv.w)};
@@ -591,7 +591,7 @@ __device__ __forceinline__ void tile_gemv(const GemvParams& p, int tile, int nex
         const float v = warp_sum(acc[r]);
         if (lane == 0) sm.part[warp][r] = v;
     }
-    if (norm) {
+    if (norm && !STAGED) {
         const float v = warp_sum(ss);
         if (lane == 0) sm.ss[warp] = v;
     }
@@ -601,14 +601,14 @@ __device__ __forceinline__ void tile_gemv(const GemvParams& p, int tile, int nex
         for (int w = 0; w < kTileWarps; ++w) t += sm.part[w][tid];
         sm.val[tid] = t;
     }
-    if (tid == 32) {
+    if (!STAGED && tid == 32) {
         float t = 0.f;
         if (norm)
             for (int w = 0; w < kTileWarps; ++w) t += sm.ss[w];
         sm.inv = norm ? 1.0f / sqrtf(t / (float)K + p.eps) : 1.0f;
     }
     __syncthreads();
-    const float inv = sm.inv;
+    const float inv = STAGED ? inv_staged : sm.inv;
     if (EPI == EPI_QKV) {
         if (tid < R / 2) {
             const int half = p.d >> 1;
@@ -1126,7 +1126,8 @@ struct RunParams {
     float* scratch;
     int* counters;
     int max_chunks;
-    unsigned* sync;
+    unsigned* sync;  // [0] barrier counter, [1] error word, [2 ..] tile counters (4 per layer)
+    uint32_t smem_bytes;
     RopeFreqs rope;
 };
 
@@ -1193,19 +1194,81 @@ __device__ __forceinline__ int tile_count(const GemvParams& p) {
                                                  : (p.N + kTileRows - 1) / kTileRows;
 }
 
-// This block's tiles of one phase, the next tile's first loads issued while the
-// current one reduces.
+// Stages the phase's input row in shared memory (times the RMSNorm gain when
+// the phase has one) and returns 1/rms (1 without a gain).  The sum of squares
+// is accumulated in the per-tile path's order (each warp over its K slice, then
+// lanes, then warps in order), so both paths produce the same bits.
+__device__ __forceinline__ float stage_input(const GemvParams& p, float* sx, TileShared& sm) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int K = p.K;
+    const int nj = (K + 255) >> 8, njw = (nj + kTileWarps - 1) / kTileWarps;
+    const int j_begin = warp * njw, j_end = min(nj, j_begin + njw);
+    const bool norm = p.g != nullptr;
+    float ss = 0.f;
+    for (int j = j_begin; j < j_end; ++j) {
+        const int k = j * 256 + lane * 8;
+        if (k >= K) continue;
+        const float4 xa = ld_act4<true>(p.in + k);
+        const float4 xb = ld_act4<true>(p.in + k + 4);
+        float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+        if (norm) {
+            const uint4 gv = *reinterpret_cast<const uint4*>(p.g + k);
+            const float gf[8] = {bf_lo(gv.x), bf_hi(gv.x), bf_lo(gv.y), bf_hi(gv.y),
+                                 bf_lo(gv.z), bf_hi(gv.z), bf_lo(gv.w), bf_hi(gv.w)};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                ss = fmaf(xv[e], xv[e], ss);
+                xv[e] *= gf[e];
+            }
+        }
+        *reinterpret_cast<float4*>(sx + k) = make_float4(xv[0], xv[1], xv[2], xv[3]);
+        *reinterpret_cast<float4*>(sx + k + 4) = make_float4(xv[4], xv[5], xv[6], xv[7]);
+    }
+    if (norm) {
+        const float v = warp_sum(ss);
+        if (lane == 0) sm.ss[warp] = v;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        float t = 0.f;
+        if (norm)
+            for (int w = 0; w < kTileWarps; ++w) t += sm.ss[w];
+        sm.inv = norm ? 1.0f / sqrtf(t / (float)K + p.eps) : 1.0f;
+    }
+    __syncthreads();
+    return sm.inv;
+}
+
+// This block's tiles of one phase.  The first tile is blockIdx.x; later ones
+// are handed out by the phase's counter (first come, first served, so blocks
+// that stream faster take more tiles), each fetched one tile ahead so that the
+// next tile's first loads are issued while the current one reduces.  The input
+// row is staged in shared memory when it fits (sx != nullptr).
 template <int EPI>
-__device__ __forceinline__ void run_tiles(const GemvParams& p, TileShared& tsm) {
+__device__ __forceinline__ void run_tiles(const GemvParams& p, TileShared& tsm, float* sx, unsigned* ctr,
+                                          int* s_next) {
     const int ntiles = tile_count<EPI>(p);
     int t = blockIdx.x;
     if (t >= ntiles) return;
     uint4 wa[kTileRows];
     tile_first_load<EPI>(p, t, wa);
+    if (threadIdx.x == 0) *s_next = (int)(gridDim.x + atomicAdd(ctr, 1u));
+    const float inv = sx ? stage_input(p, sx, tsm) : 1.f;
+    __syncthreads();
+    int nxt = *s_next;
     while (t < ntiles) {
-        const int nxt = t + gridDim.x;
-        tile_gemv<EPI, true>(p, t, nxt < ntiles ? nxt : -1, wa, tsm);
+        unsigned grabbed = 0;
+        const bool more = nxt < ntiles;
+        if (threadIdx.x == 0 && more) grabbed = gridDim.x + atomicAdd(ctr, 1u);
+        if (sx)
+            tile_gemv<EPI, true, true>(p, t, more ? nxt : -1, wa, tsm, sx, inv);
+        else
+            tile_gemv<EPI, true, false>(p, t, more ? nxt : -1, wa, tsm);
+        if (threadIdx.x == 0) *s_next = more ? (int)grabbed : ntiles;
+        __syncthreads();
         t = nxt;
+        nxt = *s_next;
+        __syncthreads();  // every thread has read s_next before it is rewritten
     }
 }
 
@@ -1214,11 +1277,13 @@ enum { PH_QKV = 0, PH_O = 1, PH_GU = 2, PH_D = 3 };
 template <int G, int D>
 __global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParams rp) {
     extern __shared__ __align__(16) unsigned char run_smem[];
-    AttnSmem<G, D>* asm2 = reinterpret_cast<AttnSmem<G, D>*>(run_smem);  // one per attention group
+    // attention: one AttnSmem per group; GEMV phases: the staged input row
+    AttnSmem<G, D>* asm2 = reinterpret_cast<AttnSmem<G, D>*>(run_smem);
+    float* sx_buf = reinterpret_cast<float*>(run_smem);
     __shared__ GemvParams s_gp[4];
     __shared__ AttnParams s_ap;
     __shared__ TileShared tsm;
-    __shared__ int s_flag;
+    __shared__ int s_flag, s_next;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int qd = rp.Hq * rp.d, nqkv = (rp.Hq + 2 * rp.Hkv) * rp.d;
     // weight pointers of phase `ph` for layer `li` of the run
@@ -1298,9 +1363,12 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParam
     const int npages = (ctx + rp.kv.page_tokens - 1) / rp.kv.page_tokens;
     const int items = rp.Hkv * npages;
     unsigned nsync = 0;
+    // the staged input row of a phase must fit the dynamic shared memory
+    auto sx_for = [&](int K) { return (size_t)K * 4 <= rp.smem_bytes ? sx_buf : nullptr; };
+    unsigned* ctr = rp.sync + 2;  // tile counters, 4 per layer, zeroed by the launcher
     for (int li = 0; li < rp.n_layers; ++li) {
         // ---- RMSNorm + QKV + RoPE + KV append
-        run_tiles<EPI_QKV>(s_gp[PH_QKV], tsm);
+        run_tiles<EPI_QKV>(s_gp[PH_QKV], tsm, sx_for(rp.H), ctr + 4 * li + PH_QKV, &s_next);
         if (tid == 0) {
             s_ap.kv.layer = rp.layer0 + li;
             if (li + 1 < rp.n_layers) set_layer(PH_QKV, li + 1);
@@ -1313,28 +1381,35 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParam
             for (int i = blockIdx.x + grp * gridDim.x; i < items; i += 2 * gridDim.x)
                 attn_group<G, D, true>(s_ap, 0, i / npages, i % npages, asm2[grp], tid & 63, 1 + grp);
         } else {
+            // HBM is otherwise idle here: pull the O-projection tiles, then the
+            // first gate/up tiles, into L2 (tiles blockIdx + k * grid; at most
+            // 40 MB of each over the grid).  Whichever block later takes a tile
+            // finds it in L2.
+            const int k0 = warp - 4;
             const GemvParams& o = s_gp[PH_O];
-            const int nt = tile_count<EPI_RESID>(o);
-            const int k = warp - 4;  // tiles blockIdx + k * grid, at most 48 MB over the grid
-            const uint64_t tile_bytes = (uint64_t)kTileRows * o.K * 2;
-            const uint64_t kfit = (48ull << 20) / (tile_bytes * gridDim.x);
-            const int kmax = kfit < 1 ? 1 : (int)kfit;
-            for (int kk = k; kk < kmax && blockIdx.x + kk * gridDim.x < nt; kk += 4)
+            const GemvParams& gu = s_gp[PH_GU];
+            const int nto = tile_count<EPI_RESID>(o), ntg = tile_count<EPI_SWIGLU>(gu);
+            const uint64_t cap = 40ull << 20;
+            const uint64_t ko = cap / ((uint64_t)kTileRows * o.K * 2 * gridDim.x);
+            const uint64_t kg = cap / ((uint64_t)kTileRows * gu.K * 2 * gridDim.x);
+            for (int kk = k0; kk < (int)(ko < 1 ? 1 : ko) && blockIdx.x + kk * gridDim.x < nto; kk += 4)
                 prefetch_tile<EPI_RESID>(o, blockIdx.x + kk * gridDim.x, lane);
+            for (int kk = k0; kk < (int)kg && blockIdx.x + kk * gridDim.x < ntg; kk += 4)
+                prefetch_tile<EPI_SWIGLU>(gu, blockIdx.x + kk * gridDim.x, lane);
         }
         if (!grid_sync(rp.sync, nsync, &s_flag)) return;
         // ---- O-projection + residual
-        run_tiles<EPI_RESID>(s_gp[PH_O], tsm);
+        run_tiles<EPI_RESID>(s_gp[PH_O], tsm, sx_for(qd), ctr + 4 * li + PH_O, &s_next);
         if (warp == 0) prefetch_tile<EPI_SWIGLU>(s_gp[PH_GU], blockIdx.x, lane);
         if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_O, li + 1);
         if (!grid_sync(rp.sync, nsync, &s_flag)) return;
         // ---- RMSNorm + gate/up SwiGLU
-        run_tiles<EPI_SWIGLU>(s_gp[PH_GU], tsm);
+        run_tiles<EPI_SWIGLU>(s_gp[PH_GU], tsm, sx_for(rp.H), ctr + 4 * li + PH_GU, &s_next);
         if (warp == 0) prefetch_tile<EPI_RESID>(s_gp[PH_D], blockIdx.x, lane);
         if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_GU, li + 1);
         if (!grid_sync(rp.sync, nsync, &s_flag)) return;
         // ---- down + residual
-        run_tiles<EPI_RESID>(s_gp[PH_D], tsm);
+        run_tiles<EPI_RESID>(s_gp[PH_D], tsm, sx_for(rp.F), ctr + 4 * li + PH_D, &s_next);
         if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_D, li + 1);
         __syncthreads();
         if (warp == 0 && li + 1 < rp.n_layers) prefetch_tile<EPI_QKV>(s_gp[PH_QKV], blockIdx.x, lane);
@@ -1342,12 +1417,24 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParam
     }
 }
 
+// Dynamic shared memory of the layer-run kernel: the two attention groups'
+// buffers, or the largest staged input row up to 96 KB (two blocks per SM).
 template <int G, int D>
-cudaError_t launch_run_t(const RunParams& rp, cudaStream_t st) {
-    const size_t smem = 2 * sizeof(AttnSmem<G, D>);
-    static bool attr = false;
+size_t run_smem_bytes(int H, int qd, int F) {
+    size_t need = 2 * sizeof(AttnSmem<G, D>);
+    const int kmax = H > qd ? (H > F ? H : F) : (qd > F ? qd : F);
+    const size_t row = (size_t)kmax * 4;
+    if (row <= (96u << 10) && row > need) need = row;
+    return need;
+}
+
+template <int G, int D>
+cudaError_t launch_run_t(RunParams& rp, cudaStream_t st) {
+    const size_t smem = run_smem_bytes<G, D>(rp.H, rp.Hq * rp.d, rp.F);
+    rp.smem_bytes = (uint32_t)smem;
+    static size_t attr_smem = 0;
     static int grid = 0;
-    if (!attr) {
+    if (attr_smem != smem) {  // per dynamic shared memory size: set the limit, size the grid from occupancy
         cudaError_t e = cudaFuncSetAttribute(decode_run_kernel<G, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)smem);
         if (e != cudaSuccess) return e;
@@ -1358,7 +1445,7 @@ cudaError_t launch_run_t(const RunParams& rp, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
         grid = sms * (per_sm < 2 ? per_sm : 2);
-        attr = true;
+        attr_smem = smem;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -1638,7 +1725,9 @@ cudaError_t launch_decode_run(const DecodeRunArgs& a, cudaStream_t st) {
                                      a.kv.page_tokens);
     rp.sync = a.sync;
     rp.rope = rope_freqs(a.theta, a.d);
-    cudaError_t e = cudaMemsetAsync(a.sync, 0, sizeof(unsigned), st);  // barrier counter only
+    // the barrier counter and the tile counters; the error word (sync[1]) is kept
+    cudaError_t e = cudaMemsetAsync(a.sync, 0, sizeof(unsigned), st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(a.sync + 2, 0, sizeof(unsigned) * 4 * a.n_layers, st);
     if (e != cudaSuccess) return e;
     const int G = a.Hq / a.Hkv;
     if (a.d == 128) {

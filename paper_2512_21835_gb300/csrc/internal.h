@@ -80,11 +80,13 @@ int* attention_counters(float* scratch, int B, int Hq, int d, int max_ctx, int p
 // layers layer0 .. layer0 + n_layers - 1 (all resident in device memory) for
 // the single row of x: for each layer, the QKV + RoPE + KV-append tiles, the
 // split attention, the O-projection, the gate/up SwiGLU and the down tiles,
-// separated by grid-wide barriers.  Blocks stay resident for the whole run and
-// prefetch the next phase's first weight tiles into L2 before each barrier.
-// Same arithmetic per output as the batch-1 kernels above.  sync[0] is the
-// barrier counter (zeroed by the launcher on the stream), sync[1] an error word
-// set to 1 when a barrier wait passes its 1 s bound (every block then leaves).
+// separated by grid-wide barriers.  Blocks stay resident for the whole run,
+// stage each phase's input row in shared memory, take tiles from per-phase
+// counters and prefetch the next phase's first weight tiles into L2 before each
+// barrier.  Same arithmetic per output as the batch-1 kernels above.  sync[0]
+// is the barrier counter and sync[2 ..] the tile counters (zeroed by the
+// launcher on the stream); sync[1] is an error word set to 1 when a barrier
+// wait passes its 1 s bound (every block then leaves).
 constexpr int kMaxRunLayers = 128;
 struct DecodeRunArgs {
     const char* base[kMaxRunLayers];  // device address of each layer's blob
@@ -97,7 +99,7 @@ struct DecodeRunArgs {
     KvView kv;                       // layer field ignored
     float* attn_scratch;             // attention_scratch_floats(scratch_rows, Hq, d, max_ctx, page_tokens)
     int scratch_rows, max_ctx;
-    unsigned* sync;                  // [2]
+    unsigned* sync;                  // [2 + 4 * kMaxRunLayers]: barrier, error word, tile counters
 };
 bool decode_run_supported(int Hq, int Hkv, int d);
 cudaError_t launch_decode_run(const DecodeRunArgs& a, cudaStream_t st);

@@ -131,7 +131,7 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     f.last_rows = take(B * 4);
     f.dec_pos = take(B * 4);
     f.page_table = take(B * max_pages * 8);
-    f.run_sync = take(16);
+    f.run_sync = take(4 * (2 + 4 * kMaxRunLayers));
     f.px = take(Mp * H * 4);
     f.py = take(Mp * H * 2);
     f.pq = take(Mp * qd * 4);
@@ -576,7 +576,7 @@ struct loip_ctx {
     // Whether a batch-B decode step computes its runs of resident layers with
     // the persistent layer-run kernel.
     bool fuse_runs(int B) const {
-        return B == 1 && !cfg.per_op_kernels && decode_run_supported(Hq, Hkv, d) && cfg.max_ctx <= 64 * 256;
+        return B == 1 && cfg.layer_run_kernel && decode_run_supported(Hq, Hkv, d) && cfg.max_ctx <= 64 * 256;
     }
 
     // Runs all layers once (decode or prefill pass) with the streaming ring.
@@ -959,7 +959,7 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     e = cudaMemsetAsync(c->arena + c->fx.attn_scratch, 0,
                         attention_scratch_floats(cfg.max_batch, c->Hq, c->d, cfg.max_ctx, cfg.page_tokens) * 4,
                         c->compute);
-    if (e == cudaSuccess) e = cudaMemsetAsync(c->arena + c->fx.run_sync, 0, 16, c->compute);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->arena + c->fx.run_sync, 0, 4 * (2 + 4 * kMaxRunLayers), c->compute);
     c->h_stage[c->h_stage_ints - 1] = 0;
     if (e == cudaSuccess) e = cudaStreamSynchronize(c->compute);
     if (e != cudaSuccess) {

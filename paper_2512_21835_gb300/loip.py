@@ -34,7 +34,7 @@ class ModelDesc(C.Structure):
 
 class Config(C.Structure):
     _fields_ = [("device_budget_bytes", C.c_uint64), ("n_slots", C.c_int32), ("page_tokens", C.c_int32),
-                ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("per_op_kernels", C.c_int32), ("mode", C.c_int32),
+                ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("layer_run_kernel", C.c_int32), ("mode", C.c_int32),
                 ("timeout_ms", C.c_uint32), ("hbm_Bps", C.c_double), ("link_Bps", C.c_double),
                 ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32)]
 
@@ -150,8 +150,9 @@ def model_desc(m: dict) -> ModelDesc:
 
 def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 2048, mode: int = MODE_OVERLAP,
            timeout_ms: int = 0, hbm_Bps: float = 6.7e12, link_Bps: float = 2.1e11, kv_reserve_bytes: int = 0,
-           max_prefill_tokens: int = 512, page_tokens: int = 64, per_op_kernels: int = 0) -> Config:
-    return Config(budget, n_slots, page_tokens, max_batch, max_ctx, per_op_kernels, mode, timeout_ms, hbm_Bps, link_Bps,
+           max_prefill_tokens: int = 512, page_tokens: int = 64, layer_run_kernel: int = 0) -> Config:
+    return Config(budget, n_slots, page_tokens, max_batch, max_ctx, layer_run_kernel, mode, timeout_ms, hbm_Bps,
+                  link_Bps,
                   kv_reserve_bytes, max_prefill_tokens)
 
 

@@ -221,8 +221,8 @@ def test_layer_run_kernel_matches_per_op_kernels(torch, L, orc, resident, K, mod
     prompt = inputs.token_ids(61, 70, m["vocab"])
     cont = [[int(t)] for t in inputs.token_ids(62, 10, m["vocab"])]
     kw = dict(max_batch=1, max_ctx=128, n_slots=K, mode=mode)
-    fused = _decode_with_timing(L, torch, m, prompt, cont, kw, resident)
-    per_op = _decode_with_timing(L, torch, m, prompt, cont, dict(kw, per_op_kernels=1), resident)
+    fused = _decode_with_timing(L, torch, m, prompt, cont, dict(kw, layer_run_kernel=1), resident)
+    per_op = _decode_with_timing(L, torch, m, prompt, cont, kw, resident)
     assert fused[2]["kernel_launches"][RUN_CLASS] > 0
     assert per_op[2]["kernel_launches"][RUN_CLASS] == 0
     assert np.array_equal(fused[0], per_op[0])
@@ -238,7 +238,8 @@ def test_layer_run_kernel_matches_oracle_llama3_heads(torch, L, orc):
     P = 70
     ref = _oracle(orc, m, prompt[:P], prompt[P:])
     cont = [[int(t)] for t in prompt[P:]]
-    toks, hids, st = _decode_with_timing(L, torch, m, prompt[:P], cont, dict(max_batch=1, max_ctx=128), 3)
+    toks, hids, st = _decode_with_timing(L, torch, m, prompt[:P], cont,
+                                         dict(max_batch=1, max_ctx=128, layer_run_kernel=1), 3)
     assert st["kernel_launches"][RUN_CLASS] == len(cont)
     for i in range(len(toks)):
         t = P - 1 + i
@@ -252,7 +253,7 @@ def test_mixed_batch_sizes_share_attention_scratch(torch, L, orc):
     larger batch's partial states never overwrite a smaller batch's counters."""
     m = TINY6
     prompts = [inputs.token_ids(91, 40, m["vocab"]), inputs.token_ids(92, 40, m["vocab"])]
-    kw = dict(max_batch=2, max_ctx=128, n_slots=2)
+    kw = dict(max_batch=2, max_ctx=128, n_slots=2, layer_run_kernel=1)
     ctx = L.Context(m, L.config(budget=_budget(L, m, kw, 6), **kw))
     ctx.load_weights_generated(configs.WEIGHT_SEED)
     first = ctx.prefill(prompts)
