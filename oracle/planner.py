@@ -157,3 +157,43 @@ def step_lower_bound(comp, load, offloaded):
     """max(compute, copy) -- no schedule can beat it."""
     return max(sum(comp), sum(c for c, o in zip(load, offloaded) if o))
 
+
+
+def refine_blocks(left: int, offloaded, mha_bytes: int, mlp_bytes: int):
+    """Fine-grained refinement of Algorithm 1 (its block-level conversion loop)
+    for one device: while the memory left after the plan can hold a block of an
+    offloaded layer, one offloaded layer is converted to block-level offloading,
+    the MLP block kept resident when it fits (the layer then streams only its MHA
+    block), else the MHA block.  Layers are converted in layer order.  Returns
+    the per-layer resident-block masks (bit 0: MHA block resident, bit 1: MLP
+    block resident; 3 = whole layer resident) and the memory still left."""
+    masks = [0 if o else 3 for o in offloaded]
+    for l in range(len(masks)):
+        if masks[l] != 0:
+            continue
+        if left >= mlp_bytes:
+            masks[l] = 2
+            left -= mlp_bytes
+        elif left >= mha_bytes:
+            masks[l] = 1
+            left -= mha_bytes
+        else:
+            break
+    return masks, left
+
+
+def eq7_choice(need: int, n_mha: int, n_mlp: int, mha_bytes: int, mlp_bytes: int):
+    """Eq. 7 on one device: the numbers (alpha, beta) of resident MHA and MLP
+    blocks to offload whose memory covers `need` bytes with the fewest bytes
+    offloaded (each offloaded byte is streamed once per step); on equal bytes,
+    fewer blocks.  None when even every available block does not cover it."""
+    best = None
+    for a in range(n_mha + 1):
+        rest = need - a * mha_bytes
+        b = 0 if rest <= 0 else -(-rest // mlp_bytes)
+        if b > n_mlp:
+            continue
+        key = (a * mha_bytes + b * mlp_bytes, a + b)
+        if best is None or key < best[0]:
+            best = (key, (a, b))
+    return None if best is None else best[1]

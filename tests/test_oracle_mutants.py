@@ -109,6 +109,10 @@ PLANNER_MUTANTS = {
     "demotion takes the upper middle": ("victim = (best_start + (best_len - 1) // 2) % L",
                                         "victim = (best_start + best_len // 2) % L"),
     "demotion takes the shortest run": ("if run > best_len:", "if best_len < 0 or run < best_len:"),
+    "refinement keeps the MHA block first": ("        if left >= mlp_bytes:\n            masks[l] = 2\n            left -= mlp_bytes\n        elif left >= mha_bytes:\n            masks[l] = 1\n            left -= mha_bytes",
+                                             "        if left >= mha_bytes:\n            masks[l] = 1\n            left -= mha_bytes\n        elif left >= mlp_bytes:\n            masks[l] = 2\n            left -= mlp_bytes"),
+    "eq7 minimises the block count": ("key = (a * mha_bytes + b * mlp_bytes, a + b)", "key = (a + b, a * mha_bytes + b * mlp_bytes)"),
+    "eq7 rounds the MLP count down": ("b = 0 if rest <= 0 else -(-rest // mlp_bytes)", "b = 0 if rest <= 0 else rest // mlp_bytes"),
 }
 
 

@@ -122,3 +122,55 @@ def test_demote_one_minimises_longest_resident_run_brute_force():
         assert all(new[i] == mask[i] for i in range(L) if i != v)
         best = min(_max_resident_run(mask[:i] + [True] + mask[i + 1:]) for i in range(L) if not mask[i])
         assert _max_resident_run(new) == best
+
+
+def test_refine_blocks_hand_cases():
+    A, M = 30, 140  # MHA and MLP block bytes of a 170-byte layer (p_A ~ 0.18)
+    off = [False, True, False, True, True]
+    # 150 left: layer 1 keeps its MLP block (140), 10 left -> nothing more
+    assert P.refine_blocks(150, off, A, M) == ([3, 2, 3, 0, 0], 10)
+    # 100 left: no MLP block fits; MHA blocks of layers 1, 3, 4 (90), 10 left
+    assert P.refine_blocks(100, off, A, M) == ([3, 1, 3, 1, 1], 10)
+    # 200 left: MLP of layer 1, then MHA of layers 3 and 4 (140 + 30 + 30 = 200)
+    assert P.refine_blocks(200, off, A, M) == ([3, 2, 3, 1, 1], 0)
+    # nothing offloaded or nothing left: unchanged
+    assert P.refine_blocks(500, [False] * 3, A, M) == ([3, 3, 3], 500)
+    assert P.refine_blocks(29, off, A, M) == ([3, 0, 3, 0, 0], 29)
+
+
+def test_refine_blocks_never_exceeds_memory_and_streams_less():
+    import random
+    rng = random.Random(3)
+    for _ in range(200):
+        L = rng.randint(1, 12)
+        off = [rng.random() < 0.5 for _ in range(L)]
+        A, M = rng.randint(1, 50), rng.randint(1, 200)
+        left0 = rng.randint(0, 600)
+        masks, left = P.refine_blocks(left0, off, A, M)
+        kept = sum((A if m & 1 else 0) + (M if m & 2 else 0) for m, o in zip(masks, off) if o)
+        assert left == left0 - kept >= 0
+        assert all(m == 3 for m, o in zip(masks, off) if not o)
+        # a layer left fully offloaded means no block fits any more
+        if any(m == 0 and o for m, o in zip(masks, off)):
+            assert left < min(A, M)
+
+
+def test_eq7_choice_brute_force():
+    import random
+    rng = random.Random(4)
+    assert P.eq7_choice(10, 3, 2, 30, 140) == (1, 0)   # one MHA block covers it
+    assert P.eq7_choice(100, 3, 2, 30, 140) == (0, 1)  # 140 beats 4 x 30 (not available) and 3 x 30 + 1 x 140
+    assert P.eq7_choice(80, 3, 2, 30, 140) == (3, 0)   # 90 < 140
+    assert P.eq7_choice(0, 3, 2, 30, 140) == (0, 0)
+    assert P.eq7_choice(10 ** 6, 3, 2, 30, 140) is None
+    for _ in range(300):
+        A, M = rng.randint(1, 60), rng.randint(1, 300)
+        na, nm = rng.randint(0, 6), rng.randint(0, 4)
+        need = rng.randint(0, na * A + nm * M + 50)
+        got = P.eq7_choice(need, na, nm, A, M)
+        cands = [(a * A + b * M, a + b, (a, b)) for a in range(na + 1) for b in range(nm + 1) if a * A + b * M >= need]
+        if not cands:
+            assert got is None
+        else:
+            best = min(cands)
+            assert got is not None and (got[0] * A + got[1] * M, sum(got)) == best[:2]
