@@ -203,6 +203,7 @@ def run_ours(args, rank, world):
         st = ctx.stats()
         ctx.set_kernel_timing(False)
         st_end = ctx.stats()
+        plan["stream_bytes"] = ctx.block_plan()["stream_bytes"]
         ctx.close()
         return report_prefill(args, w, m, lay, plan, lens, dev_s, e2e_s, st, st_end, clk, hbm_peak, tc_peak,
                               peak_kind, link_peak, world, budget, t_load, t_prefill)
@@ -255,6 +256,7 @@ def run_ours(args, rank, world):
     e2e_s = time.perf_counter() - t0
     st_end = ctx.stats()
     plan_end = ctx.plan()
+    masks = ctx.block_plan()["masks"]
     ctx.close()
     link_after = link_peak_gbs(torch)  # contention on the shared host link shows here too
 
@@ -264,7 +266,9 @@ def run_ours(args, rank, world):
     tokens = steps * Bsz * world
     n_off = st1["n_offloaded"]
     step_s = dev_s / steps
-    link_bytes = n_off * lay["l_size"]
+    # bytes the slot ring copied per timed step (blocks, not whole layers, under
+    # block-level residency; re-plans during the run included)
+    link_bytes = int((st1["h2d_weight_bytes"] - st0["h2d_weight_bytes"]) / steps) or n_off * lay["l_size"]
     mean_ctx = float(np.mean(lens)) + warm + steps / 2
     kv_layer_token = 2 * m["n_kv_heads"] * m["head_dim"] * 2  # K and V bytes per token and layer
     kv_bytes = int(mean_ctx * kv_layer_token * m["n_layers"] * Bsz)
@@ -315,6 +319,8 @@ def run_ours(args, rank, world):
                    "resident_layers": st1["n_resident"],
                    "offloaded_layers": n_off, "offloaded_at_start": n_off0,
                    "offloaded_at_end": plan_end["n_offloaded"], "replans": st_end["n_replans"],
+                   "blocks_at_end": {"whole_resident": int((masks == 3).sum()), "mha_streamed": int((masks == 2).sum()),
+                                     "mlp_streamed": int((masks == 1).sum()), "whole_streamed": int((masks == 0).sum())},
                    "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2: every step reads all weights (> 10 GB)"},
         "roofline": {"bound": "hbm", "kernel": dom_name, "achieved": round(dom_gbs, 1),
@@ -365,7 +371,7 @@ def report_prefill(args, w, m, lay, plan, lens, dev_s, e2e_s, st, st_end, clk, h
     gu_tflops = 2 * M * 2 * F * H / (gu_ms / 1e3) / 1e12
     step_s = dev_s / steps
     n_off = plan["n_offloaded"]
-    link_bytes = n_off * lay["l_size"]
+    link_bytes = plan["stream_bytes"]  # the streamed blocks of one pass over the layers
     roof = max(flops_layer * L / (tc_peak * 1e12), link_bytes / (link_peak * 1e9))
     return {
         "metric": "prefill tokens/s, 70B-shaped bf16 w/ offload (tensor cores)",

@@ -76,6 +76,11 @@ typedef struct loip_config {
     double link_Bps;
     uint64_t kv_reserve_bytes;    /* KV bytes to reserve at create (0 = max_batch*max_ctx) */
     int32_t max_prefill_tokens;   /* tokens per prefill pass (workspace size; 0 = 512) */
+    int32_t whole_layers;         /* 0: block granularity (Sec. III-D/E): memory left after the
+                                   * whole-layer plan keeps MHA/MLP blocks of offloaded layers
+                                   * resident (loip_refine_blocks), and KV growth offloads single
+                                   * blocks chosen by Eq. 7 (loip_eq7_choice); 1: whole layers
+                                   * only (one more layer offloaded per threshold) */
 } loip_config;
 
 typedef struct loip_layer_layout_t {
@@ -146,6 +151,26 @@ int loip_plan_residency(const loip_model_desc* desc, const uint64_t* layer_bytes
  * the number of KV tokens the memory left after a plan can still hold. */
 int loip_kv_threshold(uint64_t left_bytes, uint64_t kv_bytes_per_token, uint64_t* out_tokens);
 
+/* Algorithm 1's fine-grained step (Sec. III-D) on one device: a decoder layer
+ * is an MHA block (g_attn, Wqkv, Wo: loip_layer_layout's mha_bytes) and an MLP
+ * block (g_mlp, Wg, Wu, Wd: mlp_bytes).  While `left_bytes` (device memory left
+ * after the whole-layer plan) can hold a block of a still fully offloaded
+ * layer, that layer (in layer order) keeps its MLP block resident if it fits,
+ * else its MHA block.  offloaded[l] != 0 marks the plan's offloaded layers
+ * (n_layers bytes); masks[l] (n_layers bytes, caller-owned) receives the
+ * resident blocks: bit 0 MHA, bit 1 MLP (3 = whole layer).  *left_out = memory
+ * still left.  Host only. */
+int loip_refine_blocks(const loip_model_desc* desc, uint64_t left_bytes, const uint8_t* offloaded, uint8_t* masks,
+                       uint64_t* left_out);
+
+/* Eq. 7 (online memory-aware planner, Sec. III-E) on one device: the numbers
+ * of resident MHA blocks (*alpha <= n_mha) and MLP blocks (*beta <= n_mlp) to
+ * offload so that their memory covers need_bytes, with the fewest bytes
+ * offloaded (each is streamed once per step afterwards), then the fewest
+ * blocks.  LOIP_ERR_INFEASIBLE when all of them together do not cover it. */
+int loip_eq7_choice(const loip_model_desc* desc, uint64_t need_bytes, int32_t n_mha, int32_t n_mlp, int32_t* alpha,
+                    int32_t* beta);
+
 /* Bytes of the fixed device part of a context (embedding, LM head, final
  * gain, page table, workspaces) for `desc` and `cfg`. */
 int loip_fixed_bytes(const loip_model_desc* desc, const loip_config* cfg, uint64_t* out);
@@ -184,6 +209,12 @@ int loip_load_globals(loip_ctx* ctx, const uint16_t* embed, const uint16_t* lm_h
 
 /* Current plan (resident[] must hold n_layers bytes). */
 int loip_get_plan(const loip_ctx* ctx, loip_plan* out);
+
+/* The context's block-level residency: masks[l] (n_layers bytes, caller-owned)
+ * = resident blocks of layer l (bit 0 MHA, bit 1 MLP; 3 = whole layer, 0 =
+ * fully streamed); *stream_bytes_per_step = bytes the slot ring copies per
+ * pass over the layers (every non-resident block once). */
+int loip_get_block_plan(const loip_ctx* ctx, uint8_t* masks, uint64_t* stream_bytes_per_step);
 
 /* Enqueues the copy of offloaded `layer` from the pinned host pool into device
  * slot `slot` on `copy_stream` (the "stream layer" step, Sec. III-C: the slot

@@ -12,7 +12,11 @@
 //     discrete-event model of the copy and compute streams with K slots;
 //   * online threshold (Eq. 6): tokens the memory left after the plan holds;
 //     past it one more layer is demoted (the resident layer in the middle of
-//     the longest run of resident layers).
+//     the longest run of resident layers);
+//   * block granularity (Algorithm 1's fine-grained step and Eq. 7): a layer is
+//     an MHA block and an MLP block; memory left after the fill keeps blocks of
+//     offloaded layers resident, and online growth offloads the combination of
+//     resident blocks that covers the shortfall with the fewest bytes.
 #include <stdint.h>
 #include <string.h>
 
@@ -121,9 +125,72 @@ int demote_one(int L, uint8_t* off) {
     return victim;
 }
 
+uint64_t refine_blocks(uint64_t left, int L, const uint8_t* offloaded, uint64_t mha_bytes, uint64_t mlp_bytes,
+                       uint8_t* masks) {
+    for (int l = 0; l < L; ++l) masks[l] = offloaded[l] ? 0 : 3;
+    for (int l = 0; l < L; ++l) {
+        if (masks[l] != 0) continue;
+        if (left >= mlp_bytes) {  // keep the MLP block; the layer streams its MHA block only
+            masks[l] = 2;
+            left -= mlp_bytes;
+        } else if (left >= mha_bytes) {  // keep the MHA block; the MLP block streams
+            masks[l] = 1;
+            left -= mha_bytes;
+        } else {
+            break;
+        }
+    }
+    return left;
+}
+
+bool eq7_choice(uint64_t need, int n_mha, int n_mlp, uint64_t mha_bytes, uint64_t mlp_bytes, int* alpha, int* beta) {
+    bool found = false;
+    uint64_t best_bytes = 0;
+    int best_blocks = 0;
+    for (int a = 0; a <= n_mha; ++a) {
+        const uint64_t covered = (uint64_t)a * mha_bytes;
+        const uint64_t rest = need > covered ? need - covered : 0;
+        const uint64_t b = rest == 0 ? 0 : (rest + mlp_bytes - 1) / mlp_bytes;
+        if (b > (uint64_t)n_mlp) continue;
+        const uint64_t bytes = covered + b * mlp_bytes;
+        const int blocks = a + (int)b;
+        if (!found || bytes < best_bytes || (bytes == best_bytes && blocks < best_blocks)) {
+            found = true;
+            best_bytes = bytes;
+            best_blocks = blocks;
+            *alpha = a;
+            *beta = (int)b;
+        }
+    }
+    return found;
+}
+
 }  // namespace loip
 
 using namespace loip;
+
+extern "C" int loip_refine_blocks(const loip_model_desc* desc, uint64_t left_bytes, const uint8_t* offloaded,
+                                  uint8_t* masks, uint64_t* left_out) {
+    if (!desc || !offloaded || !masks || !left_out || desc->n_layers <= 0) return LOIP_ERR_INVALID;
+    loip_layer_layout_t lay;
+    int rc = loip_layer_layout(desc, &lay);
+    if (rc) return rc;
+    *left_out = refine_blocks(left_bytes, desc->n_layers, offloaded, lay.mha_bytes, lay.mlp_bytes, masks);
+    return LOIP_OK;
+}
+
+extern "C" int loip_eq7_choice(const loip_model_desc* desc, uint64_t need_bytes, int32_t n_mha, int32_t n_mlp,
+                               int32_t* alpha, int32_t* beta) {
+    if (!desc || !alpha || !beta || n_mha < 0 || n_mlp < 0) return LOIP_ERR_INVALID;
+    loip_layer_layout_t lay;
+    int rc = loip_layer_layout(desc, &lay);
+    if (rc) return rc;
+    int a = 0, b = 0;
+    if (!eq7_choice(need_bytes, n_mha, n_mlp, lay.mha_bytes, lay.mlp_bytes, &a, &b)) return LOIP_ERR_INFEASIBLE;
+    *alpha = a;
+    *beta = b;
+    return LOIP_OK;
+}
 
 extern "C" int loip_plan_residency(const loip_model_desc* desc, const uint64_t* layer_bytes, uint64_t device_budget,
                                    uint64_t kv_bytes, uint64_t fixed_bytes, int32_t n_slots, double hbm_Bps,

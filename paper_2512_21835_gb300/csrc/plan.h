@@ -15,4 +15,11 @@ double simulate_step(const std::vector<double>& comp, const std::vector<double>&
                      int n_steps);
 // marks one more layer offloaded (middle of the longest resident run); returns it or -1
 int demote_one(int L, uint8_t* off);
+// Algorithm 1's block-level refinement on one device: masks[l] = resident blocks
+// of layer l (bit 0 MHA, bit 1 MLP); returns the memory still left
+uint64_t refine_blocks(uint64_t left, int L, const uint8_t* offloaded, uint64_t mha_bytes, uint64_t mlp_bytes,
+                       uint8_t* masks);
+// Eq. 7 on one device: alpha MHA and beta MLP blocks covering `need` with the
+// fewest bytes (then the fewest blocks); false if the available blocks cannot
+bool eq7_choice(uint64_t need, int n_mha, int n_mlp, uint64_t mha_bytes, uint64_t mlp_bytes, int* alpha, int* beta);
 }  // namespace loip

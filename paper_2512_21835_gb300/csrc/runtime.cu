@@ -155,8 +155,13 @@ struct loip_ctx {
     uint64_t block_bytes = 0, blocks_off = 0;
     int n_blocks = 0;
     std::vector<int> block_kind, block_owner;
-    std::vector<int> layer_block;   // resident block of each layer, -1 if offloaded
-    std::vector<uint8_t> offloaded;
+    std::vector<int> layer_block;   // block of each layer holding one or both of its blocks, -1 if none
+    std::vector<uint8_t> offloaded;  // 1: the layer streams at least one of its blocks through the slots
+    // block granularity: resident blocks of each layer (bit 0 MHA, bit 1 MLP;
+    // 3 = whole layer) and their device addresses (nullptr: streamed)
+    std::vector<uint8_t> res_mask;
+    std::vector<char*> mha_at, mlp_at;
+    uint64_t tail_off = 0, tail_used = 0;  // memory after the whole blocks: refined resident blocks
     std::vector<int> slot_block;
     std::vector<int> off_order;     // offloaded layers in order
     // KV
@@ -264,9 +269,25 @@ struct loip_ctx {
         return wait_event(ev_done);
     }
 
-    const uint16_t* layer_weights(int l, int slot) {
-        if (layer_block[l] >= 0) return reinterpret_cast<const uint16_t*>(block_ptr(layer_block[l]));
-        return reinterpret_cast<const uint16_t*>(slot_ptr(slot));
+    // Blob-relative bases of layer l's MHA and MLP blocks: base + lay.off_x is
+    // part x, whether the block is resident (at its own address) or streamed
+    // into `slot` (the slot holds the blob layout).
+    const uint16_t* mha_base(int l, int slot) {
+        return reinterpret_cast<const uint16_t*>(mha_at[l] ? mha_at[l] : slot_ptr(slot));
+    }
+    const uint16_t* mlp_base(int l, int slot) {
+        return reinterpret_cast<const uint16_t*>(mlp_at[l] ? mlp_at[l] - lay.mha_bytes : slot_ptr(slot));
+    }
+    // bytes layer l streams per pass
+    uint64_t stream_bytes(int l) const {
+        return ((res_mask[l] & 1) ? 0 : lay.mha_bytes) + ((res_mask[l] & 2) ? 0 : lay.mlp_bytes);
+    }
+    void set_resident_block(int l, int b) {  // whole layer in block b
+        layer_block[l] = b;
+        res_mask[l] = 3;
+        mha_at[l] = block_ptr(b);
+        mlp_at[l] = block_ptr(b) + lay.mha_bytes;
+        offloaded[l] = 0;
     }
 
     KvView kv_view(int layer, const int64_t* pt) {
@@ -287,6 +308,14 @@ struct loip_ctx {
         return -1;
     }
 
+    // page groups from a freed range [ptr, ptr + bytes) of the arena (256-aligned)
+    void carve_kv(const char* ptr, uint64_t bytes) {
+        const uint64_t off = (uint64_t)(ptr - arena);
+        const uint64_t n = bytes / group_bytes;
+        for (uint64_t i = 0; i < n; ++i) free_groups.push_back((int64_t)(off + i * group_bytes));
+        kv_groups_total += n;
+    }
+
     int grow_kv() {  // converts one free block into page groups
         int b = take_free_block();
         if (b < 0) return -1;
@@ -305,9 +334,9 @@ struct loip_ctx {
         while ((int)r.pages.size() < need) {
             if (free_groups.empty()) {
                 if (grow_kv() < 0) {
-                    int rc = demote_for_kv();
+                    int rc = demote_for_kv();  // frees a block, or carves groups from offloaded blocks
                     if (rc) return rc;
-                    if (grow_kv() < 0) return fail(LOIP_ERR_OOM, "no block for the KV cache");
+                    if (free_groups.empty() && grow_kv() < 0) return fail(LOIP_ERR_OOM, "no block for the KV cache");
                 }
             }
             r.pages.push_back(free_groups.back());
@@ -358,13 +387,17 @@ struct loip_ctx {
         if (e != cudaSuccess) return cuda_fail(e, "copy wait");
         cudaEvent_t e0 = take_event(), e1 = take_event();
         cudaEventRecord(e0, cs);
-        e = cudaMemcpyAsync(slot_ptr(slot), host_layer[layer], lay.l_size, cudaMemcpyHostToDevice, cs);
+        // the blocks the layer streams, at their blob offsets
+        const uint64_t off0 = (res_mask[layer] & 1) ? lay.mha_bytes : 0;
+        const uint64_t off1 = (res_mask[layer] & 2) ? lay.mha_bytes : lay.l_size;
+        e = cudaMemcpyAsync(slot_ptr(slot) + off0, static_cast<const char*>(host_layer[layer]) + off0, off1 - off0,
+                            cudaMemcpyHostToDevice, cs);
         if (e != cudaSuccess) return cuda_fail(e, "layer copy");
         cudaEventRecord(e1, cs);
         copy_events.emplace_back(e0, e1);
         e = cudaEventRecord(slot_full[slot], cs);
         if (e != cudaSuccess) return cuda_fail(e, "slot event");
-        st.h2d_weight_bytes += lay.l_size;
+        st.h2d_weight_bytes += stream_bytes(layer);
         return LOIP_OK;
     }
 
@@ -422,7 +455,7 @@ struct loip_ctx {
     // ---- one decoder layer ---------------------------------------------------
     // Decode-time layer on rows 0..B-1 of the fixed activations.
     int decode_layer(int l, int B, const int32_t* pos_dev, cudaStream_t s, int slot) {
-        return decode_layer_w(l, B, pos_dev, s, layer_weights(l, slot), false);
+        return decode_layer_w(l, B, pos_dev, s, mha_base(l, slot), mlp_base(l, slot), false, false);
     }
 
     // Device address of offloaded layer l's host blob (mapped pinned memory).
@@ -441,31 +474,36 @@ struct loip_ctx {
     // memory: no slots, no copy stream.
     int run_layers_direct(int B, const int32_t* pos_dev, cudaStream_t s) {
         for (int l = 0; l < L; ++l) {
-            const bool off = layer_block[l] < 0;
-            if (!off && fuse_runs(B)) {
+            if (res_mask[l] == 3 && fuse_runs(B)) {
                 int e = l;
-                while (e < L && layer_block[e] >= 0) ++e;
+                while (e < L && res_mask[e] == 3) ++e;
                 int rc = decode_run(l, e, pos_dev, s);
                 if (rc) return rc;
                 l = e - 1;
                 continue;
             }
-            const uint16_t* w = off ? host_direct(l) : layer_weights(l, -1);
-            if (!w) return fail(LOIP_ERR_STATE, "offloaded layer has no device-mapped host copy");
-            int rc = decode_layer_w(l, B, pos_dev, s, w, off);
+            const bool ha = !(res_mask[l] & 1), hm = !(res_mask[l] & 2);
+            const uint16_t* hw = (ha || hm) ? host_direct(l) : nullptr;
+            if ((ha || hm) && !hw) return fail(LOIP_ERR_STATE, "offloaded layer has no device-mapped host copy");
+            const uint16_t* wa = ha ? hw : mha_base(l, -1);
+            const uint16_t* wm = hm ? hw : mlp_base(l, -1);
+            int rc = decode_layer_w(l, B, pos_dev, s, wa, wm, ha, hm);
             if (rc) return rc;
         }
         return LOIP_OK;
     }
 
-    int decode_layer_w(int l, int B, const int32_t* pos_dev, cudaStream_t s, const uint16_t* w, bool w_host) {
-        const uint16_t* g_attn = w + lay.off_g_attn / 2;
-        const uint16_t* wqkv = w + lay.off_wqkv / 2;
-        const uint16_t* wo = w + lay.off_wo / 2;
-        const uint16_t* g_mlp = w + lay.off_g_mlp / 2;
-        const uint16_t* wg = w + lay.off_wg / 2;
-        const uint16_t* wu = w + lay.off_wu / 2;
-        const uint16_t* wd = w + lay.off_wd / 2;
+    // wa, wm: blob-relative bases of the MHA and MLP blocks (mha_base, mlp_base);
+    // host_a, host_m: that block is read in place from mapped host memory
+    int decode_layer_w(int l, int B, const int32_t* pos_dev, cudaStream_t s, const uint16_t* wa, const uint16_t* wm,
+                       bool host_a, bool host_m) {
+        const uint16_t* g_attn = wa + lay.off_g_attn / 2;
+        const uint16_t* wqkv = wa + lay.off_wqkv / 2;
+        const uint16_t* wo = wa + lay.off_wo / 2;
+        const uint16_t* g_mlp = wm + lay.off_g_mlp / 2;
+        const uint16_t* wg = wm + lay.off_wg / 2;
+        const uint16_t* wu = wm + lay.off_wu / 2;
+        const uint16_t* wd = wm + lay.off_wd / 2;
         float* x = fixed_ptr<float>(fx.x);
         float* q = fixed_ptr<float>(fx.q);
         float* o = fixed_ptr<float>(fx.o);
@@ -475,7 +513,7 @@ struct loip_ctx {
         cudaError_t e;
         e = timed(0, s, [&] {
             return launch_qkv_rope(x, g_attn, wqkv, B, H, Hq, Hkv, d, desc.rms_eps, desc.rope_theta, pos_dev, q, kv,
-                                   nullptr, s, pdl(), w_host);
+                                   nullptr, s, pdl(), host_a);
         });
         if (e != cudaSuccess) return cuda_fail(e, "qkv kernel");
         chain = true;
@@ -484,20 +522,21 @@ struct loip_ctx {
                                     fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl(), cfg.max_batch);
         });
         if (e != cudaSuccess) return cuda_fail(e, "attention kernel");
-        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl(), w_host); });
+        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl(), host_a); });
         if (e != cudaSuccess) return cuda_fail(e, "o-proj kernel");
         e = timed(3, s, [&] {
-            return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s, pdl(), w_host);
+            return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s, pdl(), host_m);
         });
         if (e != cudaSuccess) return cuda_fail(e, "gate/up kernel");
-        e = timed(4, s, [&] { return launch_resid_gemv(a, wd, B, H, F, x, s, pdl(), w_host); });
+        e = timed(4, s, [&] { return launch_resid_gemv(a, wd, B, H, F, x, s, pdl(), host_m); });
         if (e != cudaSuccess) return cuda_fail(e, "down kernel");
         return LOIP_OK;
     }
 
     // Prefill layer on Mc token rows held in the prefill workspace.
     int prefill_layer(int l, int Mc, cudaStream_t s, int slot) {
-        const uint16_t* w = layer_weights(l, slot);
+        const uint16_t* wa = mha_base(l, slot);
+        const uint16_t* wm = mlp_base(l, slot);
         float* px = fixed_ptr<float>(fx.px);
         uint16_t* py = fixed_ptr<uint16_t>(fx.py);
         float* pq = fixed_ptr<float>(fx.pq);
@@ -508,10 +547,10 @@ struct loip_ctx {
         const int64_t* pt = fixed_ptr<int64_t>(fx.page_table);
         KvView kv = kv_view(l, pt);
         cudaError_t e;
-        e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, w + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s); });
+        e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, wa + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s); });
         if (e == cudaSuccess)
             e = timed(6, s, [&] {
-                return launch_tc_gemm_qkv_rope(py, w + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos, req,
+                return launch_tc_gemm_qkv_rope(py, wa + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos, req,
                                                pq, kv, s);
             });
         if (e == cudaSuccess)
@@ -519,14 +558,14 @@ struct loip_ctx {
                 return launch_attention(pq, kv, nullptr, pos, req, Mc, Hq, Hkv, d, cfg.max_ctx, false, nullptr, po,
                                         true, s);
             });
-        if (e == cudaSuccess) e = timed(8, s, [&] { return launch_tc_gemm_resid(po, w + lay.off_wo / 2, Mc, H, qd, px, s); });
+        if (e == cudaSuccess) e = timed(8, s, [&] { return launch_tc_gemm_resid(po, wa + lay.off_wo / 2, Mc, H, qd, px, s); });
         if (e == cudaSuccess)
-            e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, w + lay.off_g_mlp / 2, Mc, H, desc.rms_eps, py, s); });
+            e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, wm + lay.off_g_mlp / 2, Mc, H, desc.rms_eps, py, s); });
         if (e == cudaSuccess)
             e = timed(9, s, [&] {
-                return launch_tc_gemm_swiglu(py, w + lay.off_wg / 2, w + lay.off_wu / 2, Mc, H, F, pa, s);
+                return launch_tc_gemm_swiglu(py, wm + lay.off_wg / 2, wm + lay.off_wu / 2, Mc, H, F, pa, s);
             });
-        if (e == cudaSuccess) e = timed(10, s, [&] { return launch_tc_gemm_resid(pa, w + lay.off_wd / 2, Mc, H, F, px, s); });
+        if (e == cudaSuccess) e = timed(10, s, [&] { return launch_tc_gemm_resid(pa, wm + lay.off_wd / 2, Mc, H, F, px, s); });
         if (e != cudaSuccess) return cuda_fail(e, "prefill kernel");
         return LOIP_OK;
     }
@@ -537,7 +576,7 @@ struct loip_ctx {
         for (int b0 = l0; b0 < l1; b0 += kMaxRunLayers) {
             const int b1 = std::min(l1, b0 + kMaxRunLayers);
             DecodeRunArgs a{};
-            for (int l = b0; l < b1; ++l) a.base[l - b0] = reinterpret_cast<const char*>(layer_weights(l, -1));
+            for (int l = b0; l < b1; ++l) a.base[l - b0] = mha_at[l];  // whole layers: the blob base
             a.n_layers = b1 - b0;
             a.layer0 = b0;
             a.off_g_attn = lay.off_g_attn;
@@ -647,7 +686,103 @@ struct loip_ctx {
     }
 
     // ---- online re-planning (Eq. 6) -------------------------------------------
-    int demote_for_kv() {
+    // Eq. 7 on one device: the resident blocks to offload for one more page
+    // group, the fewest bytes first (an MHA block while any is resident); the
+    // victim layer is the middle of the longest run of whole resident layers
+    // (keeping the streamed layers evenly spaced), else the first layer still
+    // holding a block of that kind.  The freed range becomes page groups.
+    int demote_block_for_kv(uint64_t need_groups) {
+        int n_mha = 0, n_mlp = 0;
+        for (int l = 0; l < L; ++l) {
+            n_mha += (res_mask[l] & 1) ? 1 : 0;
+            n_mlp += (res_mask[l] & 2) ? 1 : 0;
+        }
+        if (lay.mha_bytes < group_bytes) n_mha = 0;  // a block that cannot hold a page group frees nothing
+        if (lay.mlp_bytes < group_bytes) n_mlp = 0;
+        int alpha = 0, beta = 0;
+        if (!eq7_choice(need_groups * group_bytes, n_mha, n_mlp, lay.mha_bytes, lay.mlp_bytes, &alpha, &beta) &&
+            !eq7_choice(group_bytes, n_mha, n_mlp, lay.mha_bytes, lay.mlp_bytes, &alpha, &beta))
+            return fail(LOIP_ERR_OOM, "KV cache does not fit even with every block offloaded");
+        int rc = sync_all();
+        if (rc) return rc;
+        rc = ensure_slots();
+        if (rc) return rc;
+        for (int which = 0; which < 2; ++which) {
+            const int count = which == 0 ? alpha : beta;
+            const uint8_t bit = which == 0 ? 1 : 2;
+            for (int c = 0; c < count; ++c) {
+                std::vector<uint8_t> mask = offloaded;
+                int victim = -1;
+                bool any_whole = false;
+                for (int l = 0; l < L; ++l) any_whole |= res_mask[l] == 3;
+                if (any_whole) victim = demote_one(L, mask.data());
+                if (victim < 0 || !(res_mask[victim] & bit))
+                    for (int l = 0; l < L && victim < 0; ++l)
+                        if (res_mask[l] & bit) victim = l;
+                if (victim < 0 || !(res_mask[victim] & bit)) return fail(LOIP_ERR_STATE, "no resident block to offload");
+                rc = ensure_host_copy(victim);
+                if (rc) return rc;
+                if (bit == 1) {
+                    carve_kv(mha_at[victim], lay.mha_bytes);
+                    mha_at[victim] = nullptr;
+                } else {
+                    carve_kv(mlp_at[victim], lay.mlp_bytes);
+                    mlp_at[victim] = nullptr;
+                }
+                res_mask[victim] &= (uint8_t)~bit;
+                offloaded[victim] = 1;
+                if (res_mask[victim] == 0 && layer_block[victim] >= 0) {  // its whole block now serves the KV cache
+                    block_kind[layer_block[victim]] = B_KV;
+                    block_owner[layer_block[victim]] = -1;
+                    layer_block[victim] = -1;
+                }
+            }
+        }
+        rebuild_order();
+        st.n_replans++;
+        return prime_slots();
+    }
+
+    // The slot ring needs its blocks once a first layer streams: free blocks, or
+    // the blocks of whole layers taken for it.
+    int ensure_slots() {
+        if (!off_order.empty()) return LOIP_OK;
+        std::vector<uint8_t> mask = offloaded;
+        for (int k = 0; k < cfg.n_slots; ++k) {
+            int b = take_free_block();
+            if (b < 0) {
+                int v2 = demote_one(L, mask.data());
+                if (v2 < 0 || res_mask[v2] != 3) return fail(LOIP_ERR_OOM, "no room for slots");
+                int rc2 = demote_layer(v2);
+                if (rc2) return rc2;
+                b = take_free_block();
+            }
+            block_kind[b] = B_SLOT;
+            block_owner[b] = k;
+            slot_block[k] = b;
+        }
+        return LOIP_OK;
+    }
+
+    // a host copy of layer l's whole blob (gathered from its resident blocks)
+    int ensure_host_copy(int l) {
+        if (host_layer[l]) return LOIP_OK;
+        HostBuf hb;
+        cudaError_t e = host_buf_alloc(lay.l_size, &hb);
+        if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned allocation for a demoted layer failed");
+        host_regions.push_back(hb);
+        host_layer[l] = hb.ptr;
+        char* h = static_cast<char*>(hb.ptr);
+        if (mha_at[l]) e = cudaMemcpy(h, mha_at[l], lay.mha_bytes, cudaMemcpyDeviceToHost);
+        if (e == cudaSuccess && mlp_at[l]) e = cudaMemcpy(h + lay.mha_bytes, mlp_at[l], lay.mlp_bytes, cudaMemcpyDeviceToHost);
+        if (e != cudaSuccess) return cuda_fail(e, "demote copy");
+        return LOIP_OK;
+    }
+
+    // KV growth past the memory left (Eq. 6): make room for need_groups more page
+    // groups (at least one) by offloading blocks (Eq. 7) or one whole layer
+    int demote_for_kv(uint64_t need_groups = 1) {
+        if (!cfg.whole_layers) return demote_block_for_kv(need_groups < 1 ? 1 : need_groups);
         // offload one more resident layer; its block becomes free
         std::vector<uint8_t> mask = offloaded;
         int victim = demote_one(L, mask.data());
@@ -680,20 +815,15 @@ struct loip_ctx {
         return prime_slots();
     }
 
-    int demote_layer(int l) {
-        if (!host_layer[l]) {
-            HostBuf hb;
-            cudaError_t e = host_buf_alloc(lay.l_size, &hb);
-            if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned allocation for a demoted layer failed");
-            host_regions.push_back(hb);
-            host_layer[l] = hb.ptr;
-            e = cudaMemcpy(host_layer[l], block_ptr(layer_block[l]), lay.l_size, cudaMemcpyDeviceToHost);
-            if (e != cudaSuccess) return cuda_fail(e, "demote copy");
-        }
+    int demote_layer(int l) {  // a whole resident layer: its block becomes free
+        int rc = ensure_host_copy(l);
+        if (rc) return rc;
         int b = layer_block[l];
         block_kind[b] = B_FREE;
         block_owner[b] = -1;
         layer_block[l] = -1;
+        res_mask[l] = 0;
+        mha_at[l] = mlp_at[l] = nullptr;
         offloaded[l] = 1;
         return LOIP_OK;
     }
@@ -770,7 +900,7 @@ struct loip_ctx {
     }
 
     uint64_t arena_used() const {
-        uint64_t used = fx.total + kv_region_bytes;
+        uint64_t used = fx.total + kv_region_bytes + tail_used;
         for (int b = 0; b < n_blocks; ++b)
             if (block_kind[b] != B_FREE) used += block_bytes;
         return used;
@@ -899,12 +1029,15 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     }
     c->offloaded.assign(c->L, 0);
     c->layer_block.assign(c->L, -1);
+    c->res_mask.assign(c->L, 0);
+    c->mha_at.assign(c->L, nullptr);
+    c->mlp_at.assign(c->L, nullptr);
     c->block_kind.assign(c->n_blocks, B_FREE);
     c->block_owner.assign(c->n_blocks, -1);
     int nb = 0;
     for (int l = 0; l < c->L; ++l) {
         if (res[l]) {
-            c->layer_block[l] = nb;
+            c->set_resident_block(l, nb);
             c->block_kind[nb] = B_LAYER;
             c->block_owner[nb] = l;
             ++nb;
@@ -925,6 +1058,26 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
             c->block_kind[nb] = B_SLOT;
             c->block_owner[nb] = k;
             ++nb;
+        }
+    }
+    // Algorithm 1's block-level refinement: the memory after the whole blocks
+    // keeps blocks of offloaded layers resident (MLP block first)
+    c->tail_off = c->blocks_off + (uint64_t)c->n_blocks * c->block_bytes;
+    if (!cfg.whole_layers && !c->off_order.empty() && c->budget > c->tail_off) {
+        std::vector<uint8_t> masks(c->L);
+        refine_blocks(c->budget - c->tail_off, c->L, c->offloaded.data(), c->lay.mha_bytes, c->lay.mlp_bytes,
+                      masks.data());
+        for (int l = 0; l < c->L; ++l) {
+            if (!c->offloaded[l] || masks[l] == 0) continue;
+            char* at = c->arena + c->tail_off + c->tail_used;
+            if (masks[l] == 2) {
+                c->mlp_at[l] = at;
+                c->tail_used += c->lay.mlp_bytes;
+            } else {
+                c->mha_at[l] = at;
+                c->tail_used += c->lay.mha_bytes;
+            }
+            c->res_mask[l] = masks[l];
         }
     }
     for (uint64_t i = 0; i < kv_groups; ++i)
@@ -980,16 +1133,29 @@ extern "C" int loip_get_plan(const loip_ctx* ctx, loip_plan* out) {
     out->n_resident = ctx->L - out->n_offloaded;
     for (int l = 0; l < ctx->L; ++l) out->resident[l] = ctx->offloaded[l] ? 0 : 1;
     std::vector<double> comp(ctx->L), load(ctx->L);
+    double copy_s = 0;
     for (int l = 0; l < ctx->L; ++l) {
-        comp[l] = (double)ctx->block_bytes / ctx->cfg.hbm_Bps;
-        load[l] = (double)ctx->block_bytes / ctx->cfg.link_Bps;
+        comp[l] = (double)ctx->lay.l_size / ctx->cfg.hbm_Bps;
+        load[l] = (double)ctx->stream_bytes(l) / ctx->cfg.link_Bps;
+        if (ctx->offloaded[l]) copy_s += load[l];
     }
     out->pred_step_s = simulate_step(comp, load, ctx->offloaded.data(), ctx->cfg.n_slots, 4);
     out->eq1_step_s = eq1_single_device(comp, load, ctx->offloaded.data());
-    out->pred_copy_s = out->n_offloaded * load[0];
+    out->pred_copy_s = copy_s;
     out->pred_compute_s = ctx->L * comp[0];
     uint64_t used = ctx->arena_used();
     out->left_bytes = ctx->budget > used ? ctx->budget - used : 0;
+    return LOIP_OK;
+}
+
+extern "C" int loip_get_block_plan(const loip_ctx* ctx, uint8_t* masks, uint64_t* stream_bytes_per_step) {
+    if (!ctx || !masks || !stream_bytes_per_step) return LOIP_ERR_INVALID;
+    uint64_t bytes = 0;
+    for (int l = 0; l < ctx->L; ++l) {
+        masks[l] = ctx->res_mask[l];
+        bytes += ctx->stream_bytes(l);
+    }
+    *stream_bytes_per_step = bytes;
     return LOIP_OK;
 }
 
@@ -1028,8 +1194,8 @@ extern "C" int loip_load_weights_generated(loip_ctx* c, uint64_t seed) {
         e = launch_generate(c->fixed_ptr<uint16_t>(c->fx.g_final), (uint64_t)c->H, 0, seed, 3, 1, c->compute);
     if (e != cudaSuccess) return c->cuda_fail(e, "generator kernel");
     for (int l = 0; l < c->L; ++l) {
-        if (c->layer_block[l] >= 0) {
-            rc = write_layer_generated(c, c->block_ptr(c->layer_block[l]), l, seed);
+        if (c->res_mask[l] == 3) {
+            rc = write_layer_generated(c, c->mha_at[l], l, seed);
             if (rc) return rc;
         } else {
             rc = c->ensure_host_pool();
@@ -1038,6 +1204,11 @@ extern "C" int loip_load_weights_generated(loip_ctx* c, uint64_t seed) {
             rc = write_layer_generated(c, tmp, l, seed);
             if (rc) return rc;
             e = cudaMemcpyAsync(c->host_layer[l], tmp, c->lay.l_size, cudaMemcpyDeviceToHost, c->compute);
+            if (e == cudaSuccess && c->mha_at[l])  // its resident block (block-level refinement)
+                e = cudaMemcpyAsync(c->mha_at[l], tmp, c->lay.mha_bytes, cudaMemcpyDeviceToDevice, c->compute);
+            if (e == cudaSuccess && c->mlp_at[l])
+                e = cudaMemcpyAsync(c->mlp_at[l], tmp + c->lay.mha_bytes, c->lay.mlp_bytes, cudaMemcpyDeviceToDevice,
+                                    c->compute);
             if (e != cudaSuccess) return c->cuda_fail(e, "host pool copy");
         }
     }
@@ -1058,12 +1229,13 @@ extern "C" int loip_load_layer(loip_ctx* c, int32_t layer, const void* host_blob
     rc = c->ensure_host_pool();  // every offloaded layer gets its pool blob before the ring is primed
     if (rc) return rc;
     cudaError_t e;
-    if (c->layer_block[layer] >= 0) {
-        e = cudaMemcpy(c->block_ptr(c->layer_block[layer]), host_blob, bytes, cudaMemcpyHostToDevice);
-        if (e != cudaSuccess) return c->cuda_fail(e, "layer upload");
-    } else {
-        memcpy(c->host_layer[layer], host_blob, bytes);
-    }
+    const char* hb = static_cast<const char*>(host_blob);
+    if (c->res_mask[layer] != 3) memcpy(c->host_layer[layer], host_blob, bytes);
+    e = cudaSuccess;
+    if (c->mha_at[layer]) e = cudaMemcpy(c->mha_at[layer], hb, c->lay.mha_bytes, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && c->mlp_at[layer])
+        e = cudaMemcpy(c->mlp_at[layer], hb + c->lay.mha_bytes, c->lay.mlp_bytes, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return c->cuda_fail(e, "layer upload");
     c->weights_loaded = true;
     rc = c->prime_slots();
     return rc ? rc : c->sync_all();
@@ -1347,7 +1519,7 @@ extern "C" int loip_replan(loip_ctx* c, int32_t lookahead_tokens) {
     }
     while (c->free_groups.size() < need) {
         if (c->grow_kv() >= 0) continue;
-        int rc = c->demote_for_kv();
+        int rc = c->demote_for_kv(need - c->free_groups.size());
         if (rc) return rc;
     }
     return LOIP_OK;

@@ -36,7 +36,7 @@ class Config(C.Structure):
     _fields_ = [("device_budget_bytes", C.c_uint64), ("n_slots", C.c_int32), ("page_tokens", C.c_int32),
                 ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("layer_run_kernel", C.c_int32), ("mode", C.c_int32),
                 ("timeout_ms", C.c_uint32), ("hbm_Bps", C.c_double), ("link_Bps", C.c_double),
-                ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32)]
+                ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32), ("whole_layers", C.c_int32)]
 
 
 class LayerLayout(C.Structure):
@@ -65,6 +65,8 @@ _SIGS = {
     "loip_layer_layout": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(LayerLayout)]),
     "loip_plan_residency": (C.c_int, [C.POINTER(ModelDesc), P, U64, U64, U64, I32, F64, F64, C.POINTER(Plan)]),
     "loip_kv_threshold": (C.c_int, [U64, U64, C.POINTER(C.c_uint64)]),
+    "loip_refine_blocks": (C.c_int, [C.POINTER(ModelDesc), U64, P, P, C.POINTER(C.c_uint64)]),
+    "loip_eq7_choice": (C.c_int, [C.POINTER(ModelDesc), U64, I32, I32, C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
     "loip_fixed_bytes": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(Config), C.POINTER(C.c_uint64)]),
     "loip_create": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(Config), P, U64, C.POINTER(C.c_void_p)]),
     "loip_destroy": (None, [P]),
@@ -73,6 +75,7 @@ _SIGS = {
     "loip_load_layer": (C.c_int, [P, I32, P, U64]),
     "loip_load_globals": (C.c_int, [P, P, P, P]),
     "loip_get_plan": (C.c_int, [P, C.POINTER(Plan)]),
+    "loip_get_block_plan": (C.c_int, [P, P, C.POINTER(C.c_uint64)]),
     "loip_stream_layer": (C.c_int, [P, I32, I32, P]),
     "loip_layer_forward": (C.c_int, [P, I32, I32, P, P, I32, P]),
     "loip_set_batch": (C.c_int, [P, I32, P]),
@@ -150,10 +153,10 @@ def model_desc(m: dict) -> ModelDesc:
 
 def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 2048, mode: int = MODE_OVERLAP,
            timeout_ms: int = 0, hbm_Bps: float = 6.7e12, link_Bps: float = 2.1e11, kv_reserve_bytes: int = 0,
-           max_prefill_tokens: int = 512, page_tokens: int = 64, layer_run_kernel: int = 0) -> Config:
+           max_prefill_tokens: int = 512, page_tokens: int = 64, layer_run_kernel: int = 0,
+           whole_layers: int = 0) -> Config:
     return Config(budget, n_slots, page_tokens, max_batch, max_ctx, layer_run_kernel, mode, timeout_ms, hbm_Bps,
-                  link_Bps,
-                  kv_reserve_bytes, max_prefill_tokens)
+                  link_Bps, kv_reserve_bytes, max_prefill_tokens, whole_layers)
 
 
 # ----------------------------------------------------------------------------
@@ -176,6 +179,26 @@ def loip_plan_residency(m: dict, layer_bytes, budget: int, kv_bytes: int, fixed_
     return {"n_resident": plan.n_resident, "n_offloaded": plan.n_offloaded, "resident": res.astype(bool),
             "pred_step_s": plan.pred_step_s, "pred_copy_s": plan.pred_copy_s, "pred_compute_s": plan.pred_compute_s,
             "eq1_step_s": plan.eq1_step_s, "left_bytes": plan.left_bytes}
+
+
+def loip_refine_blocks(m: dict, left_bytes: int, offloaded) -> tuple:
+    """Algorithm 1's block-level refinement: (per-layer resident-block masks, bytes left)."""
+    off = np.ascontiguousarray(offloaded, dtype=np.uint8)
+    masks = np.zeros(off.size, dtype=np.uint8)
+    left = C.c_uint64()
+    _check(lib().loip_refine_blocks(C.byref(model_desc(m)), left_bytes, off.ctypes.data, masks.ctypes.data,
+                                    C.byref(left)))
+    return masks, left.value
+
+
+def loip_eq7_choice(m: dict, need_bytes: int, n_mha: int, n_mlp: int):
+    """Eq. 7: (alpha, beta) resident MHA / MLP blocks to offload, or None."""
+    a, b = C.c_int32(), C.c_int32()
+    rc = lib().loip_eq7_choice(C.byref(model_desc(m)), need_bytes, n_mha, n_mlp, C.byref(a), C.byref(b))
+    if rc == 3:  # LOIP_ERR_INFEASIBLE
+        return None
+    _check(rc)
+    return a.value, b.value
 
 
 def loip_kv_threshold(left_bytes: int, kv_bytes_per_token: int) -> int:
@@ -252,6 +275,13 @@ class Context:
         self._c(lib().loip_get_plan(self.h, C.byref(p)))
         return {"n_resident": p.n_resident, "n_offloaded": p.n_offloaded, "resident": res.astype(bool),
                 "pred_step_s": p.pred_step_s, "eq1_step_s": p.eq1_step_s, "left_bytes": p.left_bytes}
+
+    def block_plan(self) -> dict:
+        """Resident blocks per layer (bit 0 MHA, bit 1 MLP) and bytes streamed per pass."""
+        masks = np.zeros(self.model["n_layers"], dtype=np.uint8)
+        b = C.c_uint64()
+        self._c(lib().loip_get_block_plan(self.h, masks.ctypes.data, C.byref(b)))
+        return {"masks": masks, "stream_bytes": b.value}
 
     def set_batch(self, ctx_lens):
         cl = np.ascontiguousarray(ctx_lens, dtype=np.int32)

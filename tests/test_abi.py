@@ -102,3 +102,24 @@ def test_fixed_bytes(L):
                                               max_prefill_tokens=1024))
     # embedding + LM head dominate: 2 x 128256 x 8192 x 2 bytes
     assert 2 * 128256 * 8192 * 2 < fb < 2 * 128256 * 8192 * 2 + 400 * 2 ** 20
+
+
+@pytest.mark.parametrize("model", ["tiny", "llama3-8b", "llama3-70b"])
+def test_block_refinement_and_eq7_match_planner_oracle(L, model):
+    """loip_refine_blocks / loip_eq7_choice (C) against the planner oracle, on the
+    model's real block sizes."""
+    import random
+    m = configs.MODELS[model]
+    lay = loip.loip_layer_layout(m)
+    A, M = lay["mha_bytes"], lay["mlp_bytes"]
+    rng = random.Random(7)
+    for _ in range(50):
+        Lm = m["n_layers"]
+        off = [rng.random() < 0.6 for _ in range(Lm)]
+        left = rng.randint(0, 3 * M)
+        masks, rest = loip.loip_refine_blocks(m, left, off)
+        want, want_rest = OP.refine_blocks(left, off, A, M)
+        assert list(masks) == want and rest == want_rest
+        na, nm = rng.randint(0, Lm), rng.randint(0, Lm)
+        need = rng.randint(0, 2 * M)
+        assert loip.loip_eq7_choice(m, need, na, nm) == OP.eq7_choice(need, na, nm, A, M)

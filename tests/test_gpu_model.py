@@ -278,3 +278,75 @@ def test_mixed_batch_sizes_share_attention_scratch(torch, L, orc):
         ctx.decode_step([seq0[40 + i]], out_hidden=h1)
         _check_hidden(h1[0].cpu().numpy(), hids0[i])
     ctx.close()
+
+
+@pytest.mark.parametrize("extra,mode", [("mlp", 0), ("mha2", 0), ("mlp", 2), ("mlp", 1)])
+def test_block_level_residency_is_bitwise_lossless(torch, L, orc, extra, mode):
+    """Algorithm 1's block-level refinement: memory left after the whole-layer
+    plan keeps the MLP block (or MHA blocks) of streamed layers resident; only
+    the other block streams, and results stay bit-identical to all-resident."""
+    m = TINY6
+    lay = L.loip_layer_layout(m)
+    prompts = [inputs.token_ids(71, 20, m["vocab"]), inputs.token_ids(72, 9, m["vocab"])]
+    cont = [[int(a), int(b)] for a, b in zip(inputs.token_ids(73, 6, 1024), inputs.token_ids(74, 6, 1024))]
+    base = _run(L, torch, m, prompts, cont, dict(max_batch=2, max_ctx=64), 6)
+    kw = dict(max_batch=2, max_ctx=64, n_slots=1 if mode == 1 else 2, mode=mode)
+    budget = _budget(L, m, kw, 2) - (lay["l_size"] + 255) // 256 * 256 // 2  # no slack beyond the whole blocks
+    budget += lay["mlp_bytes"] + 256 if extra == "mlp" else 2 * lay["mha_bytes"] + 256
+    ctx = L.Context(m, L.config(budget=budget, **kw))
+    bp = ctx.block_plan()
+    masks = list(bp["masks"])
+    assert masks.count(3) == 2
+    if extra == "mlp":
+        assert masks.count(2) == 1 and bp["stream_bytes"] == 3 * lay["l_size"] + lay["mha_bytes"]
+    else:
+        assert masks.count(1) == 2 and bp["stream_bytes"] == 4 * lay["l_size"] - 2 * lay["mha_bytes"]
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    hid = torch.empty(2, m["hidden"], dtype=torch.float32, device="cuda")
+    toks = [ctx.prefill(prompts, out_hidden=hid)]
+    hids = [hid.cpu().numpy().copy()]
+    for step in cont:
+        toks.append(ctx.decode_step(step, out_hidden=hid))
+        hids.append(hid.cpu().numpy().copy())
+    ctx.close()
+    assert np.array_equal(np.array(toks), base[0])
+    assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
+
+
+@pytest.mark.parametrize("whole", [0, 1])
+def test_kv_growth_offloads_blocks_or_layers(torch, L, orc, whole):
+    """KV growth past the reserve: block granularity (Eq. 7) offloads one MHA
+    block (the smallest resident block covering a page group); whole-layer mode
+    offloads a layer.  Results stay bit-identical either way."""
+    m = TINY6
+    prompt = inputs.token_ids(41, 60, m["vocab"])
+    cont = [[int(t)] for t in inputs.token_ids(42, 10, m["vocab"])]
+    kw = dict(max_batch=1, max_ctx=128, n_slots=2, whole_layers=whole)
+    base = _run(L, torch, m, [prompt], cont, dict(max_batch=1, max_ctx=128, n_slots=2), 6)
+    lay = L.loip_layer_layout(m)
+    cfg0 = L.config(budget=1 << 40, **kw)
+    fixed = L.loip_fixed_bytes(m, cfg0)
+    group = ((2 * m["n_kv_heads"] * 64 * m["head_dim"] * 2 * m["n_layers"]) + 255) // 256 * 256
+    blk = (lay["l_size"] + 255) // 256 * 256
+    budget = fixed + group + 256 + 6 * blk + blk // 3  # every layer resident, no room for more KV
+    ctx = L.Context(m, L.config(budget=budget, kv_reserve_bytes=group, **kw))
+    assert ctx.plan()["n_offloaded"] == 0
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    hid = torch.empty(1, m["hidden"], dtype=torch.float32, device="cuda")
+    toks = [ctx.prefill([prompt], out_hidden=hid)]
+    hids = [hid.cpu().numpy().copy()]
+    for step in cont:
+        toks.append(ctx.decode_step(step, out_hidden=hid))
+        hids.append(hid.cpu().numpy().copy())
+    st = ctx.stats()
+    masks = list(ctx.block_plan()["masks"])
+    ctx.close()
+    assert st["n_replans"] >= 1 and st["arena_used"] <= budget
+    # the first streamed layer needs the two slots: two whole layers make room for them; then the
+    # page group comes from one more whole layer, or (Eq. 7) from one MHA block
+    if whole:
+        assert masks.count(0) == 3 and masks.count(3) == 3
+    else:
+        assert masks.count(0) == 2 and masks.count(2) == 1 and masks.count(3) == 3
+    assert np.array_equal(np.array(toks), base[0])
+    assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
