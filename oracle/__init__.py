@@ -57,7 +57,7 @@ class _Tensor(C.Structure):
 class _Desc(C.Structure):
     _fields_ = [("n_layers", C.c_int32), ("hidden", C.c_int32), ("n_heads", C.c_int32),
                 ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32), ("ffn", C.c_int32),
-                ("vocab", C.c_int32), ("rms_eps", C.c_double), ("rope_theta", C.c_double)]
+                ("vocab", C.c_int32), ("rms_eps", C.c_double), ("rope_theta", C.c_double), ("qk_norm", C.c_int32)]
 
 
 _lib = None
@@ -167,13 +167,17 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
 # ----------------------------------------------------------------------------
 class ModelDesc:
     def __init__(self, n_layers, hidden, n_heads, n_kv_heads, head_dim, ffn, vocab, rms_eps=1e-5,
-                 rope_theta=500000.0):
+                 rope_theta=500000.0, qk_norm=0):
         self.n_layers, self.hidden, self.n_heads, self.n_kv_heads = n_layers, hidden, n_heads, n_kv_heads
         self.head_dim, self.ffn, self.vocab, self.rms_eps, self.rope_theta = head_dim, ffn, vocab, rms_eps, rope_theta
+        self.qk_norm = int(qk_norm)
 
     def c(self) -> _Desc:
         return _Desc(self.n_layers, self.hidden, self.n_heads, self.n_kv_heads, self.head_dim, self.ffn, self.vocab,
-                     self.rms_eps, self.rope_theta)
+                     self.rms_eps, self.rope_theta, self.qk_norm)
+
+    def n_tensors(self) -> int:
+        return 3 + 9 * self.n_layers + (2 * self.n_layers if self.qk_norm else 0)
 
     def shapes(self):
         """Per-tensor shapes in oracle order."""
@@ -182,18 +186,25 @@ class ModelDesc:
         s = [(V, H), (V, H), (H,)]
         for _ in range(self.n_layers):
             s += [(H,), (qd, H), (kvd, H), (kvd, H), (H, qd), (H,), (F, H), (F, H), (H, F)]
+        if self.qk_norm:  # g_q, g_k per layer, after every layer's main tensors
+            s += [(self.head_dim,)] * (2 * self.n_layers)
         return s
 
     def kinds(self):
         k = [0, 0, 1]
         for _ in range(self.n_layers):
             k += [1, 0, 0, 0, 0, 1, 0, 0, 0]
+        if self.qk_norm:
+            k += [1] * (2 * self.n_layers)
         return k
 
     def ids(self):
         ids = [tensor_id(-1, w) for w in range(3)]
         for l in range(self.n_layers):
             ids += [tensor_id(l, w) for w in range(9)]
+        if self.qk_norm:
+            for l in range(self.n_layers):
+                ids += [tensor_id(l, 9), tensor_id(l, 10)]
         return ids
 
 
@@ -203,7 +214,7 @@ class Weights:
 
     def __init__(self, desc: ModelDesc, seed: int, arrays=None):
         self.desc, self.seed = desc, seed
-        n = 3 + 9 * desc.n_layers
+        n = desc.n_tensors()
         self.arrays = list(arrays) if arrays is not None else [None] * n
         assert len(self.arrays) == n
 

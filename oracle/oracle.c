@@ -204,13 +204,14 @@ void orc_attention(const double* q, const double* K, const double* V, int64_t T,
 typedef struct {
     int32_t n_layers, hidden, n_heads, n_kv_heads, head_dim, ffn, vocab;
     double rms_eps, rope_theta;
+    int32_t qk_norm; /* Qwen3: per-head RMSNorm of q and k (gains g_q, g_k [d]) before RoPE */
 } orc_desc;
 
 /* Tensor order: embed [V,H], lm_head [V,H], g_final [H], then per layer:
  * g_attn [H], wq [Hq*d,H], wk [Hkv*d,H], wv [Hkv*d,H], wo [H,Hq*d], g_mlp [H],
- * wg [F,H], wu [F,H], wd [H,F]. */
+ * wg [F,H], wu [F,H], wd [H,F]; with qk_norm, then per layer g_q [d], g_k [d]. */
 enum { T_EMBED = 0, T_LMHEAD = 1, T_GFINAL = 2, T_LAYER0 = 3, T_PER_LAYER = 9 };
-enum { L_GATTN = 0, L_WQ, L_WK, L_WV, L_WO, L_GMLP, L_WG, L_WU, L_WD };
+enum { L_GATTN = 0, L_WQ, L_WK, L_WV, L_WO, L_GMLP, L_WG, L_WU, L_WD, L_GQ, L_GK };
 
 /* Tensor ids used by the generator (the device library uses the same ids). */
 uint32_t orc_tensor_id(int layer, int which) {
@@ -234,6 +235,15 @@ void orc_generated_tensors(const orc_desc* d, uint64_t seed, orc_tensor* ts) {
             t->tensor_id = orc_tensor_id(l, w);
             t->kind = (w == L_GATTN || w == L_GMLP) ? 1 : 0;
         }
+    if (d->qk_norm)
+        for (int l = 0; l < d->n_layers; ++l)
+            for (int w = 0; w < 2; ++w) {
+                orc_tensor* t = &ts[T_LAYER0 + T_PER_LAYER * d->n_layers + 2 * l + w];
+                t->data = NULL;
+                t->seed = seed;
+                t->tensor_id = orc_tensor_id(l, L_GQ + w);
+                t->kind = 1;
+            }
 }
 
 static double maybe_bf16(double v, int on) { return on ? round_bf16(v) : v; }
@@ -288,6 +298,11 @@ int orc_forward(const orc_desc* d, const orc_tensor* ts, const int32_t* tokens, 
             orc_gemv(&lt[L_WQ], H, NULL, qd, y, q);
             orc_gemv(&lt[L_WK], H, NULL, kvd, y, k);
             orc_gemv(&lt[L_WV], H, NULL, kvd, y, v);
+            if (d->qk_norm) { /* per-head RMSNorm with the layer's g_q / g_k, before the rotation */
+                const orc_tensor* qk = &ts[T_LAYER0 + T_PER_LAYER * L + 2 * l];
+                for (int h = 0; h < Hq; ++h) orc_rmsnorm(q + (size_t)h * hd, &qk[0], hd, d->rms_eps, q + (size_t)h * hd);
+                for (int h = 0; h < Hkv; ++h) orc_rmsnorm(k + (size_t)h * hd, &qk[1], hd, d->rms_eps, k + (size_t)h * hd);
+            }
             for (int h = 0; h < Hq; ++h) orc_rope(q + (size_t)h * hd, hd, t, d->rope_theta);
             for (int h = 0; h < Hkv; ++h) orc_rope(k + (size_t)h * hd, hd, t, d->rope_theta);
             for (int i = 0; i < qd; ++i) q[i] = maybe_bf16(q[i], qb);

@@ -52,11 +52,17 @@ def numpy_forward(orc, desc, W, tokens, kv_bf16=True):
         return Z / np.sqrt(np.mean(Z * Z, axis=-1, keepdims=True) + desc.rms_eps) * g
 
     causal = np.tril(np.ones((n, n), dtype=bool))
+    qk_norm = getattr(desc, "qk_norm", 0)
     for l in range(desc.n_layers):
         b = 3 + 9 * l
         Y = rms(X, T(b + 0))
-        Q = rot((Y @ T(b + 1).T).reshape(n, Hq, d))
-        K = rot((Y @ T(b + 2).T).reshape(n, Hkv, d))
+        Q = (Y @ T(b + 1).T).reshape(n, Hq, d)
+        K = (Y @ T(b + 2).T).reshape(n, Hkv, d)
+        if qk_norm:  # per-head RMSNorm of q and k with the layer's gains, then the rotation
+            gq = T(3 + 9 * desc.n_layers + 2 * l)
+            gk = T(3 + 9 * desc.n_layers + 2 * l + 1)
+            Q, K = rms(Q, gq), rms(K, gk)
+        Q, K = rot(Q), rot(K)
         V = (Y @ T(b + 3).T).reshape(n, Hkv, d)
         if kv_bf16:
             K, V = _bf16_round_np(K), _bf16_round_np(V)
@@ -176,3 +182,38 @@ def test_bad_arguments_rejected(orc):
     desc = _desc(orc)
     with pytest.raises(ValueError):
         orc.forward(desc, orc.Weights(desc, 1), np.array([0, desc.vocab], dtype=np.int32))
+
+
+QK = dict(n_layers=2, hidden=256, n_heads=8, n_kv_heads=2, head_dim=64, ffn=688, vocab=1024, rms_eps=1e-6,
+          rope_theta=1000000.0, qk_norm=1)
+
+
+def test_qk_norm_forward_matches_independent_numpy(orc):
+    """Qwen3-style layer (per-head RMSNorm of q and k before RoPE, query width 512 != hidden 256)."""
+    desc = orc.ModelDesc(**QK)
+    W = orc.Weights.materialize(desc, configs.WEIGHT_SEED)
+    toks = inputs.token_ids(9, 18, desc.vocab)
+    out = orc.forward(desc, W, toks, want_logits=True)
+    Z, LG = numpy_forward(orc, desc, W, toks)
+    assert np.max(np.abs(out["hidden"] - Z)) < 1e-9
+    assert np.max(np.abs(out["logits"] - LG)) < 1e-9
+    # the norm is really there: the generated (flag off) model differs
+    plain = orc.forward(orc.ModelDesc(**dict(QK, qk_norm=0)), orc.Weights(orc.ModelDesc(**dict(QK, qk_norm=0)),
+                                                                        configs.WEIGHT_SEED), toks)
+    assert np.max(np.abs(plain["hidden"] - out["hidden"])) > 1e-3
+
+
+def test_qk_norm_makes_attention_invariant_to_query_and_key_scale(orc):
+    """RMSNorm per head removes any positive scale of Wq or Wk (up to eps, taken
+    negligible here): the forward with Wq x 8 and Wk x 0.125 equals the original."""
+    desc = orc.ModelDesc(**dict(QK, rms_eps=1e-12))
+    W = orc.Weights.materialize(desc, 11)
+    toks = inputs.token_ids(12, 10, desc.vocab)
+    a = orc.forward(desc, W, toks, prefill_flags=0, decode_flags=0)
+    arrs = list(W.arrays)
+    for l in range(desc.n_layers):
+        for off, f in ((1, 8.0), (2, 0.125)):  # exact in bf16: powers of two
+            x = orc.bf16_bits_to_f64(arrs[3 + 9 * l + off]) * f
+            arrs[3 + 9 * l + off] = (x.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    b = orc.forward(desc, orc.Weights(desc, 11, arrs), toks, prefill_flags=0, decode_flags=0)
+    assert np.max(np.abs(a["hidden"] - b["hidden"])) < 1e-9

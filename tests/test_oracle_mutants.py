@@ -43,6 +43,9 @@ MUTANTS = {
     "keys and values swapped": ("orc_gemv(&lt[L_WK], H, NULL, kvd, y, k);\n            orc_gemv(&lt[L_WV], H, NULL, kvd, y, v);",
                                 "orc_gemv(&lt[L_WK], H, NULL, kvd, y, v);\n            orc_gemv(&lt[L_WV], H, NULL, kvd, y, k);"),
     "softmax not normalised": ("double p = s[t] / l;", "double p = s[t];"),
+    "keys and queries rotated before the qk-norm too": ("            if (d->qk_norm) { /* per-head RMSNorm with the layer's g_q / g_k, before the rotation */",
+                                   "            for (int h = 0; h < Hq; ++h) orc_rope(q + (size_t)h * hd, hd, t, d->rope_theta);\n            for (int h = 0; h < Hkv; ++h) orc_rope(k + (size_t)h * hd, hd, t, d->rope_theta);\n            if (d->qk_norm) {"),
+    "qk-norm uses the query gain for keys": ("orc_rmsnorm(k + (size_t)h * hd, &qk[1], hd,", "orc_rmsnorm(k + (size_t)h * hd, &qk[0], hd,"),
     "kv rounding skipped": ("Kl[(size_t)t * kvd + i] = maybe_bf16(k[i], kvb);", "Kl[(size_t)t * kvd + i] = k[i];"),
 }
 
