@@ -58,6 +58,8 @@ typedef struct loip_model_desc {
     int32_t n_layers, hidden, n_heads, n_kv_heads, head_dim, ffn, vocab;
     float rms_eps;    /* RMSNorm epsilon */
     float rope_theta; /* rotary base */
+    int32_t qk_norm;  /* 1: Qwen3-style layer, a per-head RMSNorm of the queries and keys
+                       * (gains g_q, g_k [head_dim], epsilon rms_eps) before the rotation */
 } loip_model_desc;
 
 typedef struct loip_config {
@@ -87,6 +89,7 @@ typedef struct loip_layer_layout_t {
     uint64_t off_g_attn, off_wqkv, off_wo, off_g_mlp, off_wg, off_wu, off_wd;
     uint64_t l_size;   /* blob bytes */
     uint64_t mha_bytes, mlp_bytes;
+    uint64_t off_g_q, off_g_k;  /* QK-norm gains (qk_norm models; inside the MHA block, after Wo) */
 } loip_layer_layout_t;
 
 typedef struct loip_plan {

@@ -19,6 +19,13 @@ MODELS = {
                       rms_eps=1e-5, rope_theta=500000.0),
     "llama3-70b": dict(n_layers=80, hidden=8192, n_heads=64, n_kv_heads=8, head_dim=128, ffn=28672, vocab=128256,
                        rms_eps=1e-5, rope_theta=500000.0),
+    # Qwen3-style layers (per-head RMSNorm of queries and keys before the rotation;
+    # query width Hq x d larger than the hidden size)
+    "tiny-qk": dict(n_layers=2, hidden=256, n_heads=8, n_kv_heads=2, head_dim=64, ffn=688, vocab=1024,
+                    rms_eps=1e-6, rope_theta=1000000.0, qk_norm=1),
+    # the paper's Qwen3-32B model shape
+    "qwen3-32b": dict(n_layers=64, hidden=5120, n_heads=64, n_kv_heads=8, head_dim=128, ffn=25600, vocab=151936,
+                      rms_eps=1e-6, rope_theta=1000000.0, qk_norm=1),
 }
 
 WEIGHT_SEED = 0x10A1B
@@ -30,6 +37,7 @@ WORKLOADS = {
     "tiny-decode": dict(model="tiny", batch=1, prompt=32, decode=16, budget=None, n_slots=2),
     "8b-decode": dict(model="llama3-8b", batch=1, prompt=512, decode=128, budget=None, n_slots=2),
     "13b-decode": dict(model="llama2-13b", batch=1, prompt=512, decode=128, budget=None, n_slots=2),
+    "32b-decode": dict(model="qwen3-32b", batch=1, prompt=512, decode=128, budget=None, n_slots=2),
     "70b-offload-decode": dict(model="llama3-70b", batch=1, prompt=1024, decode=64, budget=60_000_000_000,
                                n_slots=2),
     "70b-offload-prefill": dict(model="llama3-70b", batch=4, prompt=512, decode=0, budget=60_000_000_000,
@@ -42,4 +50,4 @@ WORKLOADS = {
 def layer_params(m: dict) -> int:
     H, F = m["hidden"], m["ffn"]
     qd, kvd = m["n_heads"] * m["head_dim"], m["n_kv_heads"] * m["head_dim"]
-    return 2 * H + (qd + 2 * kvd) * H + H * qd + 2 * F * H + H * F
+    return 2 * H + (qd + 2 * kvd) * H + H * qd + 2 * F * H + H * F + (2 * m["head_dim"] if m.get("qk_norm") else 0)

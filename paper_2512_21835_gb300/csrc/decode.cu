@@ -102,6 +102,7 @@ struct GemvParams {
     KvView kv;
     RopeFreqs rope;
     int w_host;  // weights are read in place from mapped host memory: no L2 prefetch of them
+    float* qk_raw;  // QK-norm models: query/key rows leave unrotated here ([B][(Hq + 2 Hkv) d])
 };
 
 // rows handled per warp unit, by epilogue
@@ -235,6 +236,12 @@ __device__ __forceinline__ void unit_epilogue(const GemvParams& p, int unit, flo
             if (lane != b || b >= p.B) continue;
             float v0 = acc[0][b] * inv[b], v1 = acc[1][b] * inv[b];
             const int pos = p.positions[b];
+            if (p.qk_raw && h < p.Hq + p.Hkv) {  // normalised and rotated by qk_norm_rope_kernel
+                float* raw = p.qk_raw + (size_t)b * (p.Hq + 2 * p.Hkv) * p.d + (size_t)h * p.d;
+                raw[i] = v0;
+                raw[i + half] = v1;
+                continue;
+            }
             if (h < p.Hq + p.Hkv) {
                 float cf, sf;
                 rope_cos_sin(pos, p.rope.inv_freq[i], &cf, &sf);
@@ -617,14 +624,19 @@ __device__ __forceinline__ void tile_gemv(const GemvParams& p, int tile, int nex
                 const int h = pair / half, i = pair - h * half;
                 float v0 = sm.val[tid] * inv, v1 = sm.val[tid + R / 2] * inv;
                 const int pos = p.positions[0];
-                if (h < p.Hq + p.Hkv) {
+                const bool raw = p.qk_raw && h < p.Hq + p.Hkv;  // normalised and rotated by qk_norm_rope_kernel
+                if (raw) {
+                    p.qk_raw[(size_t)h * p.d + i] = v0;
+                    p.qk_raw[(size_t)h * p.d + i + half] = v1;
+                } else if (h < p.Hq + p.Hkv) {
                     float cf, sf;
                     rope_cos_sin(pos, p.rope.inv_freq[i], &cf, &sf);
                     const float r0 = v0 * cf - v1 * sf, r1 = v1 * cf + v0 * sf;
                     v0 = r0;
                     v1 = r1;
                 }
-                if (h < p.Hq) {
+                if (raw) {
+                } else if (h < p.Hq) {
                     float* q = p.out + (size_t)h * p.d;
                     q[i] = v0;
                     q[i + half] = v1;
@@ -1461,6 +1473,63 @@ cudaError_t launch_run_t(RunParams& rp, cudaStream_t st) {
 }
 
 // ----------------------------------------------------------------------------
+// QK-norm (Qwen3-style layers)
+// ----------------------------------------------------------------------------
+struct QkNormParams {
+    const float* raw;  // [rows][(Hq + 2 Hkv) d] unrotated projections
+    int rows, Hq, Hkv, d, with_v;
+    const uint16_t *g_q, *g_k;  // [d] gains
+    float eps;
+    const int32_t* positions;
+    const int32_t* row_req;
+    float* q_out;  // [rows][Hq d]
+    KvView kv;
+    RopeFreqs rope;
+};
+
+// One block of d/2 threads per (row, head): RMSNorm of the head's d values
+// (gain g_q for query heads, g_k for key heads), the rotation at the row's
+// position, then the QKV epilogue's stores: queries to q_out (fp32), keys to
+// the KV cache (bf16); with_v: value heads are copied to the cache unchanged.
+__global__ void __launch_bounds__(64) qk_norm_rope_kernel(QkNormParams p) {
+    __shared__ float s_ss[2];
+    pdl_trigger();
+    pdl_wait();
+    const int h = blockIdx.x, b = blockIdx.y;
+    const int half = p.d >> 1, i = threadIdx.x;
+    const float* raw = p.raw + (size_t)b * (p.Hq + 2 * p.Hkv) * p.d + (size_t)h * p.d;
+    float v0 = raw[i], v1 = raw[i + half];
+    const int pos = p.positions[b];
+    if (h < p.Hq + p.Hkv) {
+        float ss = warp_sum(fmaf(v0, v0, v1 * v1));
+        if ((i & 31) == 0) s_ss[i >> 5] = ss;
+        __syncthreads();
+        ss = s_ss[0] + (half > 32 ? s_ss[1] : 0.f);
+        const float inv = 1.0f / sqrtf(ss / (float)p.d + p.eps);
+        const uint16_t* g = h < p.Hq ? p.g_q : p.g_k;
+        v0 = v0 * inv * bf2f(g[i]);
+        v1 = v1 * inv * bf2f(g[i + half]);
+        float cf, sf;
+        rope_cos_sin(pos, p.rope.inv_freq[i], &cf, &sf);
+        const float r0 = v0 * cf - v1 * sf, r1 = v1 * cf + v0 * sf;
+        v0 = r0;
+        v1 = r1;
+    }
+    if (h < p.Hq) {
+        float* q = p.q_out + (size_t)b * p.Hq * p.d + (size_t)h * p.d;
+        q[i] = v0;
+        q[i + half] = v1;
+    } else {
+        const int req = p.row_req ? p.row_req[b] : b;
+        const bool is_v = h >= p.Hq + p.Hkv;
+        const int kh = h - p.Hq - (is_v ? p.Hkv : 0);
+        uint16_t* row = reinterpret_cast<uint16_t*>(kv_row(p.kv, req, pos, is_v ? 1 : 0, kh, p.Hkv, p.d));
+        row[i] = f2bf(v0);
+        row[i + half] = f2bf(v1);
+    }
+}
+
+// ----------------------------------------------------------------------------
 // Embedding gather and generator
 // ----------------------------------------------------------------------------
 __global__ void embed_kernel(const uint16_t* E, const int32_t* tokens, int H, int V, float* x) {
@@ -1546,9 +1615,10 @@ __global__ void __launch_bounds__(256) read_stream_kernel(const uint4* src, uint
 // ----------------------------------------------------------------------------
 cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
                             int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
-                            const int32_t* row_req, cudaStream_t st, bool pdl, bool w_host) {
+                            const int32_t* row_req, cudaStream_t st, bool pdl, bool w_host, float* qk_raw) {
     GemvParams p{};
     p.w_host = w_host;
+    p.qk_raw = qk_raw;
     p.in = x;
     p.g = g;
     p.w0 = wqkv;
@@ -1685,6 +1755,28 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
         }
     }
     return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_qk_norm_rope(const float* raw, int rows, int Hq, int Hkv, int d, bool with_v, const uint16_t* g_q,
+                                const uint16_t* g_k, float eps, float theta, const int32_t* positions,
+                                const int32_t* row_req, float* q_out, KvView kv, cudaStream_t st, bool pdl) {
+    if (rows < 1 || (d != 64 && d != 128)) return cudaErrorInvalidValue;
+    QkNormParams p{};
+    p.raw = raw;
+    p.rows = rows;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.d = d;
+    p.with_v = with_v ? 1 : 0;
+    p.g_q = g_q;
+    p.g_k = g_k;
+    p.eps = eps;
+    p.positions = positions;
+    p.row_req = row_req;
+    p.q_out = q_out;
+    p.kv = kv;
+    p.rope = rope_freqs(theta, d);
+    return launch_k(qk_norm_rope_kernel, dim3(Hq + Hkv + (with_v ? Hkv : 0), rows), dim3(d / 2), 0, st, pdl, p);
 }
 
 bool decode_run_supported(int Hq, int Hkv, int d) {

@@ -42,7 +42,16 @@ struct KvView {
 // over the host link); the kernels then skip their L2 prefetch of it.
 cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* wqkv, int B, int H, int Hq, int Hkv,
                             int d, float eps, float theta, const int32_t* positions, float* q_out, KvView kv,
-                            const int32_t* row_req, cudaStream_t st, bool pdl = false, bool w_host = false);
+                            const int32_t* row_req, cudaStream_t st, bool pdl = false, bool w_host = false,
+                            float* qk_raw = nullptr);
+// QK-norm layers (Qwen3): with qk_raw set, launch_qkv_rope leaves the query and
+// key rows unrotated in qk_raw ([B][(Hq + 2 Hkv) d] fp32; values still go to the
+// cache), and launch_qk_norm_rope then applies the per-head RMSNorm (gains g_q,
+// g_k [d]) and the rotation and makes the usual stores.  with_v: the value rows
+// of `raw` are copied to the cache as well (prefill, where raw holds all rows).
+cudaError_t launch_qk_norm_rope(const float* raw, int rows, int Hq, int Hkv, int d, bool with_v, const uint16_t* g_q,
+                                const uint16_t* g_k, float eps, float theta, const int32_t* positions,
+                                const int32_t* row_req, float* q_out, KvView kv, cudaStream_t st, bool pdl = false);
 cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st,
                               bool pdl = false, bool w_host = false);
 cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,

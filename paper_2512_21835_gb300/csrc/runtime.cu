@@ -49,7 +49,7 @@ struct Request {
 
 struct Fixed {  // offsets inside the fixed region
     uint64_t embed, lm_head, g_final, x, q, o, a, z, logits, attn_scratch, lm_scratch;
-    uint64_t tokens, out_tokens, positions, ctx_lens, row_req, page_table, last_rows, dec_pos, run_sync;
+    uint64_t tokens, out_tokens, positions, ctx_lens, row_req, page_table, last_rows, dec_pos, run_sync, qk_raw;
     uint64_t px, py, pq, po, pa;
     uint64_t total;
 };
@@ -63,7 +63,7 @@ int validate_desc(const loip_model_desc* d) {
         return LOIP_ERR_INVALID;
     int G = d->n_heads / d->n_kv_heads;
     if (G != 1 && G != 2 && G != 4 && G != 8) return LOIP_ERR_INVALID;
-    if (!(d->rms_eps > 0) || !(d->rope_theta > 1)) return LOIP_ERR_INVALID;
+    if (!(d->rms_eps > 0) || !(d->rope_theta > 1) || (d->qk_norm != 0 && d->qk_norm != 1)) return LOIP_ERR_INVALID;
     return LOIP_OK;
 }
 
@@ -77,6 +77,13 @@ void layout_of(const loip_model_desc* d, loip_layer_layout_t* o) {
     off = align_up(off + (qd + 2 * kvd) * H * 2);
     o->off_wo = off;
     off = align_up(off + H * qd * 2);
+    o->off_g_q = o->off_g_k = off;
+    if (d->qk_norm) {
+        o->off_g_q = off;
+        off = align_up(off + (uint64_t)d->head_dim * 2);
+        o->off_g_k = off;
+        off = align_up(off + (uint64_t)d->head_dim * 2);
+    }
     o->mha_bytes = off;
     o->off_g_mlp = off;
     off = align_up(off + H * 2);
@@ -132,6 +139,7 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     f.dec_pos = take(B * 4);
     f.page_table = take(B * max_pages * 8);
     f.run_sync = take(4 * (2 + 4 * kMaxRunLayers));
+    f.qk_raw = d->qk_norm ? take(rows * (uint64_t)(d->n_heads + 2 * d->n_kv_heads) * d->head_dim * 4) : 0;
     f.px = take(Mp * H * 4);
     f.py = take(Mp * H * 2);
     f.pq = take(Mp * qd * 4);
@@ -511,9 +519,14 @@ struct loip_ctx {
         const int64_t* pt = fixed_ptr<int64_t>(fx.page_table);
         KvView kv = kv_view(l, pt);
         cudaError_t e;
+        float* qk_raw = desc.qk_norm ? fixed_ptr<float>(fx.qk_raw) : nullptr;
         e = timed(0, s, [&] {
-            return launch_qkv_rope(x, g_attn, wqkv, B, H, Hq, Hkv, d, desc.rms_eps, desc.rope_theta, pos_dev, q, kv,
-                                   nullptr, s, pdl(), host_a);
+            cudaError_t r = launch_qkv_rope(x, g_attn, wqkv, B, H, Hq, Hkv, d, desc.rms_eps, desc.rope_theta, pos_dev,
+                                            q, kv, nullptr, s, pdl(), host_a, qk_raw);
+            if (r == cudaSuccess && qk_raw)
+                r = launch_qk_norm_rope(qk_raw, B, Hq, Hkv, d, false, wa + lay.off_g_q / 2, wa + lay.off_g_k / 2,
+                                        desc.rms_eps, desc.rope_theta, pos_dev, nullptr, q, kv, s, pdl());
+            return r;
         });
         if (e != cudaSuccess) return cuda_fail(e, "qkv kernel");
         chain = true;
@@ -548,10 +561,21 @@ struct loip_ctx {
         KvView kv = kv_view(l, pt);
         cudaError_t e;
         e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, wa + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s); });
-        if (e == cudaSuccess)
+        if (e == cudaSuccess && !desc.qk_norm)
             e = timed(6, s, [&] {
                 return launch_tc_gemm_qkv_rope(py, wa + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos, req,
                                                pq, kv, s);
+            });
+        if (e == cudaSuccess && desc.qk_norm)  // raw projections (GEMM into zeros), then norm + rotation + stores
+            e = timed(6, s, [&] {
+                const int nqkv = (Hq + 2 * Hkv) * d;
+                float* raw = fixed_ptr<float>(fx.qk_raw);
+                cudaError_t r = cudaMemsetAsync(raw, 0, (size_t)Mc * nqkv * 4, s);
+                if (r == cudaSuccess) r = launch_tc_gemm_resid(py, wa + lay.off_wqkv / 2, Mc, nqkv, H, raw, s);
+                if (r == cudaSuccess)
+                    r = launch_qk_norm_rope(raw, Mc, Hq, Hkv, d, true, wa + lay.off_g_q / 2, wa + lay.off_g_k / 2,
+                                            desc.rms_eps, desc.rope_theta, pos, req, pq, kv, s);
+                return r;
             });
         if (e == cudaSuccess)
             e = timed(7, s, [&] {
@@ -615,7 +639,8 @@ struct loip_ctx {
     // Whether a batch-B decode step computes its runs of resident layers with
     // the persistent layer-run kernel.
     bool fuse_runs(int B) const {
-        return B == 1 && cfg.layer_run_kernel && decode_run_supported(Hq, Hkv, d) && cfg.max_ctx <= 64 * 256;
+        return B == 1 && cfg.layer_run_kernel && !desc.qk_norm && decode_run_supported(Hq, Hkv, d) &&
+               cfg.max_ctx <= 64 * 256;
     }
 
     // Runs all layers once (decode or prefill pass) with the streaming ring.
@@ -1178,6 +1203,10 @@ static int write_layer_generated(loip_ctx* c, char* dst, int l, uint64_t seed) {
     gen(y.off_wg, F * H, T(6), 0);
     gen(y.off_wu, F * H, T(7), 0);
     gen(y.off_wd, H * F, T(8), 0);
+    if (c->desc.qk_norm) {
+        gen(y.off_g_q, (uint64_t)c->d, T(9), 1);
+        gen(y.off_g_k, (uint64_t)c->d, T(10), 1);
+    }
     if (e != cudaSuccess) return c->cuda_fail(e, "generator kernel");
     return LOIP_OK;
 }

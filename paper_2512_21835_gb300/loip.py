@@ -29,7 +29,7 @@ class LoipError(RuntimeError):
 class ModelDesc(C.Structure):
     _fields_ = [("n_layers", C.c_int32), ("hidden", C.c_int32), ("n_heads", C.c_int32), ("n_kv_heads", C.c_int32),
                 ("head_dim", C.c_int32), ("ffn", C.c_int32), ("vocab", C.c_int32), ("rms_eps", C.c_float),
-                ("rope_theta", C.c_float)]
+                ("rope_theta", C.c_float), ("qk_norm", C.c_int32)]
 
 
 class Config(C.Structure):
@@ -41,7 +41,7 @@ class Config(C.Structure):
 
 class LayerLayout(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ("off_g_attn", "off_wqkv", "off_wo", "off_g_mlp", "off_wg", "off_wu",
-                                          "off_wd", "l_size", "mha_bytes", "mlp_bytes")]
+                                          "off_wd", "l_size", "mha_bytes", "mlp_bytes", "off_g_q", "off_g_k")]
 
 
 class Plan(C.Structure):
@@ -148,7 +148,7 @@ def _check(rc, ctx=None):
 
 def model_desc(m: dict) -> ModelDesc:
     return ModelDesc(m["n_layers"], m["hidden"], m["n_heads"], m["n_kv_heads"], m["head_dim"], m["ffn"], m["vocab"],
-                     m.get("rms_eps", 1e-5), m.get("rope_theta", 500000.0))
+                     m.get("rms_eps", 1e-5), m.get("rope_theta", 500000.0), int(m.get("qk_norm", 0)))
 
 
 def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 2048, mode: int = MODE_OVERLAP,

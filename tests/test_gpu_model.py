@@ -350,3 +350,44 @@ def test_kv_growth_offloads_blocks_or_layers(torch, L, orc, whole):
         assert masks.count(0) == 2 and masks.count(2) == 1 and masks.count(3) == 3
     assert np.array_equal(np.array(toks), base[0])
     assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
+
+
+TINY_QK = configs.MODELS["tiny-qk"]
+
+
+def test_qk_norm_model_matches_oracle(torch, L, orc):
+    """Qwen3-style layers (per-head RMSNorm of queries and keys before the
+    rotation, query width 512 over hidden 256): tensor-core prefill, then
+    teacher-forced decode, against the oracle."""
+    m = TINY_QK
+    prompt = inputs.token_ids(101, 52, m["vocab"])
+    P = 36
+    ref = _oracle(orc, m, prompt[:P], prompt[P:])
+    cont = [[t] for t in prompt[P:]]
+    toks, hids, plan, _ = _run(L, torch, m, [prompt[:P]], cont, dict(max_batch=1, max_ctx=64), 2)
+    assert plan["n_offloaded"] == 0
+    for i in range(len(toks)):
+        t = P - 1 + i
+        _check_hidden(hids[i][0], ref["hidden"][t])
+        assert int(toks[i][0]) == int(ref["argmax"][t])
+
+
+def test_qk_norm_batched_and_offloaded(torch, L, orc):
+    """QK-norm at batch 2 (the batched GEMV writes the raw rows of both requests)
+    with two of four layers streamed: matches the oracle per request, and is
+    bit-identical to the all-resident run."""
+    m = dict(TINY_QK, n_layers=4)
+    prompts = [inputs.token_ids(111, 21, m["vocab"]), inputs.token_ids(112, 34, m["vocab"])]
+    conts = [inputs.token_ids(113, 5, m["vocab"]), inputs.token_ids(114, 5, m["vocab"])]
+    cont = [[int(conts[0][s]), int(conts[1][s])] for s in range(5)]
+    base = _run(L, torch, m, prompts, cont, dict(max_batch=2, max_ctx=64), 4)
+    got = _run(L, torch, m, prompts, cont, dict(max_batch=2, max_ctx=64, n_slots=1), 2)
+    assert got[2]["n_offloaded"] == 2
+    assert np.array_equal(base[0], got[0])
+    assert np.array_equal(base[1].view(np.uint32), got[1].view(np.uint32))
+    for b in range(2):
+        ref = _oracle(orc, m, prompts[b], conts[b])
+        for i in range(6):
+            t = len(prompts[b]) - 1 + i
+            _check_hidden(base[1][i][b], ref["hidden"][t])
+            assert int(base[0][i][b]) == int(ref["argmax"][t])
