@@ -83,6 +83,10 @@ typedef struct loip_config {
                                    * resident (loip_refine_blocks), and KV growth offloads single
                                    * blocks chosen by Eq. 7 (loip_eq7_choice); 1: whole layers
                                    * only (one more layer offloaded per threshold) */
+    uint64_t host_budget_bytes;   /* pinned host memory for streamed layers (0 = unlimited); layers
+                                   * beyond it live in the SSD tier (ssd_dir) */
+    const char* ssd_dir;          /* directory of the SSD tier's scratch file (caller-owned string,
+                                   * read at create; NULL = /tmp) */
 } loip_config;
 
 typedef struct loip_layer_layout_t {
@@ -125,6 +129,8 @@ typedef struct loip_stats {
     double pool_min_GBps;      /* slowest host-pool blob copy when the pool was qualified */
     double pool_median_GBps;   /* median blob copy rate at qualification */
     uint64_t pool_replaced;    /* blobs moved to fresh host memory because they copied slowly */
+    int32_t n_ssd_layers;      /* streamed layers whose blob lives in the SSD tier */
+    uint64_t ssd_read_bytes;   /* bytes read from the SSD tier since create */
 } loip_stats;
 
 typedef struct loip_ctx loip_ctx;
@@ -281,6 +287,13 @@ int loip_synchronize(loip_ctx* ctx);
  * memory (the pool's allocator) to device memory on the current device.
  * Allocates and frees its own buffers.  *out_Bps in bytes per second. */
 int loip_measure_h2d(uint64_t bytes, int32_t reps, double* out_Bps);
+
+/* SSD tier check (Sec. III-C's storage tier; loip_config.ssd_dir): writes
+ * `bytes` (a multiple of 4096) of a pattern to an unlinked O_DIRECT scratch file
+ * in `dir` (NULL: /tmp) and reads it back through io_uring; *ok = 1 when the
+ * bytes match.  Host only.  LOIP_ERR_STATE when the file or the ring cannot be
+ * set up on this machine. */
+int loip_ssd_roundtrip(const char* dir, uint64_t bytes, int32_t* ok);
 
 /* Host-link throughput as direct-access kernels see it: best of `reps` timed
  * launches of a kernel that streams `bytes` (>= 1 MiB, a multiple of 16) with

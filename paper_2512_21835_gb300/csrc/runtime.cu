@@ -27,6 +27,7 @@
 #include <vector>
 
 #include "../../include/loip.h"
+#include "disktier.h"
 #include "hostpool.h"
 #include "internal.h"
 #include "plan.h"
@@ -182,6 +183,15 @@ struct loip_ctx {
     // host pool: blobs of offloaded layers inside pinned huge-page regions
     std::vector<void*> host_layer;
     std::vector<HostBuf> host_regions;
+    // SSD tier: streamed layers beyond the host budget live in a file (disk_off[l]
+    // >= 0); io_uring reads them one layer ahead, in ring order, into two pinned
+    // staging buffers that the copy stream then moves into the slots
+    DiskTier disk;
+    std::vector<int64_t> disk_off;
+    uint64_t disk_stride = 0;
+    HostBuf stage[2];
+    int stage_layer[2] = {-1, -1};           // layer whose read was queued into the buffer
+    cudaEvent_t stage_done[2] = {nullptr, nullptr};  // last copy out of the buffer
     int32_t* h_stage = nullptr;  // pinned staging for small transfers (last word: layer-run error)
     bool run_launched = false;   // a layer-run kernel has been enqueued (its error word is checked)
     size_t h_stage_ints = 0;
@@ -389,18 +399,92 @@ struct loip_ctx {
         return LOIP_OK;
     }
 
+    // ---- SSD tier -------------------------------------------------------------
+    // Queues the read of disk layer l into staging buffer b once the buffer's
+    // previous copy to a slot has finished (bounded wait).
+    int queue_read(int l, int b) {
+        int rc = wait_event(stage_done[b]);
+        if (rc) return rc;
+        std::string err;
+        if (!disk.submit_read((uint64_t)disk_off[l], stage[b].ptr, disk_stride, b, &err))
+            return fail(LOIP_ERR_CUDA, err);
+        stage_layer[b] = l;
+        st.ssd_read_bytes += disk_stride;
+        return LOIP_OK;
+    }
+    // The staging buffer holding disk layer l, its read complete.
+    int staged_blob(int l, int* b_out) {
+        int b = stage_layer[0] == l ? 0 : stage_layer[1] == l ? 1 : -1;
+        if (b < 0) {  // not read ahead (ring restart): read it now into a buffer no read is queued in
+            b = stage_layer[0] < 0 ? 0 : 1;
+            if (stage_layer[b] >= 0) {
+                std::string err;
+                if (!disk.wait(b, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
+            }
+            int rc = queue_read(l, b);
+            if (rc) return rc;
+        }
+        std::string err;
+        if (!disk.wait(b, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
+        *b_out = b;
+        return LOIP_OK;
+    }
+    // After the copy of disk layer l: queue the read of the next disk layer in
+    // ring order (it overlaps the copies and compute in between).
+    int read_ahead(int l) {
+        const int m = (int)off_order.size();
+        int pos = 0;
+        while (pos < m && off_order[pos] != l) ++pos;
+        for (int k = 1; k <= m; ++k) {
+            const int nl = off_order[(pos + k) % m];
+            if (disk_off[nl] < 0) continue;
+            if (stage_layer[0] == nl || stage_layer[1] == nl) return LOIP_OK;
+            const int b = stage_layer[0] < 0 ? 0 : (stage_layer[1] < 0 ? 1 : -1);
+            return b < 0 ? LOIP_OK : queue_read(nl, b);
+        }
+        return LOIP_OK;
+    }
+    // Writes layer l's blob (in device memory at src) to the SSD tier through
+    // staging buffer 0.
+    int write_disk_blob(int l, const char* src, cudaMemcpyKind kind) {
+        int rc = wait_event(stage_done[0]);
+        if (rc) return rc;
+        if (stage_layer[0] >= 0) {
+            std::string err;
+            if (!disk.wait(0, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
+            stage_layer[0] = -1;
+        }
+        cudaError_t e = cudaMemcpy(stage[0].ptr, src, lay.l_size, kind);
+        if (e != cudaSuccess) return cuda_fail(e, "SSD-tier staging copy");
+        std::string err;
+        if (!disk.write((uint64_t)disk_off[l], stage[0].ptr, disk_stride, &err)) return fail(LOIP_ERR_CUDA, err);
+        return LOIP_OK;
+    }
+
     // ---- streaming ------------------------------------------------------------
     int enqueue_copy(int layer, int slot, cudaStream_t cs) {
         cudaError_t e = cudaStreamWaitEvent(cs, slot_free[slot], 0);
         if (e != cudaSuccess) return cuda_fail(e, "copy wait");
+        const char* src = static_cast<const char*>(host_layer[layer]);
+        int sb = -1;
+        if (disk_off[layer] >= 0) {  // SSD tier: the staged copy of the blob
+            int rc = staged_blob(layer, &sb);
+            if (rc) return rc;
+            src = static_cast<const char*>(stage[sb].ptr);
+        }
         cudaEvent_t e0 = take_event(), e1 = take_event();
         cudaEventRecord(e0, cs);
         // the blocks the layer streams, at their blob offsets
         const uint64_t off0 = (res_mask[layer] & 1) ? lay.mha_bytes : 0;
         const uint64_t off1 = (res_mask[layer] & 2) ? lay.mha_bytes : lay.l_size;
-        e = cudaMemcpyAsync(slot_ptr(slot) + off0, static_cast<const char*>(host_layer[layer]) + off0, off1 - off0,
-                            cudaMemcpyHostToDevice, cs);
+        e = cudaMemcpyAsync(slot_ptr(slot) + off0, src + off0, off1 - off0, cudaMemcpyHostToDevice, cs);
         if (e != cudaSuccess) return cuda_fail(e, "layer copy");
+        if (sb >= 0) {
+            cudaEventRecord(stage_done[sb], cs);
+            stage_layer[sb] = -1;
+            int rc = read_ahead(layer);
+            if (rc) return rc;
+        }
         cudaEventRecord(e1, cs);
         copy_events.emplace_back(e0, e1);
         e = cudaEventRecord(slot_full[slot], cs);
@@ -859,7 +943,10 @@ struct loip_ctx {
     // fresh buffer, keeping the slow memory reserved while retrying so it is not
     // handed back.  At most 3 attempts per blob; the fastest buffer wins.
     int qualify_host_pool() {
-        if (off_order.empty()) return LOIP_OK;
+        std::vector<int> pooled;  // streamed layers with a blob in the host pool (not in the SSD tier)
+        for (int l : off_order)
+            if (host_layer[l]) pooled.push_back(l);
+        if (pooled.empty()) return LOIP_OK;
         cudaEvent_t a = take_event(), b = take_event();
         auto rate = [&](const void* src, double* gbps) -> int {
             cudaEventRecord(a, compute);
@@ -873,16 +960,16 @@ struct loip_ctx {
             return LOIP_OK;
         };
         std::vector<double> r(L, 0.0);
-        for (int l : off_order) {
+        for (int l : pooled) {
             int rc = rate(host_layer[l], &r[l]);
             if (rc) return rc;
         }
         std::vector<double> sorted;
-        for (int l : off_order) sorted.push_back(r[l]);
+        for (int l : pooled) sorted.push_back(r[l]);
         std::sort(sorted.begin(), sorted.end());
         const double median = sorted[sorted.size() / 2];
         std::vector<HostBuf> spare;  // rejected buffers, released after the search
-        for (int l : off_order) {
+        for (int l : pooled) {
             for (int attempt = 0; attempt < 3 && r[l] < 0.9 * median; ++attempt) {
                 HostBuf hb;
                 if (host_buf_alloc(lay.l_size, &hb) != cudaSuccess) break;
@@ -901,7 +988,7 @@ struct loip_ctx {
         }
         for (auto& hb : spare) host_buf_free(&hb);
         double mn = 1e30;
-        for (int l : off_order) mn = std::min(mn, r[l]);
+        for (int l : pooled) mn = std::min(mn, r[l]);
         st.pool_min_GBps = mn;
         st.pool_median_GBps = median;
         event_pool.push_back(a);
@@ -913,7 +1000,7 @@ struct loip_ctx {
     int ensure_host_pool() {
         std::vector<int> need;
         for (int l = 0; l < L; ++l)
-            if (offloaded[l] && !host_layer[l]) need.push_back(l);
+            if (offloaded[l] && !host_layer[l] && disk_off[l] < 0) need.push_back(l);
         if (need.empty()) return LOIP_OK;
         HostBuf b;
         cudaError_t e = host_buf_alloc(need.size() * lay.l_size, &b);
@@ -964,6 +1051,11 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
     if (ctx->compute) cudaStreamSynchronize(ctx->compute);
     if (ctx->copy) cudaStreamSynchronize(ctx->copy);
     for (auto& hb : ctx->host_regions) host_buf_free(&hb);
+    for (int b = 0; b < 2; ++b) {
+        host_buf_free(&ctx->stage[b]);
+        if (ctx->stage_done[b]) cudaEventDestroy(ctx->stage_done[b]);
+    }
+    ctx->disk.close();
     if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
     if (ctx->h_pt) cudaFreeHost(ctx->h_pt);
     for (auto e : ctx->slot_full) cudaEventDestroy(e);
@@ -1110,6 +1202,42 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     c->kv_groups_total = kv_groups;
     c->reqs.resize(cfg.max_batch);
     c->host_layer.assign(c->L, nullptr);
+    // SSD tier: when the host budget cannot hold every streamed layer, the rest
+    // (evenly spaced among them) go to a scratch file; two staging buffers come
+    // out of the host budget
+    c->disk_off.assign(c->L, -1);
+    if (cfg.host_budget_bytes && !c->off_order.empty()) {
+        const uint64_t fit = cfg.host_budget_bytes / c->lay.l_size;
+        const int m = (int)c->off_order.size();
+        if (fit < (uint64_t)m) {
+            if (fit < 2) {
+                g_create_error = "host budget cannot hold the SSD tier's two staging buffers";
+                loip_destroy(c);
+                return LOIP_ERR_INFEASIBLE;
+            }
+            const int nd = m - (int)(fit - 2);
+            c->disk_stride = (c->lay.l_size + DiskTier::kDiskAlign - 1) / DiskTier::kDiskAlign * DiskTier::kDiskAlign;
+            int j = 0;
+            for (int i = 0; i < m; ++i)
+                if ((int64_t)(i + 1) * nd / m > (int64_t)i * nd / m)
+                    c->disk_off[c->off_order[i]] = (int64_t)(j++) * (int64_t)c->disk_stride;
+            std::string err;
+            if (!c->disk.open(cfg.ssd_dir, &err)) {
+                g_create_error = err;
+                loip_destroy(c);
+                return LOIP_ERR_STATE;
+            }
+            for (int b = 0; b < 2; ++b) {
+                if (host_buf_alloc(c->disk_stride, &c->stage[b]) != cudaSuccess ||
+                    cudaEventCreateWithFlags(&c->stage_done[b], cudaEventDisableTiming) != cudaSuccess) {
+                    g_create_error = "SSD-tier staging buffers";
+                    loip_destroy(c);
+                    return LOIP_ERR_OOM;
+                }
+            }
+            c->st.n_ssd_layers = j;
+        }
+    }
 
     cudaError_t e;
     e = cudaStreamCreateWithFlags(&c->compute, cudaStreamNonBlocking);
@@ -1232,7 +1360,14 @@ extern "C" int loip_load_weights_generated(loip_ctx* c, uint64_t seed) {
             char* tmp = c->slot_ptr(0);
             rc = write_layer_generated(c, tmp, l, seed);
             if (rc) return rc;
-            e = cudaMemcpyAsync(c->host_layer[l], tmp, c->lay.l_size, cudaMemcpyDeviceToHost, c->compute);
+            if (c->disk_off[l] >= 0) {  // SSD tier: through a staging buffer to the file
+                rc = c->sync_all();
+                if (rc) return rc;
+                rc = c->write_disk_blob(l, tmp, cudaMemcpyDeviceToHost);
+                if (rc) return rc;
+            } else {
+                e = cudaMemcpyAsync(c->host_layer[l], tmp, c->lay.l_size, cudaMemcpyDeviceToHost, c->compute);
+            }
             if (e == cudaSuccess && c->mha_at[l])  // its resident block (block-level refinement)
                 e = cudaMemcpyAsync(c->mha_at[l], tmp, c->lay.mha_bytes, cudaMemcpyDeviceToDevice, c->compute);
             if (e == cudaSuccess && c->mlp_at[l])
@@ -1259,7 +1394,12 @@ extern "C" int loip_load_layer(loip_ctx* c, int32_t layer, const void* host_blob
     if (rc) return rc;
     cudaError_t e;
     const char* hb = static_cast<const char*>(host_blob);
-    if (c->res_mask[layer] != 3) memcpy(c->host_layer[layer], host_blob, bytes);
+    if (c->res_mask[layer] != 3 && c->disk_off[layer] >= 0) {
+        rc = c->write_disk_blob(layer, hb, cudaMemcpyHostToHost);
+        if (rc) return rc;
+    } else if (c->res_mask[layer] != 3) {
+        memcpy(c->host_layer[layer], host_blob, bytes);
+    }
     e = cudaSuccess;
     if (c->mha_at[layer]) e = cudaMemcpy(c->mha_at[layer], hb, c->lay.mha_bytes, cudaMemcpyHostToDevice);
     if (e == cudaSuccess && c->mlp_at[layer])

@@ -36,7 +36,8 @@ class Config(C.Structure):
     _fields_ = [("device_budget_bytes", C.c_uint64), ("n_slots", C.c_int32), ("page_tokens", C.c_int32),
                 ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("layer_run_kernel", C.c_int32), ("mode", C.c_int32),
                 ("timeout_ms", C.c_uint32), ("hbm_Bps", C.c_double), ("link_Bps", C.c_double),
-                ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32), ("whole_layers", C.c_int32)]
+                ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32), ("whole_layers", C.c_int32),
+                ("host_budget_bytes", C.c_uint64), ("ssd_dir", C.c_char_p)]
 
 
 class LayerLayout(C.Structure):
@@ -57,7 +58,8 @@ class Stats(C.Structure):
                 ("kv_tokens", C.c_uint64), ("kv_bytes", C.c_uint64), ("arena_used", C.c_uint64),
                 ("kernel_ms", C.c_double * 16), ("kernel_launches", C.c_uint64 * 16),
                 ("copy_ms_total", C.c_double), ("copies_total", C.c_uint64),
-                ("pool_min_GBps", C.c_double), ("pool_median_GBps", C.c_double), ("pool_replaced", C.c_uint64)]
+                ("pool_min_GBps", C.c_double), ("pool_median_GBps", C.c_double), ("pool_replaced", C.c_uint64),
+                ("n_ssd_layers", C.c_int32), ("ssd_read_bytes", C.c_uint64)]
 
 
 P, U64, I32, U32, F32, F64, VP = C.c_void_p, C.c_uint64, C.c_int32, C.c_uint32, C.c_float, C.c_double, C.c_void_p
@@ -88,6 +90,7 @@ _SIGS = {
     "loip_set_kernel_timing": (C.c_int, [P, I32]),
     "loip_measure_h2d": (C.c_int, [U64, I32, C.POINTER(C.c_double)]),
     "loip_measure_direct_read": (C.c_int, [U64, I32, C.POINTER(C.c_double)]),
+    "loip_ssd_roundtrip": (C.c_int, [C.c_char_p, U64, C.POINTER(C.c_int32)]),
     "loip_compute_stream": (C.c_void_p, [P]),
     "loip_copy_stream": (C.c_void_p, [P]),
     "loip_k_generate": (C.c_int, [P, U64, U64, U64, U32, I32, P]),
@@ -154,9 +157,10 @@ def model_desc(m: dict) -> ModelDesc:
 def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 2048, mode: int = MODE_OVERLAP,
            timeout_ms: int = 0, hbm_Bps: float = 6.7e12, link_Bps: float = 2.1e11, kv_reserve_bytes: int = 0,
            max_prefill_tokens: int = 512, page_tokens: int = 64, layer_run_kernel: int = 0,
-           whole_layers: int = 0) -> Config:
+           whole_layers: int = 0, host_budget_bytes: int = 0, ssd_dir: str | None = None) -> Config:
     return Config(budget, n_slots, page_tokens, max_batch, max_ctx, layer_run_kernel, mode, timeout_ms, hbm_Bps,
-                  link_Bps, kv_reserve_bytes, max_prefill_tokens, whole_layers)
+                  link_Bps, kv_reserve_bytes, max_prefill_tokens, whole_layers, host_budget_bytes,
+                  ssd_dir.encode() if ssd_dir else None)
 
 
 # ----------------------------------------------------------------------------
@@ -219,6 +223,13 @@ def loip_measure_direct_read(nbytes: int = 1 << 30, reps: int = 5) -> float:
     out = C.c_double()
     _check(lib().loip_measure_direct_read(nbytes, reps, C.byref(out)))
     return out.value
+
+
+def loip_ssd_roundtrip(directory: str | None = None, nbytes: int = 64 << 20) -> bool:
+    """Writes and reads back `nbytes` through the SSD tier's io_uring path; True if they match."""
+    ok = C.c_int32()
+    _check(lib().loip_ssd_roundtrip(directory.encode() if directory else None, nbytes, C.byref(ok)))
+    return bool(ok.value)
 
 
 def loip_fixed_bytes(m: dict, cfg: Config) -> int:

@@ -123,3 +123,12 @@ def test_block_refinement_and_eq7_match_planner_oracle(L, model):
         na, nm = rng.randint(0, Lm), rng.randint(0, Lm)
         need = rng.randint(0, 2 * M)
         assert loip.loip_eq7_choice(m, need, na, nm) == OP.eq7_choice(need, na, nm, A, M)
+
+
+def test_ssd_tier_roundtrip(L, tmp_path):
+    """The SSD tier's O_DIRECT file and raw io_uring reads return what was written
+    (96 MB: three 32 MB requests in flight; and a single 4 KB block)."""
+    assert loip.loip_ssd_roundtrip(str(tmp_path), 96 << 20)
+    assert loip.loip_ssd_roundtrip(str(tmp_path), 4096)
+    with pytest.raises(RuntimeError):
+        loip.loip_ssd_roundtrip(str(tmp_path), 1000)  # not a multiple of the 4 KB block
