@@ -169,7 +169,8 @@ def run_ours(args, rank, world):
     max_prefill = sum(lens) if prefill_mode else min(4096, sum(lens))
     cfg = loip.config(budget=budget, n_slots=w["n_slots"], max_batch=Bsz, max_ctx=max_ctx,
                       max_prefill_tokens=max_prefill, link_Bps=link_peak * 1e9, hbm_Bps=hbm_peak * 1e9,
-                      kv_reserve_bytes=kv_reserve, mode=mode, layer_run_kernel=1 if args.layer_run_kernel else 0)
+                      kv_reserve_bytes=kv_reserve, mode=mode, layer_run_kernel=1 if args.layer_run_kernel else 0,
+                      host_budget_bytes=w.get("host_budget", 0), ssd_dir=os.environ.get("LOIP_SSD_DIR"))
     t0 = time.time()
     ctx = loip.Context(m, cfg)
     plan = ctx.plan()
@@ -344,7 +345,11 @@ def run_ours(args, rank, world):
                           "copy_busy_frac": round((st1["copy_ms_total"] - st0["copy_ms_total"]) / 1e3 / dev_s, 4),
                           "pool_blob_GBps_min_median": [round(st1["pool_min_GBps"], 1),
                                                         round(st1["pool_median_GBps"], 1)],
-                          "pool_blobs_moved": st1["pool_replaced"]},
+                          "pool_blobs_moved": st1["pool_replaced"],
+                          "ssd_layers": st1["n_ssd_layers"],
+                          "ssd_GBps": round((st1["ssd_read_bytes"] - st0["ssd_read_bytes"]) / dev_s / 1e9, 2),
+                          "ssd_ms_per_step": {k: round((st_end[k] - st0[k]) / (steps + 4 + steps), 1)
+                                              for k in ("ssd_wait_ms", "ssd_stage_wait_ms", "ssd_copy_ms")}},
         # tokens up and down, plus the layer run's 4-byte barrier error word when it ran
         "e2e": {"value": round(tokens / e2e_s, 4), "unit": "tokens/s", "h2d_bytes_per_step": 4 * Bsz,
                 "d2h_bytes_per_step": 4 * Bsz + (4 if run_launches else 0)},
@@ -390,7 +395,11 @@ def report_prefill(args, w, m, lay, plan, lens, dev_s, e2e_s, st, st_end, clk, h
         "step_roofline": {"flops_per_step": flops_layer * L, "link_bytes_per_step": link_bytes,
                           "link_peak_GBps": round(link_peak, 1), "roofline_step_ms": round(roof * 1e3, 2),
                           "frac": round(roof / step_s, 4),
-                          "kernel_ms_per_step": {n: round(st["kernel_ms"][i], 3) for i, n in PREFILL_KERNELS.items()}},
+                          "kernel_ms_per_step": {n: round(st["kernel_ms"][i], 3) for i, n in PREFILL_KERNELS.items()},
+                          "copy_GBps_while_copying": round(
+                              st_end["h2d_weight_bytes"] / max(1e-9, st_end["copy_ms_total"] / 1e3) / 1e9, 1),
+                          "pool_blob_GBps_min_median": [round(st_end["pool_min_GBps"], 1),
+                                                        round(st_end["pool_median_GBps"], 1)]},
         "e2e": {"value": round(M * steps * world / e2e_s, 2), "unit": "tokens/s", "h2d_bytes_per_step": 4 * M + 4 * len(lens),
                 "d2h_bytes_per_step": 4 * len(lens)},
         "clocks": clk.summary(),

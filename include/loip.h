@@ -84,7 +84,8 @@ typedef struct loip_config {
                                    * blocks chosen by Eq. 7 (loip_eq7_choice); 1: whole layers
                                    * only (one more layer offloaded per threshold) */
     uint64_t host_budget_bytes;   /* pinned host memory for streamed layers (0 = unlimited); layers
-                                   * beyond it live in the SSD tier (ssd_dir) */
+                                   * beyond it live in the SSD tier (ssd_dir), read back through four
+                                   * staging buffers taken out of this budget */
     const char* ssd_dir;          /* directory of the SSD tier's scratch file (caller-owned string,
                                    * read at create; NULL = /tmp) */
 } loip_config;
@@ -131,6 +132,9 @@ typedef struct loip_stats {
     uint64_t pool_replaced;    /* blobs moved to fresh host memory because they copied slowly */
     int32_t n_ssd_layers;      /* streamed layers whose blob lives in the SSD tier */
     uint64_t ssd_read_bytes;   /* bytes read from the SSD tier since create */
+    double ssd_wait_ms;        /* host time spent waiting for SSD-tier reads to land */
+    double ssd_stage_wait_ms;  /* host time spent waiting for a staging buffer's copy to a slot */
+    double ssd_copy_ms;        /* summed duration of the copies out of staging buffers (events) */
 } loip_stats;
 
 typedef struct loip_ctx loip_ctx;

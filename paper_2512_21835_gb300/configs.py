@@ -42,6 +42,10 @@ WORKLOADS = {
                                n_slots=2),
     "70b-offload-prefill": dict(model="llama3-70b", batch=4, prompt=512, decode=0, budget=60_000_000_000,
                                 n_slots=2),
+    # SSD tier: the host pool holds 26 of the 50 streamed layers (+ 4 staging buffers), the rest
+    # are read back from a scratch file every step
+    "70b-ssd-decode": dict(model="llama3-70b", batch=1, prompt=1024, decode=16, budget=60_000_000_000,
+                           n_slots=2, host_budget=30 * 1_711_308_800),
     "70b-offload-batched": dict(model="llama3-70b", batch=8, ctx_lo=128, ctx_hi=4096, decode=256,
                                 budget=96_000_000_000, n_slots=2),
 }

@@ -93,6 +93,19 @@ cudaError_t host_buf_alloc(size_t bytes, HostBuf* out) {
     return cudaSuccess;
 }
 
+cudaError_t host_buf_alloc_plain(size_t bytes, HostBuf* out) {
+    *out = HostBuf{};
+    if (bytes == 0) return cudaSuccess;
+    void* q = nullptr;
+    cudaError_t e = cudaHostAlloc(&q, bytes, cudaHostAllocPortable | cudaHostAllocMapped);
+    if (e != cudaSuccess) return e;
+    out->ptr = q;
+    out->bytes = bytes;
+    out->mapped = false;
+    map_device(out);
+    return cudaSuccess;
+}
+
 void host_buf_free(HostBuf* b) {
     if (!b->ptr) return;
     if (b->mapped) {

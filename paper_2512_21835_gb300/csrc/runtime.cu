@@ -186,12 +186,13 @@ struct loip_ctx {
     // SSD tier: streamed layers beyond the host budget live in a file (disk_off[l]
     // >= 0); io_uring reads them one layer ahead, in ring order, into two pinned
     // staging buffers that the copy stream then moves into the slots
+    static constexpr int kStages = 4;  // staging buffers: reads run up to three layers ahead
     DiskTier disk;
     std::vector<int64_t> disk_off;
     uint64_t disk_stride = 0;
-    HostBuf stage[2];
-    int stage_layer[2] = {-1, -1};           // layer whose read was queued into the buffer
-    cudaEvent_t stage_done[2] = {nullptr, nullptr};  // last copy out of the buffer
+    HostBuf stage[kStages];
+    int stage_layer[kStages] = {-1, -1, -1, -1};  // layer whose read was queued into the buffer
+    cudaEvent_t stage_done[kStages] = {};         // last copy out of the buffer
     int32_t* h_stage = nullptr;  // pinned staging for small transfers (last word: layer-run error)
     bool run_launched = false;   // a layer-run kernel has been enqueued (its error word is checked)
     size_t h_stage_ints = 0;
@@ -202,7 +203,11 @@ struct loip_ctx {
     cudaEvent_t ev_done = nullptr, ev_step0 = nullptr, ev_step1 = nullptr, ev_reach = nullptr;
     cudaEvent_t ev_stage = nullptr;  // last transfer that read the pinned staging buffers
     bool pos_dirty = true;
-    std::deque<std::pair<cudaEvent_t, cudaEvent_t>> copy_events;
+    struct CopyEv {
+        cudaEvent_t a, b;
+        bool ssd;  // out of an SSD-tier staging buffer
+    };
+    std::deque<CopyEv> copy_events;
     std::vector<cudaEvent_t> event_pool;
     uint64_t copy_seq = 0, compute_seq = 0;
     bool ktiming = false;
@@ -403,8 +408,10 @@ struct loip_ctx {
     // Queues the read of disk layer l into staging buffer b once the buffer's
     // previous copy to a slot has finished (bounded wait).
     int queue_read(int l, int b) {
+        const auto t0 = std::chrono::steady_clock::now();
         int rc = wait_event(stage_done[b]);
         if (rc) return rc;
+        st.ssd_stage_wait_ms += std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
         std::string err;
         if (!disk.submit_read((uint64_t)disk_off[l], stage[b].ptr, disk_stride, b, &err))
             return fail(LOIP_ERR_CUDA, err);
@@ -414,10 +421,14 @@ struct loip_ctx {
     }
     // The staging buffer holding disk layer l, its read complete.
     int staged_blob(int l, int* b_out) {
-        int b = stage_layer[0] == l ? 0 : stage_layer[1] == l ? 1 : -1;
-        if (b < 0) {  // not read ahead (ring restart): read it now into a buffer no read is queued in
-            b = stage_layer[0] < 0 ? 0 : 1;
-            if (stage_layer[b] >= 0) {
+        int b = -1;
+        for (int i = 0; i < kStages && b < 0; ++i)
+            if (stage_layer[i] == l) b = i;
+        if (b < 0) {  // not read ahead (ring restart): read it now, into a free buffer if there is one
+            for (int i = 0; i < kStages && b < 0; ++i)
+                if (stage_layer[i] < 0) b = i;
+            if (b < 0) {
+                b = kStages - 1;
                 std::string err;
                 if (!disk.wait(b, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
             }
@@ -425,22 +436,32 @@ struct loip_ctx {
             if (rc) return rc;
         }
         std::string err;
+        const auto t0 = std::chrono::steady_clock::now();
         if (!disk.wait(b, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
+        st.ssd_wait_ms += std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
         *b_out = b;
         return LOIP_OK;
     }
-    // After the copy of disk layer l: queue the read of the next disk layer in
-    // ring order (it overlaps the copies and compute in between).
+    // After the copy of disk layer l: queue the reads of the next disk layers in
+    // ring order into the free staging buffers (they overlap the copies and
+    // compute in between).
     int read_ahead(int l) {
         const int m = (int)off_order.size();
         int pos = 0;
         while (pos < m && off_order[pos] != l) ++pos;
-        for (int k = 1; k <= m; ++k) {
+        for (int k = 1; k < m; ++k) {
             const int nl = off_order[(pos + k) % m];
             if (disk_off[nl] < 0) continue;
-            if (stage_layer[0] == nl || stage_layer[1] == nl) return LOIP_OK;
-            const int b = stage_layer[0] < 0 ? 0 : (stage_layer[1] < 0 ? 1 : -1);
-            return b < 0 ? LOIP_OK : queue_read(nl, b);
+            bool queued = false;
+            int b = -1;
+            for (int i = 0; i < kStages; ++i) {
+                queued |= stage_layer[i] == nl;
+                if (b < 0 && stage_layer[i] < 0) b = i;
+            }
+            if (queued) continue;
+            if (b < 0) return LOIP_OK;  // every buffer holds a pending read
+            int rc = queue_read(nl, b);
+            if (rc) return rc;
         }
         return LOIP_OK;
     }
@@ -486,7 +507,7 @@ struct loip_ctx {
             if (rc) return rc;
         }
         cudaEventRecord(e1, cs);
-        copy_events.emplace_back(e0, e1);
+        copy_events.push_back({e0, e1, sb >= 0});
         e = cudaEventRecord(slot_full[slot], cs);
         if (e != cudaSuccess) return cuda_fail(e, "slot event");
         st.h2d_weight_bytes += stream_bytes(layer);
@@ -780,15 +801,16 @@ struct loip_ctx {
     void collect_copy_time() {
         double busy = 0;
         while (!copy_events.empty()) {
-            auto pr = copy_events.front();
-            if (cudaEventQuery(pr.second) != cudaSuccess) break;
+            const CopyEv ce = copy_events.front();
+            if (cudaEventQuery(ce.b) != cudaSuccess) break;
             float ms = 0;
-            cudaEventElapsedTime(&ms, pr.first, pr.second);
+            cudaEventElapsedTime(&ms, ce.a, ce.b);
             busy += ms;
             st.copy_ms_total += ms;
             st.copies_total += 1;
-            event_pool.push_back(pr.first);
-            event_pool.push_back(pr.second);
+            if (ce.ssd) st.ssd_copy_ms += ms;
+            event_pool.push_back(ce.a);
+            event_pool.push_back(ce.b);
             copy_events.pop_front();
         }
         st.copy_busy_ms = busy;
@@ -1051,7 +1073,7 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
     if (ctx->compute) cudaStreamSynchronize(ctx->compute);
     if (ctx->copy) cudaStreamSynchronize(ctx->copy);
     for (auto& hb : ctx->host_regions) host_buf_free(&hb);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < loip_ctx::kStages; ++b) {
         host_buf_free(&ctx->stage[b]);
         if (ctx->stage_done[b]) cudaEventDestroy(ctx->stage_done[b]);
     }
@@ -1061,8 +1083,8 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
     for (auto e : ctx->slot_full) cudaEventDestroy(e);
     for (auto e : ctx->slot_free) cudaEventDestroy(e);
     for (auto& pr : ctx->copy_events) {
-        cudaEventDestroy(pr.first);
-        cudaEventDestroy(pr.second);
+        cudaEventDestroy(pr.a);
+        cudaEventDestroy(pr.b);
     }
     for (auto& k : ctx->kernel_events) {
         cudaEventDestroy(k.a);
@@ -1210,12 +1232,12 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
         const uint64_t fit = cfg.host_budget_bytes / c->lay.l_size;
         const int m = (int)c->off_order.size();
         if (fit < (uint64_t)m) {
-            if (fit < 2) {
-                g_create_error = "host budget cannot hold the SSD tier's two staging buffers";
+            if (fit < (uint64_t)loip_ctx::kStages) {
+                g_create_error = "host budget cannot hold the SSD tier's staging buffers";
                 loip_destroy(c);
                 return LOIP_ERR_INFEASIBLE;
             }
-            const int nd = m - (int)(fit - 2);
+            const int nd = m - (int)(fit - loip_ctx::kStages);
             c->disk_stride = (c->lay.l_size + DiskTier::kDiskAlign - 1) / DiskTier::kDiskAlign * DiskTier::kDiskAlign;
             int j = 0;
             for (int i = 0; i < m; ++i)
@@ -1227,8 +1249,8 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
                 loip_destroy(c);
                 return LOIP_ERR_STATE;
             }
-            for (int b = 0; b < 2; ++b) {
-                if (host_buf_alloc(c->disk_stride, &c->stage[b]) != cudaSuccess ||
+            for (int b = 0; b < loip_ctx::kStages; ++b) {
+                if (host_buf_alloc_plain(c->disk_stride, &c->stage[b]) != cudaSuccess ||
                     cudaEventCreateWithFlags(&c->stage_done[b], cudaEventDisableTiming) != cudaSuccess) {
                     g_create_error = "SSD-tier staging buffers";
                     loip_destroy(c);

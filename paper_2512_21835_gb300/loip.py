@@ -59,7 +59,8 @@ class Stats(C.Structure):
                 ("kernel_ms", C.c_double * 16), ("kernel_launches", C.c_uint64 * 16),
                 ("copy_ms_total", C.c_double), ("copies_total", C.c_uint64),
                 ("pool_min_GBps", C.c_double), ("pool_median_GBps", C.c_double), ("pool_replaced", C.c_uint64),
-                ("n_ssd_layers", C.c_int32), ("ssd_read_bytes", C.c_uint64)]
+                ("n_ssd_layers", C.c_int32), ("ssd_read_bytes", C.c_uint64), ("ssd_wait_ms", C.c_double),
+                ("ssd_stage_wait_ms", C.c_double), ("ssd_copy_ms", C.c_double)]
 
 
 P, U64, I32, U32, F32, F64, VP = C.c_void_p, C.c_uint64, C.c_int32, C.c_uint32, C.c_float, C.c_double, C.c_void_p

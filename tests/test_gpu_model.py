@@ -395,18 +395,18 @@ def test_qk_norm_batched_and_offloaded(torch, L, orc):
 
 @pytest.mark.parametrize("mode,K", [(0, 2), (0, 1), (1, 1)])
 def test_ssd_tier_is_bitwise_lossless(torch, L, orc, tmp_path, mode, K):
-    """A host budget of three layer blobs for four streamed layers: two staging
-    buffers and one pooled blob; the other three layers live in the SSD tier and
+    """A host budget of five layer blobs for eight streamed layers: four staging
+    buffers and one pooled blob; the other seven layers live in the SSD tier and
     are read back through io_uring each pass.  Bit-identical to all-resident."""
-    m = TINY6
+    m = dict(TINY, n_layers=10)
     lay = L.loip_layer_layout(m)
     prompts = [inputs.token_ids(121, 20, m["vocab"]), inputs.token_ids(122, 9, m["vocab"])]
     cont = [[int(a), int(b)] for a, b in zip(inputs.token_ids(123, 6, 1024), inputs.token_ids(124, 6, 1024))]
-    base = _run(L, torch, m, prompts, cont, dict(max_batch=2, max_ctx=64), 6)
+    base = _run(L, torch, m, prompts, cont, dict(max_batch=2, max_ctx=64), 10)
     kw = dict(max_batch=2, max_ctx=64, n_slots=K, mode=mode, whole_layers=1,
-              host_budget_bytes=3 * lay["l_size"], ssd_dir=str(tmp_path))
+              host_budget_bytes=5 * lay["l_size"], ssd_dir=str(tmp_path))
     got = _run(L, torch, m, prompts, cont, kw, 2)
-    assert got[2]["n_offloaded"] == 4
-    assert got[3]["n_ssd_layers"] == 3 and got[3]["ssd_read_bytes"] >= 3 * lay["l_size"] * len(cont)
+    assert got[2]["n_offloaded"] == 8
+    assert got[3]["n_ssd_layers"] == 7 and got[3]["ssd_read_bytes"] >= 7 * lay["l_size"] * len(cont)
     assert np.array_equal(base[0], got[0])
     assert np.array_equal(base[1].view(np.uint32), got[1].view(np.uint32))
