@@ -41,8 +41,9 @@ KERNEL_NAMES = ["qkv_rope", "attention", "o_proj", "gate_up", "down", "lm_head"]
 MODES = {"overlap": 0, "naive": 1, "direct": 2}
 RUN_CLASS = 12  # kernel-timing class of the persistent layer-run kernel
 
-# DRAM bytes (read + write) per launch of the gate/up SwiGLU GEMV at batch 1,
-# from an ncu capture of the kernel microbenchmark on the model's shape
+# DRAM bytes (read + write) per launch of the gate/up SwiGLU GEMV at batch 1
+# (the persistent kernel at the 70B shape, the block-tile kernel at 8B), from an
+# ncu capture of the kernel microbenchmark on the model's shape
 # (profiles/gemv_traffic.md has the commands and figures).  They describe the
 # kernel source they were taken on: when the decode kernels' source no longer
 # has this hash the figure is reported as null.
