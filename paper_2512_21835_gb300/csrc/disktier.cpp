@@ -197,11 +197,13 @@ bool DiskTier::submit_read(uint64_t off, void* buf, uint64_t bytes, int tag, std
 
 bool DiskTier::wait(int tag, uint32_t timeout_ms, std::string* err) {
     const uint64_t deadline = now_ms() + timeout_ms;
+    timed_out_ = false;
     while (pending_[tag] > 0) {
         if (!reap(err) && failed_[tag]) return false;
         if (pending_[tag] == 0) break;
         if (now_ms() > deadline) {
             *err = "SSD-tier read did not complete in time";
+            timed_out_ = true;
             return false;
         }
         struct timespec ts = {0, 100000};  // the wait is bounded: poll the completion ring

@@ -26,6 +26,8 @@ class DiskTier {
     // waits until every read queued under `tag` has completed; false on an I/O
     // error or when timeout_ms passes (then *err says which)
     bool wait(int tag, uint32_t timeout_ms, std::string* err);
+    // whether the last failed wait() ran out of time (else it saw an I/O error)
+    bool timed_out() const { return timed_out_; }
 
    private:
     bool reap(std::string* err);  // drains the completion ring
@@ -41,6 +43,7 @@ class DiskTier {
     static constexpr int kTags = 8;
     int pending_[kTags] = {};
     bool failed_[kTags] = {};
+    bool timed_out_ = false;
 };
 
 }  // namespace loip

@@ -407,6 +407,9 @@ struct loip_ctx {
     // ---- SSD tier -------------------------------------------------------------
     // Queues the read of disk layer l into staging buffer b once the buffer's
     // previous copy to a slot has finished (bounded wait).
+    // a failed SSD-tier wait: out of time, or an I/O error
+    int disk_fail(const std::string& err) { return fail(disk.timed_out() ? LOIP_ERR_TIMEOUT : LOIP_ERR_STATE, err); }
+
     int queue_read(int l, int b) {
         const auto t0 = std::chrono::steady_clock::now();
         int rc = wait_event(stage_done[b]);
@@ -414,7 +417,7 @@ struct loip_ctx {
         st.ssd_stage_wait_ms += std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
         std::string err;
         if (!disk.submit_read((uint64_t)disk_off[l], stage[b].ptr, disk_stride, b, &err))
-            return fail(LOIP_ERR_CUDA, err);
+            return fail(LOIP_ERR_STATE, err);
         stage_layer[b] = l;
         st.ssd_read_bytes += disk_stride;
         return LOIP_OK;
@@ -430,14 +433,14 @@ struct loip_ctx {
             if (b < 0) {
                 b = kStages - 1;
                 std::string err;
-                if (!disk.wait(b, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
+                if (!disk.wait(b, cfg.timeout_ms, &err)) return disk_fail(err);
             }
             int rc = queue_read(l, b);
             if (rc) return rc;
         }
         std::string err;
         const auto t0 = std::chrono::steady_clock::now();
-        if (!disk.wait(b, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
+        if (!disk.wait(b, cfg.timeout_ms, &err)) return disk_fail(err);
         st.ssd_wait_ms += std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
         *b_out = b;
         return LOIP_OK;
@@ -472,13 +475,13 @@ struct loip_ctx {
         if (rc) return rc;
         if (stage_layer[0] >= 0) {
             std::string err;
-            if (!disk.wait(0, cfg.timeout_ms, &err)) return fail(LOIP_ERR_TIMEOUT, err);
+            if (!disk.wait(0, cfg.timeout_ms, &err)) return disk_fail(err);
             stage_layer[0] = -1;
         }
         cudaError_t e = cudaMemcpy(stage[0].ptr, src, lay.l_size, kind);
         if (e != cudaSuccess) return cuda_fail(e, "SSD-tier staging copy");
         std::string err;
-        if (!disk.write((uint64_t)disk_off[l], stage[0].ptr, disk_stride, &err)) return fail(LOIP_ERR_CUDA, err);
+        if (!disk.write((uint64_t)disk_off[l], stage[0].ptr, disk_stride, &err)) return fail(LOIP_ERR_STATE, err);
         return LOIP_OK;
     }
 
@@ -1225,8 +1228,8 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     c->reqs.resize(cfg.max_batch);
     c->host_layer.assign(c->L, nullptr);
     // SSD tier: when the host budget cannot hold every streamed layer, the rest
-    // (evenly spaced among them) go to a scratch file; two staging buffers come
-    // out of the host budget
+    // (evenly spaced among them) go to a scratch file; kStages staging buffers
+    // come out of the host budget
     c->disk_off.assign(c->L, -1);
     if (cfg.host_budget_bytes && !c->off_order.empty()) {
         const uint64_t fit = cfg.host_budget_bytes / c->lay.l_size;
