@@ -820,8 +820,12 @@ struct AttnParams {
     int* counters;
     void* o;         // [B, Hq*d] fp32 or bf16
     int o_bf16;
-    int split;
+    int split;  // kAttnSingle, kAttnSplit or kAttnWide
 };
+// single: one 64-thread block per (row, kv head) over every page; split: one
+// 64-thread block per page, partial states in global scratch, combined by the
+// last block to finish; wide: split with a 256-thread block per page
+enum { kAttnSingle = 0, kAttnSplit = 1, kAttnWide = 2 };
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
@@ -868,7 +872,7 @@ __device__ __forceinline__ void attn_group(const AttnParams& p, int row, int kvh
     const int P = p.kv.page_tokens;  // 64
     const int npages = (ctx + P - 1) / P;
     int pg0, pg1;
-    if (p.split) {
+    if (p.split == kAttnSplit) {
         pg0 = chunk;
         pg1 = pg0 + 1;
         if (pg0 >= npages) return;
@@ -1004,7 +1008,7 @@ __device__ __forceinline__ void attn_group(const AttnParams& p, int row, int kvh
             float c1 = (m1 == -INFINITY) ? 0.f : expf(m1 - mn);
             float lt = l[g] * c0 + l1 * c1;
             const int h = kvh * G + g;
-            if (p.split) {
+            if (p.split == kAttnSplit) {
                 float* part = p.scratch + (((size_t)row * p.Hq + h) * p.max_chunks + chunk) * (D + 2);
 #pragma unroll
                 for (int c = 0; c < DPL; ++c) part[lane * DPL + c] = o[g][c] * c0 + sm.s_o[g][lane * DPL + c] * c1;
@@ -1026,7 +1030,7 @@ __device__ __forceinline__ void attn_group(const AttnParams& p, int row, int kvh
             }
         }
     }
-    if (!p.split) return;
+    if (p.split != kAttnSplit) return;
     // The last group of this (row, kv head) to finish combines every page's
     // state: exp-weighted sum of the partial outputs over the summed weights.
     __threadfence();
@@ -1116,6 +1120,230 @@ template <int G, int D>
 cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st, bool pdl) {
     dim3 grid(p.split ? p.max_chunks : 1, p.Hkv, p.B);
     return launch_k(attn_kernel<G, D>, grid, dim3(64), 0, st, pdl, p);
+}
+
+// ----------------------------------------------------------------------------
+// Split-K attention, one 256-thread block per (page, kv head, request row).
+// The 64-thread groups above leave one or two warps per SM to hide every
+// shared-memory and shuffle latency of a page; here eight warps share it:
+//   load    the page's keys (16-byte chunks rotated by row) and values with
+//           asynchronous copies, eight per thread, and the G query rows;
+//   scores  thread (position, dim quarter) forms G partial dot products, the
+//           quarters are summed in shared memory;
+//   softmax warp g takes query head g over the page's positions: page max m,
+//           weights exp(s - m), their sum l;
+//   values  thread (dim pair, head) accumulates the weighted value rows in
+//           position order.
+// The page's unnormalised state (o, m, l) goes to scratch; the last block of
+// the (row, kv head) to arrive (completion ticket) combines every page's state
+// with the usual softmax merge: weights exp(m_c - max m) / sum, outputs summed in
+// page order, sixteen pages' loads in flight per thread.
+template <int G, int D>
+struct AttnPageSmem {
+    alignas(16) uint16_t sK[64 * D];
+    alignas(16) uint16_t sV[64 * D];
+    alignas(16) float sq[G][D];
+    float sc[4][G][64];  // partial scores per dim quarter
+    float sp[G][64];     // exp(s - m) of the page's positions
+    int last;
+};
+
+template <int G, int D>
+__global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
+    constexpr int NT = 256, CH = D / 8, P = 64;
+    constexpr int PAIRS = D / 2, GS = NT / PAIRS, NG = (G + GS - 1) / GS;
+    static_assert(G * kMaxChunks * sizeof(float) <= sizeof(uint16_t) * 64 * D, "combine weights fit a stage");
+    __shared__ AttnPageSmem<G, D> sm;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int chunk = blockIdx.x, kvh = blockIdx.y, row = blockIdx.z;
+    pdl_trigger();
+    pdl_wait();
+    const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
+    const int npages = (ctx + P - 1) / P;
+    if (chunk >= npages) return;
+    const int req = p.row_req ? p.row_req[row] : row;
+    const int nvalid = min(P, ctx - chunk * P);
+    {
+        const char* page = p.kv.base + p.kv.page_offsets[(int64_t)req * p.kv.max_pages + chunk] +
+                           (uint64_t)p.kv.layer * p.kv.layer_page_bytes;
+        const uint16_t* Kh = reinterpret_cast<const uint16_t*>(page) + (size_t)kvh * P * D;
+        const uint16_t* Vh = reinterpret_cast<const uint16_t*>(page) + ((size_t)p.Hkv + kvh) * P * D;
+        for (int i = tid; i < nvalid * CH; i += NT) {
+            const int t = i / CH, c = i - t * CH;
+            cp_async16(&sm.sK[(t * CH + ((c + t) & (CH - 1))) * 8], Kh + (size_t)t * D + c * 8);
+            cp_async16(&sm.sV[(t * CH + c) * 8], Vh + (size_t)t * D + c * 8);
+        }
+        const float* qs = p.q + (size_t)row * p.Hq * D + (size_t)kvh * G * D;
+        for (int i = tid; i < G * D / 4; i += NT)
+            reinterpret_cast<float4*>(&sm.sq[0][0])[i] = ld_act4<false>(qs + 4 * i);
+        cp_async_wait_all();
+        __syncthreads();
+    }
+    {  // scores: a warp holds 32 consecutive positions of one dim quarter
+        const int pos = tid & 63, dq = tid >> 6;
+        float sc[G];
+#pragma unroll
+        for (int g = 0; g < G; ++g) sc[g] = 0.f;
+        if (pos < nvalid) {
+#pragma unroll
+            for (int u = 0; u < CH / 4; ++u) {
+                const int c = dq * (CH / 4) + u;
+                const uint4 kk = *reinterpret_cast<const uint4*>(&sm.sK[(pos * CH + ((c + pos) & (CH - 1))) * 8]);
+                const float kf[8] = {bf_lo(kk.x), bf_hi(kk.x), bf_lo(kk.y), bf_hi(kk.y),
+                                     bf_lo(kk.z), bf_hi(kk.z), bf_lo(kk.w), bf_hi(kk.w)};
+#pragma unroll
+                for (int g = 0; g < G; ++g) {
+                    const float4 qa = *reinterpret_cast<const float4*>(&sm.sq[g][c * 8]);
+                    const float4 qb = *reinterpret_cast<const float4*>(&sm.sq[g][c * 8 + 4]);
+                    float a = sc[g];
+                    a = fmaf(qa.x, kf[0], a);
+                    a = fmaf(qa.y, kf[1], a);
+                    a = fmaf(qa.z, kf[2], a);
+                    a = fmaf(qa.w, kf[3], a);
+                    a = fmaf(qb.x, kf[4], a);
+                    a = fmaf(qb.y, kf[5], a);
+                    a = fmaf(qb.z, kf[6], a);
+                    a = fmaf(qb.w, kf[7], a);
+                    sc[g] = a;
+                }
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < G; ++g) sm.sc[dq][g][pos] = sc[g];
+    }
+    __syncthreads();
+    float m_pg = 0.f, l_pg = 0.f;  // this warp's head (warp < G)
+    if (warp < G) {
+        const int g = warp;
+        float s[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int t = lane + 32 * h;
+            s[h] = t < nvalid ? (((sm.sc[0][g][t] + sm.sc[1][g][t]) + sm.sc[2][g][t]) + sm.sc[3][g][t]) * p.scale
+                              : -INFINITY;
+        }
+        m_pg = warp_max(fmaxf(s[0], s[1]));  // finite: the page holds at least one position
+        float lsum = 0.f;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const float e = lane + 32 * h < nvalid ? expf(s[h] - m_pg) : 0.f;
+            sm.sp[g][lane + 32 * h] = e;
+            lsum += e;
+        }
+        l_pg = warp_sum(lsum);
+    }
+    __syncthreads();
+    const int dp = tid % PAIRS, g0 = tid / PAIRS;
+    float acc[NG][2];
+#pragma unroll
+    for (int k = 0; k < NG; ++k) acc[k][0] = acc[k][1] = 0.f;
+    for (int t = 0; t < nvalid; ++t) {
+        const uint32_t vv = *reinterpret_cast<const uint32_t*>(&sm.sV[t * D + 2 * dp]);
+        const float v0 = bf_lo(vv), v1 = bf_hi(vv);
+#pragma unroll
+        for (int k = 0; k < NG; ++k) {
+            const int g = g0 + k * GS;
+            if (g < G) {
+                const float pr = sm.sp[g][t];
+                acc[k][0] = fmaf(pr, v0, acc[k][0]);
+                acc[k][1] = fmaf(pr, v1, acc[k][1]);
+            }
+        }
+    }
+    const size_t hstride = (size_t)p.max_chunks * (D + 2);
+    float* base = p.scratch + ((size_t)row * p.Hq + (size_t)kvh * G) * hstride;
+#pragma unroll
+    for (int k = 0; k < NG; ++k) {
+        const int g = g0 + k * GS;
+        if (g < G)
+            *reinterpret_cast<float2*>(base + g * hstride + (size_t)chunk * (D + 2) + 2 * dp) =
+                make_float2(acc[k][0], acc[k][1]);
+    }
+    if (warp < G && lane == 0) {
+        float* part = base + warp * hstride + (size_t)chunk * (D + 2);
+        part[D] = m_pg;
+        part[D + 1] = l_pg;
+    }
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+        int* cnt = p.counters + (size_t)row * p.Hq + kvh;
+        const int ticket = atomicAdd(cnt, 1);
+        sm.last = ticket == npages - 1;
+        if (sm.last) atomicExch(cnt, 0);  // every page has arrived: reset for the next launch
+    }
+    __syncthreads();
+    if (!sm.last) return;
+    __threadfence();
+    // the stages are dead: page weights and denominators reuse them
+    float(*s_w)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sm.sK[0]);
+    float(*s_l)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sm.sV[0]);
+    for (int i = tid; i < G * npages; i += NT) {
+        const int g = i / npages, c = i - g * npages;
+        const float* pc = base + g * hstride + (size_t)c * (D + 2);
+        s_w[g][c] = __ldcg(pc + D);
+        s_l[g][c] = __ldcg(pc + D + 1);
+    }
+    __syncthreads();
+    if (warp < G) {
+        const int g = warp;
+        float mx = -INFINITY;
+        for (int c = lane; c < npages; c += 32) mx = fmaxf(mx, s_w[g][c]);
+        mx = warp_max(mx);
+        float lsum = 0.f;
+        for (int c = lane; c < npages; c += 32) {
+            const float w = expf(s_w[g][c] - mx);
+            s_w[g][c] = w;
+            lsum = fmaf(s_l[g][c], w, lsum);
+        }
+        lsum = warp_sum(lsum);
+        const float inv = 1.0f / lsum;
+        for (int c = lane; c < npages; c += 32) s_w[g][c] *= inv;
+    }
+    __syncthreads();
+    constexpr int NOUT = (G * D + NT - 1) / NT, PB = 16;
+    float o[NOUT];
+#pragma unroll
+    for (int k = 0; k < NOUT; ++k) o[k] = 0.f;
+    for (int c0 = 0; c0 < npages; c0 += PB) {
+        float v[PB][NOUT];
+#pragma unroll
+        for (int u = 0; u < PB; ++u)
+#pragma unroll
+            for (int k = 0; k < NOUT; ++k) {
+                const int e = tid + NT * k, g = e / D, j = e - g * D;
+                v[u][k] = (e < G * D && c0 + u < npages) ? __ldcg(base + g * hstride + (size_t)(c0 + u) * (D + 2) + j)
+                                                          : 0.f;
+            }
+#pragma unroll
+        for (int u = 0; u < PB; ++u)
+#pragma unroll
+            for (int k = 0; k < NOUT; ++k) {
+                const int e = tid + NT * k;
+                if (e < G * D && c0 + u < npages) o[k] = fmaf(v[u][k], s_w[e / D][c0 + u], o[k]);
+            }
+    }
+#pragma unroll
+    for (int k = 0; k < NOUT; ++k) {
+        const int e = tid + NT * k;
+        if (e < G * D) {
+            const size_t idx = (size_t)row * p.Hq * D + (size_t)kvh * G * D + e;
+            if (p.o_bf16)
+                reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(o[k]);
+            else
+                reinterpret_cast<float*>(p.o)[idx] = o[k];
+        }
+    }
+}
+
+template <int G, int D>
+cudaError_t launch_attn_page_t(AttnParams& p, cudaStream_t st, bool pdl) {
+    return launch_k(attn_page_kernel<G, D>, dim3(p.max_chunks, p.Hkv, p.B), dim3(256), 0, st, pdl, p);
+}
+
+template <int G, int D>
+cudaError_t launch_attn_any(AttnParams& p, cudaStream_t st, bool pdl) {
+    return p.split == kAttnWide ? launch_attn_page_t<G, D>(p, st, pdl) : launch_attn_t<G, D>(p, st, pdl);
 }
 
 // ----------------------------------------------------------------------------
@@ -1370,7 +1598,7 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParam
         a.scratch = rp.scratch;
         a.counters = rp.counters;
         a.o = rp.o;
-        a.split = 1;
+        a.split = kAttnSplit;
         s_ap = a;
     }
     __syncthreads();
@@ -1723,7 +1951,8 @@ int* attention_counters(float* scratch, int B, int Hq, int d, int max_ctx, int p
 
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
-                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl, int scratch_rows) {
+                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl, int scratch_rows,
+                             bool wide) {
     AttnParams p{};
     p.q = q;
     p.kv = kv;
@@ -1741,21 +1970,22 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
     p.counters = split ? attention_counters(scratch, scratch_rows, Hq, d, max_ctx, kv.page_tokens) : nullptr;
     p.o = o;
     p.o_bf16 = o_bf16 ? 1 : 0;
-    p.split = split ? 1 : 0;
+    p.split = split ? kAttnSplit : kAttnSingle;
+    if (split && wide) p.split = kAttnWide;
     const int G = Hq / Hkv;
     if (d == 128) {
         switch (G) {
-            case 1: return launch_attn_t<1, 128>(p, st, pdl);
-            case 2: return launch_attn_t<2, 128>(p, st, pdl);
-            case 4: return launch_attn_t<4, 128>(p, st, pdl);
-            case 8: return launch_attn_t<8, 128>(p, st, pdl);
+            case 1: return launch_attn_any<1, 128>(p, st, pdl);
+            case 2: return launch_attn_any<2, 128>(p, st, pdl);
+            case 4: return launch_attn_any<4, 128>(p, st, pdl);
+            case 8: return launch_attn_any<8, 128>(p, st, pdl);
         }
     } else if (d == 64) {
         switch (G) {
-            case 1: return launch_attn_t<1, 64>(p, st, pdl);
-            case 2: return launch_attn_t<2, 64>(p, st, pdl);
-            case 4: return launch_attn_t<4, 64>(p, st, pdl);
-            case 8: return launch_attn_t<8, 64>(p, st, pdl);
+            case 1: return launch_attn_any<1, 64>(p, st, pdl);
+            case 2: return launch_attn_any<2, 64>(p, st, pdl);
+            case 4: return launch_attn_any<4, 64>(p, st, pdl);
+            case 8: return launch_attn_any<8, 64>(p, st, pdl);
         }
     }
     return cudaErrorInvalidValue;

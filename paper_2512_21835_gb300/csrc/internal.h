@@ -74,11 +74,12 @@ size_t lm_head_scratch_bytes(int B, int V);
 // over all pages.  o_bf16: write o as bf16 (prefill) instead of fp32.
 // scratch_rows: the batch the scratch was sized for (attention_scratch_floats);
 // the completion counters sit after that many rows of partial states, so the
-// same scratch serves every batch up to it (0 = B).
+// same scratch serves every batch up to it (0 = B).  wide: split mode with a
+// 256-thread block per page (same scratch layout and counters).
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
                              float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl = false,
-                             int scratch_rows = 0);
+                             int scratch_rows = 0, bool wide = false);
 size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens);
 // Split attention keeps one int completion counter per (row, head) after the
 // partial states; they must be zero before a launch and every launch leaves

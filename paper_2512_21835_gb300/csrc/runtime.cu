@@ -640,7 +640,7 @@ struct loip_ctx {
         chain = true;
         e = timed(1, s, [&] {
             return launch_attention(q, kv, nullptr, pos_dev, nullptr, B, Hq, Hkv, d, cfg.max_ctx, true,
-                                    fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl(), cfg.max_batch);
+                                    fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl(), cfg.max_batch, true);
         });
         if (e != cudaSuccess) return cuda_fail(e, "attention kernel");
         e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl(), host_a); });
@@ -1890,7 +1890,7 @@ extern "C" int loip_k_attention(const float* q, const void* kv_base, const int64
                                     (size_t)B * Hq * sizeof(int), (cudaStream_t)stream);
     if (e != cudaSuccess) return LOIP_ERR_CUDA;
     return cerr(launch_attention(q, kv, ctx_lens, nullptr, nullptr, B, Hq, Hkv, d, max_ctx, true, scratch, o, false,
-                                 (cudaStream_t)stream));
+                                 (cudaStream_t)stream, false, 0, true));
 }
 
 extern "C" int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x,

@@ -92,12 +92,16 @@ def _paged_cache(torch, n_pages, Hkv, P, d, seed):
     return buf, order, layer_page_bytes
 
 
+# max_ctx 256: one cluster of 4 blocks per (request, kv head); 1088: 16 blocks
+# of up to two pages each, some left without a page; 2112 (33 pages): split-K
+# blocks with the last-block combine
+@pytest.mark.parametrize("max_ctx,ctx_list", [(256, (1, 70, 200, 64)), (1088, (1, 700, 1088, 129)),
+                                              (2112, (1, 2112, 999, 64))])
 @pytest.mark.parametrize("Hq,Hkv,d", [(8, 2, 128), (4, 2, 64), (32, 8, 128), (64, 8, 128)])
-def test_attention_parity(torch, L, orc, Hq, Hkv, d):
+def test_attention_parity(torch, L, orc, Hq, Hkv, d, max_ctx, ctx_list):
     P = 64
-    ctx = np.array([1, 70, 200, 64], dtype=np.int32)
+    ctx = np.array(ctx_list, dtype=np.int32)
     B = len(ctx)
-    max_ctx = 256
     max_pages = max_ctx // P
     n_pages = B * max_pages
     buf, order, lpb = _paged_cache(torch, n_pages, Hkv, P, d, 3)

@@ -214,9 +214,10 @@ RUN_CLASS = 12  # kernel-timing class of the persistent layer-run kernel
 @pytest.mark.parametrize("resident,K,mode", [(6, 2, 0), (3, 2, 0), (1, 1, 0), (2, 2, 2)])
 def test_layer_run_kernel_matches_per_op_kernels(torch, L, orc, resident, K, mode):
     """Batch-1 decode through the persistent layer-run kernel (runs of resident
-    layers in one launch) equals the per-operation kernels bit for bit: at this
-    shape both use the block-tile GEMV for every projection and the same
-    attention groups."""
+    layers in one launch) matches the per-operation kernels: at this shape both
+    use the block-tile GEMV for every projection; attention sums the same terms
+    in a different order (64-thread page groups against 256-thread page blocks),
+    so tokens agree exactly and the final hidden states to rounding."""
     m = TINY6
     prompt = inputs.token_ids(61, 70, m["vocab"])
     cont = [[int(t)] for t in inputs.token_ids(62, 10, m["vocab"])]
@@ -226,7 +227,7 @@ def test_layer_run_kernel_matches_per_op_kernels(torch, L, orc, resident, K, mod
     assert fused[2]["kernel_launches"][RUN_CLASS] > 0
     assert per_op[2]["kernel_launches"][RUN_CLASS] == 0
     assert np.array_equal(fused[0], per_op[0])
-    assert np.array_equal(fused[1].view(np.uint32), per_op[1].view(np.uint32))
+    assert np.max(np.abs(fused[1] - per_op[1])) <= 1e-4
 
 
 def test_layer_run_kernel_matches_oracle_llama3_heads(torch, L, orc):
