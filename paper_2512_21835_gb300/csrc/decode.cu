@@ -736,14 +736,10 @@ template <int EPI>
 cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, bool pdl, int* nblocks_out = nullptr) {
     // Batch 1: matrices with few rows (QKV, O-proj, down) keep too few units per
     // warp for the persistent kernel to ramp up; the block-tile kernel issues a
-    // whole tile at once.  Row-rich ones (LM head, large gate/up) stream better
-    // persistent.  A mid-size gate/up (<= 32768 rows) whose K splits evenly over
-    // the tile's warps also goes to the tile kernel: its many short blocks let
-    // the next kernel of the chain start early, which outweighs its lower
-    // bandwidth alone.
+    // whole tile at once.  Row-rich ones (gate/up, LM head) stream better
+    // persistent.
     const int rows = (EPI == EPI_SWIGLU) ? 2 * p.n_units : p.N;
-    const bool even_k = ((p.K + 255) / 256) % kTileWarps == 0;
-    if (p.B == 1 && (rows <= 16384 || (EPI == EPI_SWIGLU && rows <= 32768 && even_k))) {
+    if (p.B == 1 && rows <= 16384) {
         const int per_tile = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? kTileRows / 2 : kTileRows;
         const int units = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? p.n_units : p.N;
         const int tiles = (units + per_tile - 1) / per_tile;
