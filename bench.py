@@ -42,13 +42,13 @@ MODES = {"overlap": 0, "naive": 1, "direct": 2}
 RUN_CLASS = 12  # kernel-timing class of the persistent layer-run kernel
 
 # DRAM bytes (read + write) per launch of the gate/up SwiGLU GEMV at batch 1
-# (the persistent kernel at the 70B shape, the block-tile kernel at 8B), from an
+# (the persistent kernel, at the 70B and the 8B shape), from an
 # ncu capture of the kernel microbenchmark on the model's shape
 # (profiles/gemv_traffic.md has the commands and figures).  They describe the
 # kernel source they were taken on: when the decode kernels' source no longer
 # has this hash the figure is reported as null.
-GATE_UP_TRAFFIC = {"llama3-70b": 939_863_552, "llama3-8b": 235_085_056}
-GATE_UP_TRAFFIC_SRC = "c05452902abd6c74c355fd0d99e782aa1713c71169d911d60545dfe374b02438"
+GATE_UP_TRAFFIC = {"llama3-70b": 940_226_304, "llama3-8b": 235_006_464}
+GATE_UP_TRAFFIC_SRC = "93c9b4e842ff028457e9b13ed80a702364b1842b216d0fec7ed0b90456b59037"
 
 
 def gate_up_traffic(model, batch):

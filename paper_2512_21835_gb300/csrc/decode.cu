@@ -103,6 +103,8 @@ struct GemvParams {
     RopeFreqs rope;
     int w_host;  // weights are read in place from mapped host memory: no L2 prefetch of them
     float* qk_raw;  // QK-norm models: query/key rows leave unrotated here ([B][(Hq + 2 Hkv) d])
+    int pf_stride;  // block-tile kernel, > 0: before its dependency wait, block b pulls tiles
+                    // b + pf_stride, b + 2 pf_stride, ... (the later waves) into L2
 };
 
 // rows handled per warp unit, by epilogue
@@ -685,12 +687,30 @@ __device__ __forceinline__ void tile_gemv(const GemvParams& p, int tile, int nex
     __syncthreads();  // the shared partials are reused by the block's next tile
 }
 
+// L2 prefetch of the weight rows of one tile (lanes 0..7 of the calling warp),
+// in pieces of at most 32 KB.
+template <int EPI>
+__device__ __forceinline__ void prefetch_tile(const GemvParams& p, int tile, int lane) {
+    if (lane < kTileRows) {
+        bool v;
+        const uint16_t* r = tile_row<EPI>(p, tile, lane, v);
+        if (v) {
+            const uint32_t bytes = (uint32_t)p.K * 2u;  // a multiple of 16 (K % 8 == 0)
+            for (uint32_t off = 0; off < bytes; off += 32768u)
+                prefetch_l2(reinterpret_cast<const char*>(r) + off, min(32768u, bytes - off));
+        }
+    }
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(kTileWarps * 32, 2) gemv_tile_kernel(GemvParams p) {
     __shared__ TileShared sm;
     pdl_trigger();
     uint4 wa[kTileRows];
     tile_first_load<EPI>(p, blockIdx.x, wa);  // weights do not depend on the previous kernel
+    if (p.pf_stride > 0 && threadIdx.x < 32)
+        for (int t = blockIdx.x + p.pf_stride; t < (int)gridDim.x; t += p.pf_stride)
+            prefetch_tile<EPI>(p, t, threadIdx.x);
     pdl_wait();
     tile_gemv<EPI, false>(p, blockIdx.x, -1, wa, sm);
 }
@@ -1413,21 +1433,6 @@ __device__ __forceinline__ bool grid_sync(unsigned* sync, unsigned& nsync, int* 
     return *s_flag == 0;
 }
 
-// L2 prefetch of the weight rows of one tile (lanes 0..7 of the calling warp),
-// in pieces of at most 32 KB.
-template <int EPI>
-__device__ __forceinline__ void prefetch_tile(const GemvParams& p, int tile, int lane) {
-    if (lane < kTileRows) {
-        bool v;
-        const uint16_t* r = tile_row<EPI>(p, tile, lane, v);
-        if (v) {
-            const uint32_t bytes = (uint32_t)p.K * 2u;  // a multiple of 16 (K % 8 == 0)
-            for (uint32_t off = 0; off < bytes; off += 32768u)
-                prefetch_l2(reinterpret_cast<const char*>(r) + off, min(32768u, bytes - off));
-        }
-    }
-}
-
 template <int EPI>
 __device__ __forceinline__ int tile_count(const GemvParams& p) {
     return (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? (p.n_units + kTileRows / 2 - 1) / (kTileRows / 2)
@@ -1867,9 +1872,19 @@ cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* w
 }
 
 cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st,
-                              bool pdl, bool w_host) {
+                              bool pdl, bool w_host, bool prefetch_waves) {
     GemvParams p{};
     p.w_host = w_host;
+    if (prefetch_waves && !w_host) {  // two block-tile blocks are resident per SM
+        static int sms = 0;
+        if (!sms) {
+            int dev = 0;
+            if (cudaGetDevice(&dev) != cudaSuccess ||
+                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+                sms = 0;
+        }
+        p.pf_stride = 2 * sms;
+    }
     p.in = in;
     p.w0 = w;
     p.B = B;

@@ -52,8 +52,12 @@ cudaError_t launch_qkv_rope(const float* x, const uint16_t* g, const uint16_t* w
 cudaError_t launch_qk_norm_rope(const float* raw, int rows, int Hq, int Hkv, int d, bool with_v, const uint16_t* g_q,
                                 const uint16_t* g_k, float eps, float theta, const int32_t* positions,
                                 const int32_t* row_req, float* q_out, KvView kv, cudaStream_t st, bool pdl = false);
+// x += W in (W [N, K] bf16).  prefetch_waves: batch-1 tiles beyond the first
+// wave are pulled into L2 by the first-wave blocks while they wait on the
+// previous kernel (for the O-projection, whose predecessor, attention, leaves
+// HBM idle; behind a bandwidth-bound kernel the prefetch only competes).
 cudaError_t launch_resid_gemv(const float* in, const uint16_t* w, int B, int N, int K, float* x, cudaStream_t st,
-                              bool pdl = false, bool w_host = false);
+                              bool pdl = false, bool w_host = false, bool prefetch_waves = false);
 cudaError_t launch_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int B, int H,
                            int F, float eps, float* a, cudaStream_t st, bool pdl = false, bool w_host = false);
 // Streams `bytes` (a multiple of 16) from `src` with 128-bit loads over `blocks`

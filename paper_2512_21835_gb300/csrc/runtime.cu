@@ -643,7 +643,7 @@ struct loip_ctx {
                                     fixed_ptr<float>(fx.attn_scratch), o, false, s, pdl(), cfg.max_batch, true);
         });
         if (e != cudaSuccess) return cuda_fail(e, "attention kernel");
-        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl(), host_a); });
+        e = timed(2, s, [&] { return launch_resid_gemv(o, wo, B, H, qd, x, s, pdl(), host_a, true); });
         if (e != cudaSuccess) return cuda_fail(e, "o-proj kernel");
         e = timed(3, s, [&] {
             return launch_gate_up(x, g_mlp, wg, wu, B, H, F, desc.rms_eps, a, s, pdl(), host_m);
