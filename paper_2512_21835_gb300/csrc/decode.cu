@@ -757,9 +757,10 @@ cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, bool pdl, int* nblocks_o
     // Batch 1: matrices with few rows (QKV, O-proj, down) keep too few units per
     // warp for the persistent kernel to ramp up; the block-tile kernel issues a
     // whole tile at once.  Row-rich ones (gate/up, LM head) stream better
-    // persistent.
+    // persistent, and so does a QKV of more than 8192 rows (13B: 15360, two or
+    // more RoPE pairs per warp), whose tiles would take six waves.
     const int rows = (EPI == EPI_SWIGLU) ? 2 * p.n_units : p.N;
-    if (p.B == 1 && rows <= 16384) {
+    if (p.B == 1 && rows <= (EPI == EPI_QKV ? 8192 : 16384)) {
         const int per_tile = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? kTileRows / 2 : kTileRows;
         const int units = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? p.n_units : p.N;
         const int tiles = (units + per_tile - 1) / per_tile;

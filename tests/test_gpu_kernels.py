@@ -42,8 +42,9 @@ def test_embed_exact(torch, L, orc):
     assert np.array_equal(x.cpu().numpy().astype(np.float64), orc.bf16_bits_to_f64(E[toks]))
 
 
+# batch 1: block-tile kernel up to 16384 gate + up rows, persistent kernel above (1, 512, 9000)
 @pytest.mark.parametrize("B,H,F", [(1, 1000, 300), (3, 4096, 1000), (8, 2048, 700), (1, 13000, 64),
-                                   (5, 4096, 129), (2, 256, 688)])
+                                   (5, 4096, 129), (2, 256, 688), (1, 512, 9000)])
 def test_gate_up_parity(torch, L, orc, B, H, F):
     eps = 1e-5
     x = inputs.normal_f32(B * 7 + H, (B, H), 1.5)
@@ -64,8 +65,9 @@ def test_gate_up_parity(torch, L, orc, B, H, F):
         assert np.all(np.abs(got[b] - want) <= tol), (b, np.max(np.abs(got[b] - want) / tol))
 
 
+# batch 1: block-tile kernel up to 16384 rows, persistent kernel above (1, 17000, 256)
 @pytest.mark.parametrize("B,N,K", [(1, 300, 1000), (2, 777, 4096), (8, 100, 14336), (1, 4096, 14336),
-                                   (3, 513, 2048), (1, 256, 256)])
+                                   (3, 513, 2048), (1, 256, 256), (1, 17000, 256)])
 def test_residual_projection_parity(torch, L, orc, B, N, K):
     a = inputs.normal_f32(11 + K, (B, K), 0.7)
     x0 = inputs.normal_f32(12 + N, (B, N), 1.0)
@@ -135,10 +137,15 @@ def test_attention_parity(torch, L, orc, Hq, Hkv, d, max_ctx, ctx_list):
         assert np.max(np.abs(got[b] - want)) <= tol, (b, np.max(np.abs(got[b] - want)), tol)
 
 
-@pytest.mark.parametrize("Hq,Hkv,d,H", [(4, 2, 64, 256), (32, 8, 128, 4096), (8, 8, 128, 1024)])
-def test_qkv_rope_parity(torch, L, orc, Hq, Hkv, d, H):
+# one row (batch-1 decode) runs the block-tile kernel up to 8192 QKV rows and the
+# persistent kernel above (64 x 128 query + 2 x 8 x 128 kv rows = 10240)
+@pytest.mark.parametrize("single", [False, True])
+@pytest.mark.parametrize("Hq,Hkv,d,H", [(4, 2, 64, 256), (32, 8, 128, 4096), (8, 8, 128, 1024), (64, 8, 128, 1024)])
+def test_qkv_rope_parity(torch, L, orc, Hq, Hkv, d, H, single):
     P, eps, theta = 64, 1e-5, 500000.0
     pos = np.array([0, 5, 130, 1000], dtype=np.int32)[: 3 if Hq == 8 else 4]
+    if single:
+        pos = np.array([1000], dtype=np.int32)
     B = len(pos)
     max_pages = 1000 // P + 1
     buf, order, lpb = _paged_cache(torch, B * max_pages, Hkv, P, d, 4)
