@@ -758,9 +758,12 @@ cudaError_t launch_gemv(GemvParams& p, cudaStream_t st, bool pdl, int* nblocks_o
     // warp for the persistent kernel to ramp up; the block-tile kernel issues a
     // whole tile at once.  Row-rich ones (gate/up, LM head) stream better
     // persistent, and so does a QKV of more than 8192 rows (13B: 15360, two or
-    // more RoPE pairs per warp), whose tiles would take six waves.
+    // more RoPE pairs per warp), whose tiles would take six waves.  Weights in
+    // mapped host memory always go to the persistent kernel: over the host link
+    // a tile's serial chunk loads along a long row (down, K = 28672) ran at
+    // 183 GB/s against the link's 211, which the persistent kernel reaches.
     const int rows = (EPI == EPI_SWIGLU) ? 2 * p.n_units : p.N;
-    if (p.B == 1 && rows <= (EPI == EPI_QKV ? 8192 : 16384)) {
+    if (p.B == 1 && !p.w_host && rows <= (EPI == EPI_QKV ? 8192 : 16384)) {
         const int per_tile = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? kTileRows / 2 : kTileRows;
         const int units = (EPI == EPI_QKV || EPI == EPI_SWIGLU) ? p.n_units : p.N;
         const int tiles = (units + per_tile - 1) / per_tile;
@@ -1150,7 +1153,8 @@ cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st, bool pdl) {
 //   softmax warp g takes query head g over the page's positions: page max m,
 //           weights exp(s - m), their sum l;
 //   values  thread (dim pair, head) accumulates the weighted value rows in
-//           position order.
+//           position order (with fewer than 512 outputs, groups of threads take
+//           consecutive position ranges and their sums are added in order).
 // The page's unnormalised state (o, m, l) goes to scratch; the last block of
 // the (row, kv head) to arrive (completion ticket) combines every page's state
 // with the usual softmax merge: weights exp(m_c - max m) / sum, outputs summed in
@@ -1162,6 +1166,8 @@ struct AttnPageSmem {
     alignas(16) float sq[G][D];
     float sc[4][G][64];  // partial scores per dim quarter
     float sp[G][64];     // exp(s - m) of the page's positions
+    // value partial sums of the position groups, when G x d < 512 (else unused)
+    alignas(8) float pv[G * D < 512 ? 512 : 2];
     int last;
 };
 
@@ -1169,6 +1175,7 @@ template <int G, int D>
 __global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
     constexpr int NT = 256, CH = D / 8, P = 64;
     constexpr int PAIRS = D / 2, GS = NT / PAIRS, NG = (G + GS - 1) / GS;
+    constexpr int PV_SPLIT = G * PAIRS >= NT ? 1 : NT / (G * PAIRS);
     static_assert(G * kMaxChunks * sizeof(float) <= sizeof(uint16_t) * 64 * D, "combine weights fit a stage");
     __shared__ AttnPageSmem<G, D> sm;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -1250,31 +1257,59 @@ __global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
         l_pg = warp_sum(lsum);
     }
     __syncthreads();
-    const int dp = tid % PAIRS, g0 = tid / PAIRS;
-    float acc[NG][2];
+    const size_t hstride = (size_t)p.max_chunks * (D + 2);
+    float* base = p.scratch + ((size_t)row * p.Hq + (size_t)kvh * G) * hstride;
+    const int dp = tid % PAIRS;
+    if constexpr (PV_SPLIT == 1) {
+        const int g0 = tid / PAIRS;
+        float acc[NG][2];
 #pragma unroll
-    for (int k = 0; k < NG; ++k) acc[k][0] = acc[k][1] = 0.f;
-    for (int t = 0; t < nvalid; ++t) {
-        const uint32_t vv = *reinterpret_cast<const uint32_t*>(&sm.sV[t * D + 2 * dp]);
-        const float v0 = bf_lo(vv), v1 = bf_hi(vv);
+        for (int k = 0; k < NG; ++k) acc[k][0] = acc[k][1] = 0.f;
+        for (int t = 0; t < nvalid; ++t) {
+            const uint32_t vv = *reinterpret_cast<const uint32_t*>(&sm.sV[t * D + 2 * dp]);
+            const float v0 = bf_lo(vv), v1 = bf_hi(vv);
+#pragma unroll
+            for (int k = 0; k < NG; ++k) {
+                const int g = g0 + k * GS;
+                if (g < G) {
+                    const float pr = sm.sp[g][t];
+                    acc[k][0] = fmaf(pr, v0, acc[k][0]);
+                    acc[k][1] = fmaf(pr, v1, acc[k][1]);
+                }
+            }
+        }
 #pragma unroll
         for (int k = 0; k < NG; ++k) {
             const int g = g0 + k * GS;
-            if (g < G) {
-                const float pr = sm.sp[g][t];
-                acc[k][0] = fmaf(pr, v0, acc[k][0]);
-                acc[k][1] = fmaf(pr, v1, acc[k][1]);
-            }
+            if (g < G)
+                *reinterpret_cast<float2*>(base + g * hstride + (size_t)chunk * (D + 2) + 2 * dp) =
+                    make_float2(acc[k][0], acc[k][1]);
         }
-    }
-    const size_t hstride = (size_t)p.max_chunks * (D + 2);
-    float* base = p.scratch + ((size_t)row * p.Hq + (size_t)kvh * G) * hstride;
+    } else {
+        // fewer outputs than threads (G x d / 2 < 256): PV_SPLIT thread groups take
+        // consecutive position ranges, and group 0 adds the partial sums in order
+        constexpr int SPAN = P / PV_SPLIT;
+        const int rest = tid / PAIRS, g = rest % G, part = rest / G;
+        const int t0 = part * SPAN, t1 = min(nvalid, t0 + SPAN);
+        float a0 = 0.f, a1 = 0.f;
+        for (int t = t0; t < t1; ++t) {
+            const uint32_t vv = *reinterpret_cast<const uint32_t*>(&sm.sV[t * D + 2 * dp]);
+            const float pr = sm.sp[g][t];
+            a0 = fmaf(pr, bf_lo(vv), a0);
+            a1 = fmaf(pr, bf_hi(vv), a1);
+        }
+        *reinterpret_cast<float2*>(&sm.pv[(part * G + g) * D + 2 * dp]) = make_float2(a0, a1);
+        __syncthreads();
+        if (part == 0) {
+            float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-    for (int k = 0; k < NG; ++k) {
-        const int g = g0 + k * GS;
-        if (g < G)
-            *reinterpret_cast<float2*>(base + g * hstride + (size_t)chunk * (D + 2) + 2 * dp) =
-                make_float2(acc[k][0], acc[k][1]);
+            for (int q = 0; q < PV_SPLIT; ++q) {
+                const float2 v = *reinterpret_cast<const float2*>(&sm.pv[(q * G + g) * D + 2 * dp]);
+                s0 += v.x;
+                s1 += v.y;
+            }
+            *reinterpret_cast<float2*>(base + g * hstride + (size_t)chunk * (D + 2) + 2 * dp) = make_float2(s0, s1);
+        }
     }
     if (warp < G && lane == 0) {
         float* part = base + warp * hstride + (size_t)chunk * (D + 2);

@@ -165,8 +165,10 @@ def test_multi_head_model_matches_oracle(torch, L, orc):
 
 def test_direct_access_decode_copies_nothing(torch, L, orc):
     """LOIP_MODE_DIRECT: decode steps read the offloaded layers in place from the
-    host pool (no weight copies after the prefill's) and stay bit-identical to
-    the all-resident run."""
+    host pool (no weight copies after the prefill's).  The prefill (through the
+    slots) is bit-identical to the all-resident run; decode reads host weights
+    with the persistent GEMV, whose summation order differs from the block-tile
+    kernel's, so decode tokens agree exactly and hidden states to rounding."""
     m = TINY6
     prompts = [inputs.token_ids(51, 30, m["vocab"])]
     cont = [[int(t)] for t in inputs.token_ids(52, 8, m["vocab"])]
@@ -187,7 +189,8 @@ def test_direct_access_decode_copies_nothing(torch, L, orc):
     assert ctx.stats()["h2d_weight_bytes"] == after_prefill
     ctx.close()
     assert np.array_equal(np.array(toks), base[0])
-    assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
+    assert np.array_equal(hids[0].view(np.uint32), base[1][0].view(np.uint32))
+    assert np.max(np.abs(np.array(hids) - base[1])) <= 1e-4
 
 
 def _decode_with_timing(L, torch, m, prompt, cont, cfg_kw, resident_layers):
