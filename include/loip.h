@@ -377,7 +377,9 @@ int loip_k_attention_noalloc(const float* q, const void* kv_base, const int64_t*
                              int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx, float* o,
                              void* stream);
 
-/* x += wo o  (output projection with the residual add); o fp32 [B, Hq*d]. */
+/* x += wo o  (output projection with the residual add); o fp32 [B, Hq*d].  As in
+ * decode, at batch 1 the blocks of the first wave also pull the later blocks'
+ * weight tiles into L2 (a cache hint: results equal loip_k_down's bit for bit). */
 int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x, void* stream);
 
 /* a = silu(wg y) * (wu y) with y = RMSNorm(x) * g (SwiGLU MLP input half);

@@ -1896,7 +1896,7 @@ extern "C" int loip_k_attention(const float* q, const void* kv_base, const int64
 extern "C" int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x,
                             void* stream) {
     if (!o || !wo || !x || B < 1 || B > 8 || K % 8 || H < 1 || !al16(wo) || !al16(o)) return LOIP_ERR_INVALID;
-    return cerr(launch_resid_gemv(o, wo, B, H, K, x, (cudaStream_t)stream));
+    return cerr(launch_resid_gemv(o, wo, B, H, K, x, (cudaStream_t)stream, false, false, true));
 }
 
 extern "C" int loip_k_gate_up(const float* x, const uint16_t* g, const uint16_t* wg, const uint16_t* wu, int32_t B,

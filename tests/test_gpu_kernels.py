@@ -80,7 +80,8 @@ def test_residual_projection_parity(torch, L, orc, B, N, K):
         want = x0[b].astype(np.float64) + orc.gemv(W, K, a[b].astype(np.float64))
         tol = dot_bound(W64, a[b].astype(np.float64), K) + 4 * U * np.abs(want)
         assert np.all(np.abs(got[b] - want) <= tol)
-    # the o-projection entry point is the same product
+    # the o-projection entry point is the same product (at batch 1 its first-wave
+    # blocks also prefetch the later tiles into L2: (1, 4096, 14336) has 512 tiles)
     x2 = dev_f32(x0)
     L.loip_k_oproj(dev_f32(a), dev_bits(W), x2)
     assert np.array_equal(x2.cpu().numpy(), x.cpu().numpy())
