@@ -100,7 +100,10 @@ def _paged_cache(torch, n_pages, Hkv, P, d, seed):
 # blocks with the last-block combine
 @pytest.mark.parametrize("max_ctx,ctx_list", [(256, (1, 70, 200, 64)), (1088, (1, 700, 1088, 129)),
                                               (2112, (1, 2112, 999, 64))])
-@pytest.mark.parametrize("Hq,Hkv,d", [(8, 2, 128), (4, 2, 64), (32, 8, 128), (64, 8, 128)])
+# G = Hq / Hkv from 1 to 8 at head_dim 64 and 128: with fewer than 512 outputs per kv
+# head (G x d) the value sums are split over position groups
+@pytest.mark.parametrize("Hq,Hkv,d", [(8, 2, 128), (4, 2, 64), (32, 8, 128), (64, 8, 128), (8, 8, 128),
+                                      (4, 4, 64), (16, 4, 64)])
 def test_attention_parity(torch, L, orc, Hq, Hkv, d, max_ctx, ctx_list):
     P = 64
     ctx = np.array(ctx_list, dtype=np.int32)
