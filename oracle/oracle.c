@@ -102,7 +102,9 @@ uint16_t orc_gen_elem(uint64_t seed, uint32_t tensor_id, uint64_t index, int kin
 }
 
 void orc_gen_tensor(uint64_t seed, uint32_t tensor_id, uint64_t first, uint64_t n, int kind, uint16_t* out) {
-    for (uint64_t i = 0; i < n; ++i) out[i] = orc_gen_elem(seed, tensor_id, first + i, kind);
+    /* each element depends on its index only: the order of evaluation is free */
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < (int64_t)n; ++i) out[i] = orc_gen_elem(seed, tensor_id, first + (uint64_t)i, kind);
 }
 
 /* ------------------------------------------------------------------------- */
