@@ -51,7 +51,11 @@ enum {
  *   pinned host pool through its device mapping (zero-copy over the host link;
  *   the counterpart of the paper's UMA-aware loading, Sec. III-C, on a
  *   discrete-memory GPU).  Prefill, loip_stream_layer and loip_layer_forward
- *   keep using the slots, so the plan still reserves them. */
+ *   keep using the slots, so the plan still reserves them.  At batch 1 the
+ *   projections of host-resident weights run on the persistent GEMV (the
+ *   resident path uses the block-tile one for row-poor matrices), so decode
+ *   results equal an all-resident run's to rounding, tokens included in
+ *   practice, rather than bit for bit; at larger batches both paths are the same. */
 enum { LOIP_MODE_OVERLAP = 0, LOIP_MODE_NAIVE = 1, LOIP_MODE_DIRECT = 2 };
 
 typedef struct loip_model_desc {
