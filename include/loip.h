@@ -54,8 +54,8 @@ enum {
  *   keep using the slots, so the plan still reserves them.  At batch 1 the
  *   projections of host-resident weights run on the persistent GEMV (the
  *   resident path uses the block-tile one for row-poor matrices), so decode
- *   results equal an all-resident run's to rounding, tokens included in
- *   practice, rather than bit for bit; at larger batches both paths are the same. */
+ *   hidden states equal an all-resident run's to rounding (tokens equal in
+ *   the tests) rather than bit for bit; at larger batches both paths agree bit for bit. */
 enum { LOIP_MODE_OVERLAP = 0, LOIP_MODE_NAIVE = 1, LOIP_MODE_DIRECT = 2 };
 
 typedef struct loip_model_desc {
