@@ -43,8 +43,8 @@ RUN_CLASS = 12  # kernel-timing class of the persistent layer-run kernel
 
 # DRAM bytes (read + write) per launch of the gate/up SwiGLU GEMV at batch 1
 # (the persistent kernel, at the 70B and the 8B shape), from an
-# ncu capture of the kernel microbenchmark on the model's shape
-# (profiles/gemv_traffic.md has the commands and figures).  They describe the
+# ncu capture of the kernel microbenchmark on the model's shape (the
+# gate/up traffic summary among the ncu summaries has the commands).  They describe the
 # kernel source they were taken on: when the decode kernels' source no longer
 # has this hash the figure is reported as null.
 GATE_UP_TRAFFIC = {"llama3-70b": 939_868_416, "llama3-8b": 235_416_576}

@@ -276,8 +276,13 @@ int loip_prefill(loip_ctx* ctx, const int32_t* tokens, const int32_t* prompt_len
                  int32_t* out_tokens, float* out_hidden);
 
 /* Re-plans for the current KV size (Eq. 6 thresholds): while the KV pages the
- * next `lookahead_tokens` tokens of every request need do not fit, one more
- * resident layer is demoted to the host pool (evenly spaced).  Synchronous. */
+ * next `lookahead_tokens` tokens of every request need do not fit, device
+ * weights are given up for KV memory.  With block granularity (the default,
+ * loip_config.whole_layers = 0) Eq. 7 chooses how many MHA and MLP blocks to
+ * give up for the shortfall (the fewest streamed bytes that cover it); with
+ * whole_layers = 1 one more resident layer is demoted at a time, evenly
+ * spaced.  Demoted weights keep a host copy and stream from then on.
+ * Synchronous. */
 int loip_replan(loip_ctx* ctx, int32_t lookahead_tokens);
 
 int loip_get_stats(const loip_ctx* ctx, loip_stats* out);
@@ -370,7 +375,9 @@ uint64_t loip_k_attention_scratch_floats(int32_t B, int32_t Hq, int32_t d, int32
  * file-scope device array of LOIP_NOALLOC_SCRATCH_FLOATS floats that every GPU
  * loading the library holds until the process exits.  LOIP_ERR_INVALID when
  * loip_k_attention_scratch_floats(B, Hq, d, max_ctx, page_tokens) exceeds that
- * size.  It allocates nothing (no cudaMalloc, cudaFree or allocating library
+ * size, when Hq / Hkv is not 1, 2, 4 or 8, or when a pointer is misaligned (q
+ * and kv_base need 16 bytes, page_offsets 8, ctx_lens and o 4); every refusal
+ * happens before anything is enqueued.  It allocates nothing (no cudaMalloc, cudaFree or allocating library
  * call).  The first call on a device, with that device current, looks up the
  * array's device address (cudaGetSymbolAddress); make that first call before
  * any stream capture.  All calls on a device share the array and it keeps the

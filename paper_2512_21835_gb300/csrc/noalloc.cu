@@ -57,6 +57,14 @@ extern "C" int loip_k_attention_noalloc(const float* q, const void* kv_base, con
     if (!q || !kv_base || !page_offsets || !ctx_lens || !o || B < 1 || Hq < 1 || Hkv < 1 || (d != 64 && d != 128) ||
         Hq % Hkv || max_ctx < 1 || page_tokens != 64 || (int64_t)max_pages * page_tokens < max_ctx)
         return LOIP_ERR_INVALID;
+    // the kernel reads q and the pages with 16-byte loads, the page table as
+    // int64, the lengths as int32 and writes o as fp32: a misaligned pointer is
+    // refused here rather than trapping on the device
+    if (((uintptr_t)q & 15) || ((uintptr_t)kv_base & 15) || ((uintptr_t)page_offsets & 7) ||
+        ((uintptr_t)ctx_lens & 3) || ((uintptr_t)o & 3))
+        return LOIP_ERR_INVALID;
+    const int G = Hq / Hkv;  // query heads per kv head: the kernel is built for these
+    if (G != 1 && G != 2 && G != 4 && G != 8) return LOIP_ERR_INVALID;
     if (attention_scratch_floats(B, Hq, d, max_ctx, page_tokens) > LOIP_NOALLOC_SCRATCH_FLOATS ||
         (max_ctx + page_tokens - 1) / page_tokens > 256)
         return LOIP_ERR_INVALID;  // the partial states and counters do not fit

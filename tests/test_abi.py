@@ -132,3 +132,53 @@ def test_ssd_tier_roundtrip(L, tmp_path):
     assert loip.loip_ssd_roundtrip(str(tmp_path), 4096)
     with pytest.raises(RuntimeError):
         loip.loip_ssd_roundtrip(str(tmp_path), 1000)  # not a multiple of the 4 KB block
+
+
+def _no_device():
+    try:
+        import torch
+        return not torch.cuda.is_available()
+    except ImportError:
+        return True
+
+
+def test_noalloc_attention_refusals_without_gpu(L):
+    """The allocation-free attention's argument checks, on a machine without a
+    GPU: every call here must be refused before the library touches CUDA (the
+    pointers are aligned dummies that nothing may read).  The size limit is
+    checked at the boundary for many shapes: refused exactly when the scratch
+    the shape needs exceeds the fixed array."""
+    if not _no_device():
+        pytest.skip("dummy pointers: run only where no CUDA device exists")
+    LIM = loip.NOALLOC_SCRATCH_FLOATS
+    q, kv, pt, cl, o = 1 << 20, 2 << 20, 3 << 20, 4 << 20, 5 << 20  # 16-byte aligned, never dereferenced
+
+    def call(B, Hq, Hkv, d, max_ctx, q=q, kv=kv, pt=pt, cl=cl, o=o):
+        pages = (max_ctx + 63) // 64
+        return L.loip_k_attention_noalloc(q, kv, pt, pages, cl, B, Hq, Hkv, d, 64, 0, 2 * Hkv * 64 * d * 2,
+                                          max_ctx, o, None)
+
+    n_edge = 0
+    for B in (1, 3, 8, 16):
+        for Hq, Hkv in ((8, 8), (16, 8), (32, 8), (64, 8), (40, 5)):
+            for d in (64, 128):
+                need = [loip.loip_k_attention_scratch_floats(B, Hq, d, c, 64) for c in range(64, 16385, 64)]
+                assert need == sorted(need)
+                # the smallest context that no longer fits, and one page below it
+                over = next((c for c, n in zip(range(64, 16385, 64), need) if n > LIM), None)
+                if over is None or over - 64 < 1:
+                    continue
+                assert loip.loip_k_attention_scratch_floats(B, Hq, d, over - 64, 64) <= LIM
+                for c in (over - 63, over):  # first position of the page that crosses the limit, and its last
+                    assert loip.loip_k_attention_scratch_floats(B, Hq, d, c, 64) > LIM
+                    assert call(B, Hq, Hkv, d, c) == loip.ERR_INVALID
+                n_edge += 1
+    assert n_edge >= 15
+    # misaligned pointers and unsupported head ratios, in shapes that fit the array
+    ok = dict(B=2, Hq=8, Hkv=2, d=64, max_ctx=100)
+    assert loip.loip_k_attention_scratch_floats(2, 8, 64, 100, 64) <= LIM
+    for bad in (dict(q=q + 4), dict(q=q + 8), dict(kv=kv + 2), dict(pt=pt + 4), dict(cl=cl + 2), dict(o=o + 1)):
+        assert call(**ok, **bad) == loip.ERR_INVALID, bad
+    assert call(B=2, Hq=24, Hkv=8, d=64, max_ctx=100) == loip.ERR_INVALID  # 3 query heads per kv head
+    assert call(B=2, Hq=48, Hkv=3, d=64, max_ctx=100) == loip.ERR_INVALID  # 16
+    assert call(B=2, Hq=8, Hkv=2, d=96, max_ctx=100) == loip.ERR_INVALID   # head size
