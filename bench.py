@@ -239,6 +239,15 @@ def run_ours(args, rank, world):
     step_ms = [round(ev0.elapsed_time(step_ev[0]), 2)] + [round(step_ev[i - 1].elapsed_time(step_ev[i]), 2)
                                                           for i in range(1, steps)]
     st1 = ctx.stats()
+    # per-copy link rates of the timed region (copy-stream events), grouped by step
+    n_cp = int(st1["copies_total"] - st0["copies_total"])
+    cp_ms, cp_by = ctx.copy_log()
+    cp_ms, cp_by = cp_ms[len(cp_ms) - min(n_cp, len(cp_ms)):], cp_by[len(cp_by) - min(n_cp, len(cp_by)):]
+    cp_rate = cp_by / np.maximum(cp_ms, 1e-9) / 1e6  # GB/s
+    per_step = max(1, len(cp_ms) // steps)
+    step_copy_GBps = [round(float(cp_by[i:i + per_step].sum() / max(1e-9, cp_ms[i:i + per_step].sum()) / 1e6), 1)
+                      for i in range(0, per_step * (len(cp_ms) // per_step), per_step)]
+    pool_nodes = ctx.pool_nodes()
     # ---- per-kernel durations (CUDA events around every launch, separate pass) ----
     ctx.set_kernel_timing(True)
     for _ in range(steps):
@@ -347,6 +356,13 @@ def run_ours(args, rank, world):
                           "pool_blob_GBps_min_median": [round(st1["pool_min_GBps"], 1),
                                                         round(st1["pool_median_GBps"], 1)],
                           "pool_blobs_moved": st1["pool_replaced"],
+                          "pool_numa": {"node": st1["pool_numa_node"], "blobs": st1["pool_blobs"],
+                                        "blobs_on_node": st1["pool_blobs_on_node"],
+                                        "nodes_seen": sorted({int(v) for v in pool_nodes if v >= 0})},
+                          "copy_GBps_min_median_max": ([round(float(np.min(cp_rate)), 1),
+                                                        round(float(np.median(cp_rate)), 1),
+                                                        round(float(np.max(cp_rate)), 1)] if len(cp_rate) else None),
+                          "step_copy_GBps": step_copy_GBps,
                           "ssd_layers": st1["n_ssd_layers"],
                           "ssd_GBps": round((st1["ssd_read_bytes"] - st0["ssd_read_bytes"]) / dev_s / 1e9, 2),
                           "ssd_ms_per_step": {k: round((st_end[k] - st0[k]) / (steps + 4 + steps), 1)

@@ -139,6 +139,9 @@ typedef struct loip_stats {
     double ssd_wait_ms;        /* host time spent waiting for SSD-tier reads to land */
     double ssd_stage_wait_ms;  /* host time spent waiting for a staging buffer's copy to a slot */
     double ssd_copy_ms;        /* summed duration of the copies out of staging buffers (events) */
+    int32_t pool_numa_node;    /* host NUMA node the pool's pages were asked for (the GPU's, -1: none) */
+    int32_t pool_blobs;        /* streamed layers with a blob in the host pool */
+    int32_t pool_blobs_on_node;/* of those, blobs whose sampled pages are mostly on pool_numa_node */
 } loip_stats;
 
 typedef struct loip_ctx loip_ctx;
@@ -275,6 +278,57 @@ int loip_decode_step_device(loip_ctx* ctx, const int32_t* tokens_dev, int32_t ba
 int loip_prefill(loip_ctx* ctx, const int32_t* tokens, const int32_t* prompt_lens, int32_t n_prompts,
                  int32_t* out_tokens, float* out_hidden);
 
+/* The most recent completed layer copies into the slots (up to 8192 kept):
+ * writes min(max_n, kept) entries, oldest first, of their duration (ms, CUDA
+ * events on the copy stream) and size (bytes) to ms / bytes (host arrays of
+ * max_n) and returns the count, or -1 on bad arguments.  Per-copy rates show
+ * which steps the host link slowed (Sec. III-C's loading path). */
+int32_t loip_get_copy_log(loip_ctx* ctx, double* ms, uint64_t* bytes, int32_t max_n);
+
+/* Host NUMA node holding most of each layer's pool blob (host int32
+ * [n_layers]; -1 for layers without a blob, or when the kernel cannot tell),
+ * read with move_pages queries of 32 pages per blob when the pool was filled.
+ * The pool asks for the GPU's host node (loip_stats.pool_numa_node). */
+int loip_get_pool_nodes(loip_ctx* ctx, int32_t* nodes);
+
+/* Fault injection, for tests of the failure handling (the paper has no
+ * counterpart: it reports only out-of-memory and out-of-time outcomes, Sec.
+ * IV-A).  Arms one fault on the context; it fires once, at the next place
+ * named below, and is made on the host or as a bounded device wait -- never as
+ * a GPU fault, trap or hang:
+ *   LOIP_FAULT_WAIT        the next host wait on the device treats its event
+ *                          as still pending: the call returns LOIP_ERR_TIMEOUT
+ *                          after loip_config.timeout_ms (the device work itself
+ *                          completes) and the context then refuses every call
+ *                          with LOIP_ERR_STATE;
+ *   LOIP_FAULT_COPY        the next weight copy into a slot reports a CUDA error
+ *                          before anything is enqueued: LOIP_ERR_CUDA, context
+ *                          failed;
+ *   LOIP_FAULT_HOST_ALLOC  the next pinned host-pool allocation fails:
+ *                          LOIP_ERR_OOM (the context stays usable);
+ *   LOIP_FAULT_BARRIER     the next layer-run kernel launch (batch-1 decode with
+ *                          loip_config.layer_run_kernel = 1): block `arg` does
+ *                          not arrive at the first grid barrier and every
+ *                          barrier wait of that launch gives up after 10 ms; the
+ *                          kernel sets its error word and returns, and the step
+ *                          returns LOIP_ERR_TIMEOUT (context failed; the GPU and
+ *                          other contexts stay usable);
+ *   LOIP_FAULT_NONE        disarms.
+ * LOIP_ERR_INVALID for an unknown kind or a negative block. */
+#define LOIP_FAULT_NONE 0
+#define LOIP_FAULT_WAIT 1
+#define LOIP_FAULT_COPY 2
+#define LOIP_FAULT_HOST_ALLOC 3
+#define LOIP_FAULT_BARRIER 4
+int loip_inject_fault(loip_ctx* ctx, int32_t kind, int32_t arg);
+
+/* The deadline loop every host wait of the library runs, driven by a fake
+ * device that reports "pending" for `pending_polls` polls (< 0: forever):
+ * LOIP_OK once it reports done, LOIP_ERR_TIMEOUT once timeout_ms of wall time
+ * have passed; *waited_ms (may be NULL) gets the time spent.  Makes no CUDA
+ * call, so it checks the deadline logic on a machine without a GPU. */
+int loip_poll_deadline_check(uint32_t timeout_ms, int32_t pending_polls, double* waited_ms);
+
 /* Re-plans for the current KV size (Eq. 6 thresholds): while the KV pages the
  * next `lookahead_tokens` tokens of every request need do not fit, device
  * weights are given up for KV memory.  With block granularity (the default,
@@ -406,6 +460,15 @@ int loip_k_down(const float* a, const uint16_t* wd, int32_t B, int32_t H, int32_
  * (N % 4 == 0), fp32 accumulation (tcgen05, TMA; the product the prefill runs
  * for the output and down projections). */
 int loip_k_gemm_bf16(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N, int32_t K, float* x, void* stream);
+
+/* The prefill's projection at fp32 activation precision: x[M, N] += A W^T
+ * where A (fp32 [M, K]) is given as a split pair of bf16 planes A2 = [2][M][K]:
+ * A2[0] = bf16(A) and A2[1] = bf16(A - A2[0]), so A2[0] + A2[1] carries A to
+ * ~2^-17 relative.  Every K step issues two tensor-core MMAs into the same
+ * fp32 accumulator (A2[0] W^T + A2[1] W^T); W stays the unmodified bf16 weight
+ * (the losslessness of Sec. IV-A: no weight is changed).  Same layout, sizes
+ * and alignment rules as loip_k_gemm_bf16; M * K elements per plane. */
+int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t M, int32_t N, int32_t K, float* x, void* stream);
 
 /* 0 if no tensor-core GEMM launch has recorded a failure (a bounded pipeline
  * wait that ran out); otherwise the first failure code.  -1 if unreadable. */

@@ -25,10 +25,8 @@ _DIR = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_DIR, "oracle.c")
 _LIB_PATH = os.path.join(_DIR, "liboracle.so")
 
-KV_BF16 = 1
-ACT_BF16 = 2
-Q_BF16 = 4
-PREFILL_FLAGS = KV_BF16 | ACT_BF16 | Q_BF16
+KV_BF16 = 1  # keys and values rounded to bf16 as they enter the cache (the device's cache type)
+PREFILL_FLAGS = KV_BF16
 DECODE_FLAGS = KV_BF16
 
 # tensor order inside a model (mirrors oracle.c)

@@ -16,13 +16,13 @@
  * SwiGLU MLP, untied LM head, greedy argmax (lowest index on ties).
  * Arithmetic is fp64, sequential sums, no blocking or reordering.
  *
- * Storage-precision mirrors (flags), so that integer decisions are taken on the
- * same numbers the kernels see:
- *   ORC_KV_BF16  keys (after rotation) and values are rounded to bf16 when they
- *                enter the cache (the device cache holds bf16).
- *   ORC_ACT_BF16 inputs of the four projections (normed x, attention output,
- *                SwiGLU output) are rounded to bf16 (tensor-core prefill path).
- *   ORC_Q_BF16   queries (after rotation) are rounded to bf16 (prefill path).
+ * Storage precision.  The one value the method stores in a narrower type than
+ * it computes is the KV cache: the device keeps keys (after rotation) and values
+ * in bf16.  Flag ORC_KV_BF16 rounds them to bf16 as they enter the cache, so that
+ * the oracle attends over the same stored values.  Every other quantity stays
+ * fp64 here (the device computes activations in fp32, and its prefill feeds the
+ * tensor cores each activation as a pair of bf16 terms whose sum carries ~16
+ * significant bits, so no activation rounding is mirrored).
  * The argmax is decided on logits rounded to fp32, the precision in which the
  * device decides it.
  *
@@ -39,8 +39,6 @@
 #endif
 
 #define ORC_KV_BF16 1
-#define ORC_ACT_BF16 2
-#define ORC_Q_BF16 4
 
 /* ------------------------------------------------------------------------- */
 /* Seeded synthetic weights: SplitMix64 (Steele, Lea & Flood, "Fast splittable
@@ -287,7 +285,7 @@ int orc_forward(const orc_desc* d, const orc_tensor* ts, const int32_t* tokens, 
 
     for (int64_t t = 0; t < n; ++t) {
         const int flags = t < n_prefill ? prefill_flags : decode_flags;
-        const int kvb = flags & ORC_KV_BF16, actb = flags & ORC_ACT_BF16, qb = flags & ORC_Q_BF16;
+        const int kvb = flags & ORC_KV_BF16;
         /* embedding row */
         for (int i = 0; i < H; ++i) x[i] = tensor_at(&ts[T_EMBED], (uint64_t)tokens[t] * H + i);
         for (int l = 0; l < L; ++l) {
@@ -296,7 +294,6 @@ int orc_forward(const orc_desc* d, const orc_tensor* ts, const int32_t* tokens, 
             double* Vl = Vc + (size_t)l * (size_t)n * kvd;
             /* attention block */
             orc_rmsnorm(x, &lt[L_GATTN], H, d->rms_eps, y);
-            for (int i = 0; i < H; ++i) y[i] = maybe_bf16(y[i], actb);
             orc_gemv(&lt[L_WQ], H, NULL, qd, y, q);
             orc_gemv(&lt[L_WK], H, NULL, kvd, y, k);
             orc_gemv(&lt[L_WV], H, NULL, kvd, y, v);
@@ -307,21 +304,18 @@ int orc_forward(const orc_desc* d, const orc_tensor* ts, const int32_t* tokens, 
             }
             for (int h = 0; h < Hq; ++h) orc_rope(q + (size_t)h * hd, hd, t, d->rope_theta);
             for (int h = 0; h < Hkv; ++h) orc_rope(k + (size_t)h * hd, hd, t, d->rope_theta);
-            for (int i = 0; i < qd; ++i) q[i] = maybe_bf16(q[i], qb);
             for (int i = 0; i < kvd; ++i) {
                 Kl[(size_t)t * kvd + i] = maybe_bf16(k[i], kvb);
                 Vl[(size_t)t * kvd + i] = maybe_bf16(v[i], kvb);
             }
             orc_attention(q, Kl, Vl, t + 1, Hq, Hkv, hd, o, NULL);
-            for (int i = 0; i < qd; ++i) o[i] = maybe_bf16(o[i], actb);
             orc_gemv(&lt[L_WO], qd, NULL, H, o, r);
             for (int i = 0; i < H; ++i) x[i] += r[i];
             /* MLP block */
             orc_rmsnorm(x, &lt[L_GMLP], H, d->rms_eps, y);
-            for (int i = 0; i < H; ++i) y[i] = maybe_bf16(y[i], actb);
             orc_gemv(&lt[L_WG], H, NULL, F, y, gt);
             orc_gemv(&lt[L_WU], H, NULL, F, y, ut);
-            for (int i = 0; i < F; ++i) a[i] = maybe_bf16(orc_silu(gt[i]) * ut[i], actb);
+            for (int i = 0; i < F; ++i) a[i] = orc_silu(gt[i]) * ut[i];
             orc_gemv(&lt[L_WD], F, NULL, H, a, r);
             for (int i = 0; i < H; ++i) x[i] += r[i];
         }

@@ -838,14 +838,29 @@ struct AttnParams {
     float scale;
     float* scratch;  // split: [B][Hq][max_chunks][d + 2] partial states, then int counters [B][Hq]
     int* counters;
-    void* o;         // [B, Hq*d] fp32 or bf16
-    int o_bf16;
+    void* o;         // [B, Hq*d] fp32, or (o_split) two bf16 planes [2][B][Hq*d]
+    int o_split;
     int split;  // kAttnSingle, kAttnSplit or kAttnWide
 };
 // single: one 64-thread block per (row, kv head) over every page; split: one
 // 64-thread block per page, partial states in global scratch, combined by the
 // last block to finish; wide: split with a 256-thread block per page
 enum { kAttnSingle = 0, kAttnSplit = 1, kAttnWide = 2 };
+
+// Attention output element idx: fp32, or (o_split, the prefill's tensor-core
+// operand) the pair hi = bf16(v) in the first plane and lo = bf16(v - hi) in the
+// second, B * Hq * d elements further on; hi + lo carries v to ~2^-17 relative.
+template <int D>
+__device__ __forceinline__ void store_o(const AttnParams& p, size_t idx, float v) {
+    if (p.o_split) {
+        uint16_t* o16 = reinterpret_cast<uint16_t*>(p.o);
+        const uint16_t hi = f2bf(v);
+        o16[idx] = hi;
+        o16[idx + (size_t)p.B * p.Hq * D] = f2bf(v - bf2f(hi));
+    } else {
+        reinterpret_cast<float*>(p.o)[idx] = v;
+    }
+}
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
@@ -1042,10 +1057,7 @@ __device__ __forceinline__ void attn_group(const AttnParams& p, int row, int kvh
                 for (int c = 0; c < DPL; ++c) {
                     float v = (o[g][c] * c0 + sm.s_o[g][lane * DPL + c] * c1) * invl;
                     size_t idx = (size_t)row * p.Hq * D + (size_t)h * D + lane * DPL + c;
-                    if (p.o_bf16)
-                        reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(v);
-                    else
-                        reinterpret_cast<float*>(p.o)[idx] = v;
+                    store_o<D>(p, idx, v);
                 }
             }
         }
@@ -1119,10 +1131,7 @@ __device__ __forceinline__ void attn_group(const AttnParams& p, int row, int kvh
     for (int k = 0; k < NOUT; ++k) {
         const int e = tid + 64 * k, g = e / D, j = e - g * D;
         const size_t idx = (size_t)row * p.Hq * D + (size_t)(kvh * G + g) * D + j;
-        if (p.o_bf16)
-            reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(acc[k]);
-        else
-            reinterpret_cast<float*>(p.o)[idx] = acc[k];
+        store_o<D>(p, idx, acc[k]);
     }
 }
 
@@ -1380,10 +1389,7 @@ __global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
         const int e = tid + NT * k;
         if (e < G * D) {
             const size_t idx = (size_t)row * p.Hq * D + (size_t)kvh * G * D + e;
-            if (p.o_bf16)
-                reinterpret_cast<uint16_t*>(p.o)[idx] = f2bf(o[k]);
-            else
-                reinterpret_cast<float*>(p.o)[idx] = o[k];
+            store_o<D>(p, idx, o[k]);
         }
     }
 }
@@ -1424,6 +1430,8 @@ struct RunParams {
     int max_chunks;
     unsigned* sync;  // [0] barrier counter, [1] error word, [2 ..] tile counters (4 per layer)
     uint32_t smem_bytes;
+    int skip_block;             // fault injection: this block skips its first barrier arrival (-1: none)
+    uint64_t barrier_limit_ns;  // bound of every barrier wait
     RopeFreqs rope;
 };
 
@@ -1439,15 +1447,18 @@ __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
 }
 
 // Grid-wide barrier: every block arrives once per barrier on a monotonic
-// counter.  The wait is bounded (1 s); a block that gives up sets the error
-// word, and a block that sees the error word stops waiting, so every block
-// leaves the kernel instead of hanging.  Returns false on error.
-__device__ __forceinline__ bool grid_sync(unsigned* sync, unsigned& nsync, int* s_flag) {
+// counter.  The wait is bounded (limit_ns, 1 s by default); a block that gives
+// up sets the error word, and a block that sees the error word stops waiting,
+// so every block leaves the kernel instead of hanging.  Returns false on error.
+// skip_block (fault injection for tests): that block does not arrive at the
+// first barrier, so the barrier cannot complete and every wait runs out.
+__device__ __forceinline__ bool grid_sync(unsigned* sync, unsigned& nsync, int* s_flag, int skip_block,
+                                          uint64_t limit_ns) {
     __syncthreads();
     ++nsync;
     if (threadIdx.x == 0) {
         __threadfence();
-        atomicAdd(&sync[0], 1u);
+        if (!(nsync == 1 && (int)blockIdx.x == skip_block)) atomicAdd(&sync[0], 1u);
         const unsigned target = nsync * gridDim.x;
         const uint64_t t0 = globaltimer_ns();
         int bad = 0;
@@ -1456,7 +1467,7 @@ __device__ __forceinline__ bool grid_sync(unsigned* sync, unsigned& nsync, int* 
                 bad = 1;
                 break;
             }
-            if (globaltimer_ns() - t0 > 1000000000ull) {
+            if (globaltimer_ns() - t0 > limit_ns) {
                 atomicCAS(&sync[1], 0u, 1u);
                 bad = 1;
                 break;
@@ -1654,7 +1665,7 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParam
             s_ap.kv.layer = rp.layer0 + li;
             if (li + 1 < rp.n_layers) set_layer(PH_QKV, li + 1);
         }
-        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        if (!grid_sync(rp.sync, nsync, &s_flag, rp.skip_block, rp.barrier_limit_ns)) return;
         // ---- split attention (groups = warp pairs 0-1 and 2-3); warps 4-7
         //      prefetch this block's O-projection tiles meanwhile
         if (warp < 4) {
@@ -1678,23 +1689,23 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2) decode_run_kernel(RunParam
             for (int kk = k0; kk < (int)kg && blockIdx.x + kk * gridDim.x < ntg; kk += 4)
                 prefetch_tile<EPI_SWIGLU>(gu, blockIdx.x + kk * gridDim.x, lane);
         }
-        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        if (!grid_sync(rp.sync, nsync, &s_flag, rp.skip_block, rp.barrier_limit_ns)) return;
         // ---- O-projection + residual
         run_tiles<EPI_RESID>(s_gp[PH_O], tsm, sx_for(qd), ctr + 4 * li + PH_O, &s_next);
         if (warp == 0) prefetch_tile<EPI_SWIGLU>(s_gp[PH_GU], blockIdx.x, lane);
         if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_O, li + 1);
-        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        if (!grid_sync(rp.sync, nsync, &s_flag, rp.skip_block, rp.barrier_limit_ns)) return;
         // ---- RMSNorm + gate/up SwiGLU
         run_tiles<EPI_SWIGLU>(s_gp[PH_GU], tsm, sx_for(rp.H), ctr + 4 * li + PH_GU, &s_next);
         if (warp == 0) prefetch_tile<EPI_RESID>(s_gp[PH_D], blockIdx.x, lane);
         if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_GU, li + 1);
-        if (!grid_sync(rp.sync, nsync, &s_flag)) return;
+        if (!grid_sync(rp.sync, nsync, &s_flag, rp.skip_block, rp.barrier_limit_ns)) return;
         // ---- down + residual
         run_tiles<EPI_RESID>(s_gp[PH_D], tsm, sx_for(rp.F), ctr + 4 * li + PH_D, &s_next);
         if (tid == 0 && li + 1 < rp.n_layers) set_layer(PH_D, li + 1);
         __syncthreads();
         if (warp == 0 && li + 1 < rp.n_layers) prefetch_tile<EPI_QKV>(s_gp[PH_QKV], blockIdx.x, lane);
-        if (li + 1 < rp.n_layers && !grid_sync(rp.sync, nsync, &s_flag)) return;
+        if (li + 1 < rp.n_layers && !grid_sync(rp.sync, nsync, &s_flag, rp.skip_block, rp.barrier_limit_ns)) return;
     }
 }
 
@@ -1998,7 +2009,7 @@ int* attention_counters(float* scratch, int B, int Hq, int d, int max_ctx, int p
 
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
-                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl, int scratch_rows,
+                             float* scratch, void* o, bool o_split, cudaStream_t st, bool pdl, int scratch_rows,
                              bool wide) {
     AttnParams p{};
     p.q = q;
@@ -2016,7 +2027,7 @@ cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens,
     if (scratch_rows < B) scratch_rows = B;
     p.counters = split ? attention_counters(scratch, scratch_rows, Hq, d, max_ctx, kv.page_tokens) : nullptr;
     p.o = o;
-    p.o_bf16 = o_bf16 ? 1 : 0;
+    p.o_split = o_split ? 1 : 0;
     p.split = split ? kAttnSplit : kAttnSingle;
     if (split && wide) p.split = kAttnWide;
     const int G = Hq / Hkv;
@@ -2097,6 +2108,8 @@ cudaError_t launch_decode_run(const DecodeRunArgs& a, cudaStream_t st) {
     rp.counters = attention_counters(a.attn_scratch, a.scratch_rows < 1 ? 1 : a.scratch_rows, a.Hq, a.d, a.max_ctx,
                                      a.kv.page_tokens);
     rp.sync = a.sync;
+    rp.skip_block = a.skip_block;
+    rp.barrier_limit_ns = a.barrier_limit_us ? (uint64_t)a.barrier_limit_us * 1000ull : 1000000000ull;
     rp.rope = rope_freqs(a.theta, a.d);
     // the barrier counter and the tile counters; the error word (sync[1]) is kept
     cudaError_t e = cudaMemsetAsync(a.sync, 0, sizeof(unsigned), st);

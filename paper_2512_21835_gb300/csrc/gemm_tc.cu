@@ -1,13 +1,23 @@
 // gemm_tc.cu -- prefill projections on the 5th-generation tensor cores.
 //
-// C[M, N] = A[M, K] * W[N, K]^T with A the bf16 activations of M prompt tokens
-// and W a bf16 weight matrix (both K-contiguous), fp32 accumulation in tensor
+// C[M, N] = A[M, K] * W[N, K]^T with A the activations of M prompt tokens and
+// W a bf16 weight matrix (both K-contiguous), fp32 accumulation in tensor
 // memory, fused epilogues (query/key rotation + KV-cache write, residual add,
 // SwiGLU).
 //
+// Activations are fp32 on this path; the tensor cores take bf16 operands of
+// one type (kind::f16).  So an activation matrix is given as a pair of bf16
+// planes, A = A_hi + A_lo with A_hi = bf16(A) and A_lo = bf16(A - A_hi) (a
+// "split" operand, ~16 significant bits), and every K step issues two MMAs
+// into the same accumulator: A_hi W^T and A_lo W^T.  The weights are the
+// model's unmodified bf16 values, so the product equals the fp32-activation
+// product up to fp32 accumulation and the 2^-17 relative residue of the pair.
+// A single bf16 plane (no split) is also supported.
+//
 // One CTA computes a 128 x 256 output tile:
-//   warp 0     TMA producer: 4-stage ring of 48 KB (A 128x64, W 256x64, bf16,
-//              128-byte swizzle), one mbarrier per stage with transaction bytes;
+//   warp 0     TMA producer: a ring of stages (A_hi [, A_lo] 128x64 and W
+//              256x64, bf16, 128-byte swizzle; 4 stages of 48 KB, or 3 of
+//              64 KB when split), one mbarrier per stage with transaction bytes;
 //   warp 1     allocates 256 TMEM columns, one lane issues tcgen05.mma
 //              (M 128, N 256, K 16) and frees a stage with tcgen05.commit;
 //   warps 2-5  epilogue: tcgen05.ld of their 32-lane quadrant, one output row
@@ -31,11 +41,16 @@ __device__ int g_tc_error;  // first failure code of any tensor-core GEMM launch
 
 namespace {
 
-constexpr int TBM = 128, TBN = 256, TBK = 64, STAGES = 4;
-constexpr int A_BYTES = TBM * TBK * 2;          // 16 KB
+constexpr int TBM = 128, TBN = 256, TBK = 64;
+constexpr int A_BYTES = TBM * TBK * 2;          // 16 KB: one plane of the A tile
 constexpr int B_HALF = 128 * TBK * 2;           // 16 KB: one 128-row TMA box of W
-constexpr int STAGE_BYTES = A_BYTES + 2 * B_HALF;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+template <int SPLIT>
+struct Ring {
+    static constexpr int STAGES = SPLIT ? 3 : 4;
+    static constexpr int B_OFF = (SPLIT ? 2 : 1) * A_BYTES;  // W tile after the A plane(s)
+    static constexpr int STAGE_BYTES = B_OFF + 2 * B_HALF;
+    static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+};
 constexpr int kThreadsTC = 192;
 constexpr uint32_t kTmemCols = 256;
 // instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
@@ -48,7 +63,7 @@ enum { T_QKV = 0, T_RESID = 1, T_SWIGLU = 2 };
 struct TcParams {
     int M, N, K;  // N: output columns (QKV, RESID) or F (SWIGLU)
     float* x;
-    uint16_t* a;
+    uint16_t* a;  // SWIGLU output: split pair [2][M][N] (hi plane, then lo plane)
     float* q;
     int Hq, Hkv, d;
     const int32_t* positions;
@@ -133,6 +148,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 __device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
+__device__ __forceinline__ float bf2f(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
 
 __device__ __forceinline__ void record_error(int code) { atomicCAS(&g_tc_error, 0, code); }
 
@@ -171,21 +187,30 @@ __device__ __forceinline__ void epilogue(const TcParams& p, uint32_t tbase, int 
             tmem_ld32(tbase + 128 + c0, u);
             if (!live) continue;
             uint16_t* ar = p.a + (size_t)row * p.N + f0 + c0;
+            const size_t plane = (size_t)p.M * p.N;
             if (f0 + c0 + 32 <= p.N) {
 #pragma unroll
                 for (int j = 0; j < 32; j += 8) {
-                    uint32_t w[4];
+                    uint32_t w[4], wl[4];
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        float s0 = g[j + 2 * e] / (1.0f + expf(-g[j + 2 * e])) * u[j + 2 * e];
-                        float s1 = g[j + 2 * e + 1] / (1.0f + expf(-g[j + 2 * e + 1])) * u[j + 2 * e + 1];
-                        w[e] = (uint32_t)f2bf(s0) | ((uint32_t)f2bf(s1) << 16);
+                        const float s0 = g[j + 2 * e] / (1.0f + expf(-g[j + 2 * e])) * u[j + 2 * e];
+                        const float s1 = g[j + 2 * e + 1] / (1.0f + expf(-g[j + 2 * e + 1])) * u[j + 2 * e + 1];
+                        const uint16_t h0 = f2bf(s0), h1 = f2bf(s1);
+                        w[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+                        wl[e] = (uint32_t)f2bf(s0 - bf2f(h0)) | ((uint32_t)f2bf(s1 - bf2f(h1)) << 16);
                     }
                     *reinterpret_cast<uint4*>(ar + j) = make_uint4(w[0], w[1], w[2], w[3]);
+                    *reinterpret_cast<uint4*>(ar + plane + j) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
                 }
             } else {
                 for (int j = 0; j < 32; ++j)
-                    if (f0 + c0 + j < p.N) ar[j] = f2bf(g[j] / (1.0f + expf(-g[j])) * u[j]);
+                    if (f0 + c0 + j < p.N) {
+                        const float sv = g[j] / (1.0f + expf(-g[j])) * u[j];
+                        const uint16_t h = f2bf(sv);
+                        ar[j] = h;
+                        ar[plane + j] = f2bf(sv - bf2f(h));
+                    }
             }
         }
     } else {  // T_QKV: the tile holds 256 / d whole heads
@@ -245,10 +270,11 @@ __device__ __forceinline__ void epilogue(const TcParams& p, uint32_t tbase, int 
     }
 }
 
-template <int EPI>
+template <int EPI, int SPLIT>
 __global__ void __launch_bounds__(kThreadsTC, 1)
-    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
-                   const __grid_constant__ CUtensorMap tmB1, TcParams p) {
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmAlo,
+                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1, TcParams p) {
+    constexpr int STAGES = Ring<SPLIT>::STAGES, STAGE_BYTES = Ring<SPLIT>::STAGE_BYTES, B_OFF = Ring<SPLIT>::B_OFF;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
@@ -293,8 +319,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
                 mbar_expect_tx(full0 + 8 * s, STAGE_BYTES);
                 tma_load_2d(sa, &tmA, kb * TBK, m0, full0 + 8 * s);
-                tma_load_2d(sa + A_BYTES, &tmB0, kb * TBK, y0, full0 + 8 * s);
-                tma_load_2d(sa + A_BYTES + B_HALF, mb1, kb * TBK, y1, full0 + 8 * s);
+                if (SPLIT) tma_load_2d(sa + A_BYTES, &tmAlo, kb * TBK, m0, full0 + 8 * s);
+                tma_load_2d(sa + B_OFF, &tmB0, kb * TBK, y0, full0 + 8 * s);
+                tma_load_2d(sa + B_OFF + B_HALF, mb1, kb * TBK, y1, full0 + 8 * s);
                 ++issued;
             }
             // the copies of the last stages must land before this CTA's shared
@@ -313,10 +340,12 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 }
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
-                const uint64_t da = smem_desc(sa), db = smem_desc(sa + A_BYTES);
+                const uint64_t da = smem_desc(sa), db = smem_desc(sa + B_OFF);
 #pragma unroll
-                for (int k = 0; k < TBK / 16; ++k)  // 32 bytes along K per instruction
+                for (int k = 0; k < TBK / 16; ++k) {  // 32 bytes along K per instruction
                     umma_bf16(tmem, da + 2 * k, db + 2 * k, (kb | k) != 0 ? 1u : 0u);
+                    if (SPLIT) umma_bf16(tmem, smem_desc(sa + A_BYTES) + 2 * k, db + 2 * k, 1u);  // + A_lo W^T
+                }
                 umma_commit(empty0 + 8 * s);
             }
             umma_commit(accb);  // arrives once every MMA issued above has completed
@@ -364,32 +393,44 @@ cudaError_t make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t K)
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int EPI>
-cudaError_t launch_tc(const void* A, const void* W0, const void* W1, uint64_t w_rows, TcParams& p, int n_tiles,
-                      cudaStream_t st) {
+template <int EPI, int SPLIT>
+cudaError_t launch_tc_t(const void* A, const void* W0, const void* W1, uint64_t w_rows, TcParams& p, int n_tiles,
+                        cudaStream_t st) {
     cudaError_t e = encoder();
     if (e != cudaSuccess) return e;
     if (p.M <= 0 || n_tiles <= 0) return cudaSuccess;
-    CUtensorMap ma, mb0, mb1;
-    if ((e = make_map(&ma, A, (uint64_t)p.M, (uint64_t)p.K)) != cudaSuccess) return e;
+    CUtensorMap ma, malo, mb0, mb1;
+    const uint16_t* A16 = static_cast<const uint16_t*>(A);
+    if ((e = make_map(&ma, A16, (uint64_t)p.M, (uint64_t)p.K)) != cudaSuccess) return e;
+    // the lo plane follows the hi plane (M * K elements on)
+    if ((e = make_map(&malo, SPLIT ? A16 + (size_t)p.M * p.K : A16, (uint64_t)p.M, (uint64_t)p.K)) != cudaSuccess)
+        return e;
     if ((e = make_map(&mb0, W0, w_rows, (uint64_t)p.K)) != cudaSuccess) return e;
     if ((e = make_map(&mb1, W1 ? W1 : W0, w_rows, (uint64_t)p.K)) != cudaSuccess) return e;
+    constexpr int SMEM = Ring<SPLIT>::SMEM_BYTES;
     static bool attr = false;
     if (!attr) {
-        e = cudaFuncSetAttribute(tc_gemm_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+        e = cudaFuncSetAttribute(tc_gemm_kernel<EPI, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
         if (e != cudaSuccess) return e;
         attr = true;
     }
     dim3 grid((p.M + TBM - 1) / TBM, n_tiles);
-    tc_gemm_kernel<EPI><<<grid, kThreadsTC, SMEM_BYTES, st>>>(ma, mb0, mb1, p);
+    tc_gemm_kernel<EPI, SPLIT><<<grid, kThreadsTC, SMEM, st>>>(ma, malo, mb0, mb1, p);
     return cudaGetLastError();
+}
+
+template <int EPI>
+cudaError_t launch_tc(const void* A, bool split, const void* W0, const void* W1, uint64_t w_rows, TcParams& p,
+                      int n_tiles, cudaStream_t st) {
+    return split ? launch_tc_t<EPI, 1>(A, W0, W1, w_rows, p, n_tiles, st)
+                 : launch_tc_t<EPI, 0>(A, W0, W1, w_rows, p, n_tiles, st);
 }
 
 }  // namespace
 
-cudaError_t launch_tc_gemm_qkv_rope(const uint16_t* y, const uint16_t* wqkv, int M, int H, int Hq, int Hkv, int d,
-                                 float theta, const int32_t* positions, const int32_t* row_req, float* q, KvView kv,
-                                 cudaStream_t st) {
+cudaError_t launch_tc_gemm_qkv_rope(const uint16_t* y, bool split, const uint16_t* wqkv, int M, int H, int Hq,
+                                    int Hkv, int d, float theta, const int32_t* positions, const int32_t* row_req,
+                                    float* q, KvView kv, cudaStream_t st) {
     if (TBN % d != 0) return cudaErrorInvalidValue;
     TcParams p{};
     p.M = M;
@@ -403,26 +444,27 @@ cudaError_t launch_tc_gemm_qkv_rope(const uint16_t* y, const uint16_t* wqkv, int
     p.row_req = row_req;
     p.kv = kv;
     p.rope = rope_freqs(theta, d);
-    return launch_tc<T_QKV>(y, wqkv, nullptr, (uint64_t)p.N, p, (p.N + TBN - 1) / TBN, st);
+    return launch_tc<T_QKV>(y, split, wqkv, nullptr, (uint64_t)p.N, p, (p.N + TBN - 1) / TBN, st);
 }
 
-cudaError_t launch_tc_gemm_resid(const uint16_t* a, const uint16_t* w, int M, int N, int K, float* x, cudaStream_t st) {
+cudaError_t launch_tc_gemm_resid(const uint16_t* a, bool split, const uint16_t* w, int M, int N, int K, float* x,
+                                 cudaStream_t st) {
     TcParams p{};
     p.M = M;
     p.N = N;
     p.K = K;
     p.x = x;
-    return launch_tc<T_RESID>(a, w, nullptr, (uint64_t)N, p, (N + TBN - 1) / TBN, st);
+    return launch_tc<T_RESID>(a, split, w, nullptr, (uint64_t)N, p, (N + TBN - 1) / TBN, st);
 }
 
-cudaError_t launch_tc_gemm_swiglu(const uint16_t* y, const uint16_t* wg, const uint16_t* wu, int M, int H, int F,
-                               uint16_t* a, cudaStream_t st) {
+cudaError_t launch_tc_gemm_swiglu(const uint16_t* y, bool split, const uint16_t* wg, const uint16_t* wu, int M, int H,
+                                  int F, uint16_t* a, cudaStream_t st) {
     TcParams p{};
     p.M = M;
     p.N = F;
     p.K = H;
     p.a = a;
-    return launch_tc<T_SWIGLU>(y, wg, wu, (uint64_t)F, p, (F + 127) / 128, st);
+    return launch_tc<T_SWIGLU>(y, split, wg, wu, (uint64_t)F, p, (F + 127) / 128, st);
 }
 
 cudaError_t tc_error(int* code) {

@@ -13,13 +13,24 @@
 // pages in), then registered with cudaHostRegister; cudaHostAlloc is the
 // fallback when that fails.  Every buffer is registered mapped, so kernels can
 // also read it in place through its device address (direct-access decode).
+//
+// Placement: before the first touch the mapping is given the memory policy
+// MPOL_PREFERRED for the host NUMA node closest to the GPU
+// (cudaDevAttrHostNumaId), so that its pages come from the memory next to the
+// link the copy engine reads over (preferred, not bound: when that node runs
+// out the kernel falls back to another node instead of failing the fault).  The
+// runtime reads back where the pages landed (move_pages queries).
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
 #include <sys/mman.h>
+#include <sys/stat.h>
+#include <sys/syscall.h>
 #include <unistd.h>
+
+#include <vector>
 
 #include "hostpool.h"
 
@@ -50,6 +61,53 @@ static void map_device(HostBuf* b) {
     }
 }
 
+int gpu_host_node() {
+    int dev = 0, node = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&node, cudaDevAttrHostNumaId, dev) != cudaSuccess) {
+        cudaGetLastError();
+        return -1;
+    }
+    if (node < 0 || node >= 1024) return -1;
+    char path[64];
+    snprintf(path, sizeof path, "/sys/devices/system/node/node%d", node);
+    struct stat st;
+    return stat(path, &st) == 0 ? node : -1;
+}
+
+// MPOL_PREFERRED for `node` on [p, p + bytes) (Linux memory-policy constant).
+static bool prefer_node(void* p, size_t bytes, int node) {
+    constexpr int kMpolPreferred = 1;
+    unsigned long mask[1024 / (8 * sizeof(unsigned long))] = {};
+    mask[node / (8 * sizeof(unsigned long))] |= 1ul << (node % (8 * sizeof(unsigned long)));
+    return syscall(SYS_mbind, p, bytes, kMpolPreferred, mask, (unsigned long)1024, 0u) == 0;
+}
+
+int host_range_node(const void* p, size_t bytes, int samples, double* frac) {
+    if (frac) *frac = 0.0;
+    if (!p || bytes == 0 || samples < 1) return -1;
+    const size_t pg = (size_t)sysconf(_SC_PAGESIZE);
+    std::vector<void*> pages(samples);
+    std::vector<int> status(samples, -1);
+    for (int i = 0; i < samples; ++i) {
+        const uintptr_t a = reinterpret_cast<uintptr_t>(p) + (bytes - 1) * (size_t)i / (size_t)(samples > 1 ? samples - 1 : 1);
+        pages[i] = reinterpret_cast<void*>(a / pg * pg);
+    }
+    if (syscall(SYS_move_pages, 0, (unsigned long)samples, pages.data(), nullptr, status.data(), 0) != 0) return -1;
+    int best = -1, best_n = 0;
+    for (int i = 0; i < samples; ++i) {
+        if (status[i] < 0) continue;
+        int n = 0;
+        for (int j = 0; j < samples; ++j) n += status[j] == status[i];
+        if (n > best_n) {
+            best_n = n;
+            best = status[i];
+        }
+    }
+    if (frac) *frac = (double)best_n / samples;
+    return best;
+}
+
 cudaError_t host_buf_alloc(size_t bytes, HostBuf* out) {
     *out = HostBuf{};
     if (bytes == 0) return cudaSuccess;
@@ -69,6 +127,8 @@ cudaError_t host_buf_alloc(size_t bytes, HostBuf* out) {
     void* base = mmap(nullptr, map_bytes, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
     if (base != MAP_FAILED) {
         char* p = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(base) + hp - 1) / hp * hp);
+        const int node = gpu_host_node();
+        const bool placed = node >= 0 && prefer_node(p, bytes, node);
         madvise(p, bytes, MADV_HUGEPAGE);
         memset(p, 0, bytes);
         if (cudaHostRegister(p, bytes, cudaHostRegisterPortable | cudaHostRegisterMapped) == cudaSuccess) {
@@ -77,6 +137,7 @@ cudaError_t host_buf_alloc(size_t bytes, HostBuf* out) {
             out->ptr = p;
             out->bytes = bytes;
             out->mapped = true;
+            out->node = placed ? node : -1;
             map_device(out);
             return cudaSuccess;
         }

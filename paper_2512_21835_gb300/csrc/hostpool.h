@@ -11,7 +11,15 @@ struct HostBuf {
     size_t bytes = 0;
     bool mapped = false;   // mmap + cudaHostRegister (else cudaHostAlloc)
     void* dev = nullptr;   // device address of ptr (registered mapped), or nullptr
+    int node = -1;         // host NUMA node the pages were asked for (-1: none)
 };
+// Host NUMA node closest to the current device (cudaDevAttrHostNumaId), or -1
+// when the system reports none or the node does not exist on this host.
+int gpu_host_node();
+// Majority NUMA node of `samples` pages spread evenly over [p, p + bytes)
+// (move_pages query, pages already touched); *frac gets the share of sampled
+// pages on that node.  -1 when the kernel cannot tell.
+int host_range_node(const void* p, size_t bytes, int samples, double* frac);
 cudaError_t host_buf_alloc(size_t bytes, HostBuf* out);
 // plain cudaHostAlloc buffer (the SSD tier's staging buffers: O_DIRECT reads
 // land in them, and copies out of registered huge-page mappings that direct I/O

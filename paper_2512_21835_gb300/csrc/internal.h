@@ -75,14 +75,16 @@ size_t lm_head_scratch_bytes(int B, int V);
 // page-table row (NULL = identity).  split: one block per page writes its
 // partial state to scratch and the last block of each (row, kv head) combines
 // them into o (max_ctx <= 16384); otherwise one block per (row, kv head) loops
-// over all pages.  o_bf16: write o as bf16 (prefill) instead of fp32.
+// over all pages.  o_split: write o as a pair of bf16 planes [2][B][Hq d],
+// hi = bf16(v) and lo = bf16(v - hi) (the prefill's tensor-core operand),
+// instead of fp32.
 // scratch_rows: the batch the scratch was sized for (attention_scratch_floats);
 // the completion counters sit after that many rows of partial states, so the
 // same scratch serves every batch up to it (0 = B).  wide: split mode with a
 // 256-thread block per page (same scratch layout and counters).
 cudaError_t launch_attention(const float* q, KvView kv, const int32_t* ctx_lens, const int32_t* positions,
                              const int32_t* row_req, int B, int Hq, int Hkv, int d, int max_ctx, bool split,
-                             float* scratch, void* o, bool o_bf16, cudaStream_t st, bool pdl = false,
+                             float* scratch, void* o, bool o_split, cudaStream_t st, bool pdl = false,
                              int scratch_rows = 0, bool wide = false);
 size_t attention_scratch_floats(int B, int Hq, int d, int max_ctx, int page_tokens);
 // Split attention keeps one int completion counter per (row, head) after the
@@ -114,6 +116,8 @@ struct DecodeRunArgs {
     float* attn_scratch;             // attention_scratch_floats(scratch_rows, Hq, d, max_ctx, page_tokens)
     int scratch_rows, max_ctx;
     unsigned* sync;                  // [2 + 4 * kMaxRunLayers]: barrier, error word, tile counters
+    int skip_block;                  // fault injection: block that skips its first barrier arrival (-1: none)
+    uint32_t barrier_limit_us;       // bound of each barrier wait (0: 1 s)
 };
 bool decode_run_supported(int Hq, int Hkv, int d);
 cudaError_t launch_decode_run(const DecodeRunArgs& a, cudaStream_t st);
@@ -124,17 +128,21 @@ cudaError_t launch_advance(int32_t* positions, int B, cudaStream_t st, bool pdl 
 cudaError_t launch_generate(uint16_t* out, uint64_t n, uint64_t first, uint64_t seed, uint32_t tensor_id, int kind,
                             cudaStream_t st);
 
-// Prefill (M tokens at once).
-cudaError_t launch_rmsnorm_bf16(const float* x, const uint16_t* g, int M, int H, float eps, uint16_t* y,
-                                cudaStream_t st);
-// Prefill projections on the tensor cores (tcgen05, TMA), fused epilogues.
-cudaError_t launch_tc_gemm_qkv_rope(const uint16_t* y, const uint16_t* wqkv, int M, int H, int Hq, int Hkv, int d,
-                                    float theta, const int32_t* positions, const int32_t* row_req, float* q,
-                                    KvView kv, cudaStream_t st);
-cudaError_t launch_tc_gemm_resid(const uint16_t* a, const uint16_t* w, int M, int N, int K, float* x,
+// Prefill (M tokens at once).  y = RMSNorm(x) * g as a split pair of bf16
+// planes [2][M][H]: hi = bf16(y), lo = bf16(y - hi).
+cudaError_t launch_rmsnorm_split(const float* x, const uint16_t* g, int M, int H, float eps, uint16_t* y,
                                  cudaStream_t st);
-cudaError_t launch_tc_gemm_swiglu(const uint16_t* y, const uint16_t* wg, const uint16_t* wu, int M, int H, int F,
-                                  uint16_t* a, cudaStream_t st);
+// Prefill projections on the tensor cores (tcgen05, TMA), fused epilogues.
+// The activation operand (y, a) is a split pair of bf16 planes [2][M][K] when
+// `split` is set (two MMAs per K step), else one bf16 plane [M][K].  The
+// SwiGLU output `a` is always written as a split pair [2][M][F].
+cudaError_t launch_tc_gemm_qkv_rope(const uint16_t* y, bool split, const uint16_t* wqkv, int M, int H, int Hq,
+                                    int Hkv, int d, float theta, const int32_t* positions, const int32_t* row_req,
+                                    float* q, KvView kv, cudaStream_t st);
+cudaError_t launch_tc_gemm_resid(const uint16_t* a, bool split, const uint16_t* w, int M, int N, int K, float* x,
+                                 cudaStream_t st);
+cudaError_t launch_tc_gemm_swiglu(const uint16_t* y, bool split, const uint16_t* wg, const uint16_t* wu, int M, int H,
+                                  int F, uint16_t* a, cudaStream_t st);
 // First failure code recorded by a tensor-core GEMM launch (0 = none).
 cudaError_t tc_error(int* code);
 cudaError_t launch_gather_rows(const float* x, const int32_t* rows, int n, int H, float* out, cudaStream_t st);

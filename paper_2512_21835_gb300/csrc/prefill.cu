@@ -1,7 +1,9 @@
 // prefill.cu -- the row-wise pieces of a prefill pass: the RMSNorm that feeds
-// each tensor-core projection (its output rounded to bf16, the GEMM operand
-// type; the residual stream stays fp32) and a row gather.  The projections
-// themselves are in gemm_tc.cu.
+// each tensor-core projection and a row gather.  The projections themselves
+// are in gemm_tc.cu.  The normed rows are computed in fp32 and written as the
+// GEMM's split operand, a pair of bf16 planes: hi = bf16(y) and lo =
+// bf16(y - hi), so the projection sees y to ~2^-17 relative (the residual
+// stream stays fp32).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -15,7 +17,7 @@ namespace {
 __device__ __forceinline__ float bf2f(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
 __device__ __forceinline__ uint16_t f2bf(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
 
-__global__ void rmsnorm_bf16_kernel(const float* x, const uint16_t* g, int H, float eps, uint16_t* y) {
+__global__ void rmsnorm_split_kernel(const float* x, const uint16_t* g, int H, float eps, uint16_t* y) {
     __shared__ float red[32];
     const int m = blockIdx.x;
     const float* xr = x + (size_t)m * H;
@@ -31,7 +33,13 @@ __global__ void rmsnorm_bf16_kernel(const float* x, const uint16_t* g, int H, fl
     }
     __syncthreads();
     const float inv = red[0];
-    for (int k = threadIdx.x; k < H; k += blockDim.x) y[(size_t)m * H + k] = f2bf(xr[k] * inv * bf2f(g[k]));
+    const size_t plane = (size_t)gridDim.x * H;  // rows = gridDim.x
+    for (int k = threadIdx.x; k < H; k += blockDim.x) {
+        const float v = xr[k] * inv * bf2f(g[k]);
+        const uint16_t hi = f2bf(v);
+        y[(size_t)m * H + k] = hi;
+        y[plane + (size_t)m * H + k] = f2bf(v - bf2f(hi));
+    }
 }
 
 __global__ void gather_rows_kernel(const float* x, const int32_t* rows, int H, float* out) {
@@ -42,10 +50,10 @@ __global__ void gather_rows_kernel(const float* x, const int32_t* rows, int H, f
 
 }  // namespace
 
-cudaError_t launch_rmsnorm_bf16(const float* x, const uint16_t* g, int M, int H, float eps, uint16_t* y,
-                                cudaStream_t st) {
+cudaError_t launch_rmsnorm_split(const float* x, const uint16_t* g, int M, int H, float eps, uint16_t* y,
+                                 cudaStream_t st) {
     if (M <= 0) return cudaSuccess;
-    rmsnorm_bf16_kernel<<<M, 256, 0, st>>>(x, g, H, eps, y);
+    rmsnorm_split_kernel<<<M, 256, 0, st>>>(x, g, H, eps, y);
     return cudaGetLastError();
 }
 

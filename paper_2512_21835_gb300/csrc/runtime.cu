@@ -38,6 +38,31 @@ namespace {
 
 thread_local std::string g_create_error;
 
+// The deadline loop of every host wait: polls query() (cudaSuccess: done,
+// cudaErrorNotReady: pending, anything else: failed) until it is not pending
+// or timeout_ms of wall time have passed (*timed_out set, returns
+// cudaErrorNotReady).  Host code only; the poll is the only device contact.
+template <class Q>
+cudaError_t poll_until(Q query, uint32_t timeout_ms, bool* timed_out, double* waited_ms) {
+    const auto t0 = std::chrono::steady_clock::now();
+    auto ms = [&] { return std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count(); };
+    *timed_out = false;
+    for (;;) {
+        const cudaError_t r = query();
+        if (r != cudaErrorNotReady) {
+            if (waited_ms) *waited_ms = ms();
+            return r;
+        }
+        const double w = ms();
+        if (w > (double)timeout_ms) {
+            *timed_out = true;
+            if (waited_ms) *waited_ms = w;
+            return cudaErrorNotReady;
+        }
+        std::this_thread::yield();
+    }
+}
+
 constexpr uint64_t kAlign = 256;
 inline uint64_t align_up(uint64_t v, uint64_t a = kAlign) { return (v + a - 1) / a * a; }
 
@@ -141,11 +166,12 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     f.page_table = take(B * max_pages * 8);
     f.run_sync = take(4 * (2 + 4 * kMaxRunLayers));
     f.qk_raw = d->qk_norm ? take(rows * (uint64_t)(d->n_heads + 2 * d->n_kv_heads) * d->head_dim * 4) : 0;
+    // prefill: residual rows fp32; GEMM operands as split pairs of bf16 planes
     f.px = take(Mp * H * 4);
-    f.py = take(Mp * H * 2);
+    f.py = take(2 * Mp * H * 2);
     f.pq = take(Mp * qd * 4);
-    f.po = take(Mp * qd * 2);
-    f.pa = take(Mp * F * 2);
+    f.po = take(2 * Mp * qd * 2);
+    f.pa = take(2 * Mp * F * 2);
     f.total = off;
     return f;
 }
@@ -206,8 +232,15 @@ struct loip_ctx {
     struct CopyEv {
         cudaEvent_t a, b;
         bool ssd;  // out of an SSD-tier staging buffer
+        uint64_t bytes;
     };
     std::deque<CopyEv> copy_events;
+    // duration and size of the most recent completed layer copies (loip_get_copy_log)
+    static constexpr size_t kCopyLog = 8192;
+    std::vector<std::pair<float, uint64_t>> copy_log;
+    size_t copy_log_next = 0;
+    // where the host pool's pages landed: majority NUMA node of each pooled blob (-1: none)
+    std::vector<int> pool_node;
     std::vector<cudaEvent_t> event_pool;
     uint64_t copy_seq = 0, compute_seq = 0;
     bool ktiming = false;
@@ -222,6 +255,13 @@ struct loip_ctx {
     std::deque<KEv> kernel_events;
     bool weights_loaded = false;
     bool failed = false;
+    // fault injection (loip_inject_fault): one armed fault, fired once
+    int fault_kind = 0, fault_arg = 0;
+    bool take_fault(int kind) {
+        if (fault_kind != kind) return false;
+        fault_kind = 0;
+        return true;
+    }
     int active_batch = 0;
     loip_stats st{};
     std::string err;
@@ -257,18 +297,17 @@ struct loip_ctx {
     }
 
     int wait_event(cudaEvent_t e) {
-        auto t0 = std::chrono::steady_clock::now();
-        for (;;) {
-            cudaError_t r = cudaEventQuery(e);
-            if (r == cudaSuccess) return LOIP_OK;
-            if (r != cudaErrorNotReady) return cuda_fail(r, "device work failed");
-            double ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0).count();
-            if (ms > (double)cfg.timeout_ms) {
-                failed = true;
-                return fail(LOIP_ERR_TIMEOUT, "timed out waiting for the device");
-            }
-            std::this_thread::yield();
+        // an injected wait fault reports the event as pending until the deadline
+        const bool stuck = take_fault(LOIP_FAULT_WAIT);
+        bool timed_out = false;
+        cudaError_t r = poll_until([&] { return stuck ? cudaErrorNotReady : cudaEventQuery(e); }, cfg.timeout_ms,
+                                   &timed_out, nullptr);
+        if (timed_out) {
+            failed = true;
+            return fail(LOIP_ERR_TIMEOUT, "timed out waiting for the device");
         }
+        if (r != cudaSuccess) return cuda_fail(r, "device work failed");
+        return LOIP_OK;
     }
 
     // After a host sync point: a layer-run kernel whose grid barrier timed out
@@ -487,6 +526,8 @@ struct loip_ctx {
 
     // ---- streaming ------------------------------------------------------------
     int enqueue_copy(int layer, int slot, cudaStream_t cs) {
+        if (take_fault(LOIP_FAULT_COPY))  // as if the copy call had failed; nothing is enqueued
+            return cuda_fail(cudaErrorInvalidValue, "layer copy (injected fault)");
         cudaError_t e = cudaStreamWaitEvent(cs, slot_free[slot], 0);
         if (e != cudaSuccess) return cuda_fail(e, "copy wait");
         const char* src = static_cast<const char*>(host_layer[layer]);
@@ -510,7 +551,7 @@ struct loip_ctx {
             if (rc) return rc;
         }
         cudaEventRecord(e1, cs);
-        copy_events.push_back({e0, e1, sb >= 0});
+        copy_events.push_back({e0, e1, sb >= 0, off1 - off0});
         e = cudaEventRecord(slot_full[slot], cs);
         if (e != cudaSuccess) return cuda_fail(e, "slot event");
         st.h2d_weight_bytes += stream_bytes(layer);
@@ -668,18 +709,18 @@ struct loip_ctx {
         const int64_t* pt = fixed_ptr<int64_t>(fx.page_table);
         KvView kv = kv_view(l, pt);
         cudaError_t e;
-        e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, wa + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s); });
+        e = timed(11, s, [&] { return launch_rmsnorm_split(px, wa + lay.off_g_attn / 2, Mc, H, desc.rms_eps, py, s); });
         if (e == cudaSuccess && !desc.qk_norm)
             e = timed(6, s, [&] {
-                return launch_tc_gemm_qkv_rope(py, wa + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos, req,
-                                               pq, kv, s);
+                return launch_tc_gemm_qkv_rope(py, true, wa + lay.off_wqkv / 2, Mc, H, Hq, Hkv, d, desc.rope_theta, pos,
+                                               req, pq, kv, s);
             });
         if (e == cudaSuccess && desc.qk_norm)  // raw projections (GEMM into zeros), then norm + rotation + stores
             e = timed(6, s, [&] {
                 const int nqkv = (Hq + 2 * Hkv) * d;
                 float* raw = fixed_ptr<float>(fx.qk_raw);
                 cudaError_t r = cudaMemsetAsync(raw, 0, (size_t)Mc * nqkv * 4, s);
-                if (r == cudaSuccess) r = launch_tc_gemm_resid(py, wa + lay.off_wqkv / 2, Mc, nqkv, H, raw, s);
+                if (r == cudaSuccess) r = launch_tc_gemm_resid(py, true, wa + lay.off_wqkv / 2, Mc, nqkv, H, raw, s);
                 if (r == cudaSuccess)
                     r = launch_qk_norm_rope(raw, Mc, Hq, Hkv, d, true, wa + lay.off_g_q / 2, wa + lay.off_g_k / 2,
                                             desc.rms_eps, desc.rope_theta, pos, req, pq, kv, s);
@@ -690,14 +731,16 @@ struct loip_ctx {
                 return launch_attention(pq, kv, nullptr, pos, req, Mc, Hq, Hkv, d, cfg.max_ctx, false, nullptr, po,
                                         true, s);
             });
-        if (e == cudaSuccess) e = timed(8, s, [&] { return launch_tc_gemm_resid(po, wa + lay.off_wo / 2, Mc, H, qd, px, s); });
         if (e == cudaSuccess)
-            e = timed(11, s, [&] { return launch_rmsnorm_bf16(px, wm + lay.off_g_mlp / 2, Mc, H, desc.rms_eps, py, s); });
+            e = timed(8, s, [&] { return launch_tc_gemm_resid(po, true, wa + lay.off_wo / 2, Mc, H, qd, px, s); });
+        if (e == cudaSuccess)
+            e = timed(11, s, [&] { return launch_rmsnorm_split(px, wm + lay.off_g_mlp / 2, Mc, H, desc.rms_eps, py, s); });
         if (e == cudaSuccess)
             e = timed(9, s, [&] {
-                return launch_tc_gemm_swiglu(py, wm + lay.off_wg / 2, wm + lay.off_wu / 2, Mc, H, F, pa, s);
+                return launch_tc_gemm_swiglu(py, true, wm + lay.off_wg / 2, wm + lay.off_wu / 2, Mc, H, F, pa, s);
             });
-        if (e == cudaSuccess) e = timed(10, s, [&] { return launch_tc_gemm_resid(pa, wm + lay.off_wd / 2, Mc, H, F, px, s); });
+        if (e == cudaSuccess)
+            e = timed(10, s, [&] { return launch_tc_gemm_resid(pa, true, wm + lay.off_wd / 2, Mc, H, F, px, s); });
         if (e != cudaSuccess) return cuda_fail(e, "prefill kernel");
         return LOIP_OK;
     }
@@ -735,6 +778,12 @@ struct loip_ctx {
             a.scratch_rows = cfg.max_batch;
             a.max_ctx = cfg.max_ctx;
             a.sync = fixed_ptr<unsigned>(fx.run_sync);
+            a.skip_block = -1;
+            a.barrier_limit_us = 0;
+            if (take_fault(LOIP_FAULT_BARRIER)) {  // one block misses the first barrier; waits give up after 10 ms
+                a.skip_block = fault_arg;
+                a.barrier_limit_us = 10000;
+            }
             chain = false;
             cudaError_t e = timed(12, s, [&] { return launch_decode_run(a, s); });
             chain = false;
@@ -811,6 +860,9 @@ struct loip_ctx {
             busy += ms;
             st.copy_ms_total += ms;
             st.copies_total += 1;
+            if (copy_log.size() < kCopyLog) copy_log.resize(kCopyLog);
+            copy_log[copy_log_next % kCopyLog] = {ms, ce.bytes};
+            ++copy_log_next;
             if (ce.ssd) st.ssd_copy_ms += ms;
             event_pool.push_back(ce.a);
             event_pool.push_back(ce.b);
@@ -1016,9 +1068,28 @@ struct loip_ctx {
         for (int l : pooled) mn = std::min(mn, r[l]);
         st.pool_min_GBps = mn;
         st.pool_median_GBps = median;
+        record_pool_placement(pooled);
         event_pool.push_back(a);
         event_pool.push_back(b);
         return LOIP_OK;
+    }
+
+    // Where the pooled blobs' pages landed (32 sampled pages per blob) against
+    // the node the pool asked for (the GPU's host node).
+    void record_pool_placement(const std::vector<int>& pooled) {
+        pool_node.assign(L, -1);
+        int want = -1;
+        for (const HostBuf& hb : host_regions)
+            if (hb.node >= 0) want = hb.node;
+        int on = 0;
+        for (int l : pooled) {
+            double frac = 0;
+            pool_node[l] = host_range_node(host_layer[l], lay.l_size, 32, &frac);
+            on += (want >= 0 && pool_node[l] == want) ? 1 : 0;
+        }
+        st.pool_numa_node = want;
+        st.pool_blobs = (int32_t)pooled.size();
+        st.pool_blobs_on_node = on;
     }
 
     // One pinned region for every offloaded layer that has no host copy yet.
@@ -1028,7 +1099,8 @@ struct loip_ctx {
             if (offloaded[l] && !host_layer[l] && disk_off[l] < 0) need.push_back(l);
         if (need.empty()) return LOIP_OK;
         HostBuf b;
-        cudaError_t e = host_buf_alloc(need.size() * lay.l_size, &b);
+        cudaError_t e = take_fault(LOIP_FAULT_HOST_ALLOC) ? cudaErrorMemoryAllocation
+                                                           : host_buf_alloc(need.size() * lay.l_size, &b);
         if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
         host_regions.push_back(b);
         for (size_t i = 0; i < need.size(); ++i)
@@ -1701,6 +1773,50 @@ extern "C" int loip_prefill(loip_ctx* c, const int32_t* tokens, const int32_t* p
     return LOIP_OK;
 }
 
+extern "C" int32_t loip_get_copy_log(loip_ctx* c, double* ms, uint64_t* bytes, int32_t max_n) {
+    if (!c || max_n < 0 || (max_n > 0 && (!ms || !bytes))) return -1;
+    c->collect_copy_time();
+    const size_t have = std::min<size_t>(c->copy_log_next, loip_ctx::kCopyLog);
+    const size_t n = std::min<size_t>(have, (size_t)max_n);
+    for (size_t i = 0; i < n; ++i) {  // oldest of the last n first
+        const auto& e = c->copy_log[(c->copy_log_next - n + i) % loip_ctx::kCopyLog];
+        ms[i] = e.first;
+        bytes[i] = e.second;
+    }
+    return (int32_t)n;
+}
+
+extern "C" int loip_get_pool_nodes(loip_ctx* c, int32_t* nodes) {
+    if (!c || !nodes) return LOIP_ERR_INVALID;
+    for (int l = 0; l < c->L; ++l) nodes[l] = l < (int)c->pool_node.size() ? c->pool_node[l] : -1;
+    return LOIP_OK;
+}
+
+extern "C" int loip_inject_fault(loip_ctx* c, int32_t kind, int32_t arg) {
+    CTX_GUARD(c);
+    if (kind != LOIP_FAULT_NONE && kind != LOIP_FAULT_WAIT && kind != LOIP_FAULT_COPY &&
+        kind != LOIP_FAULT_HOST_ALLOC && kind != LOIP_FAULT_BARRIER)
+        return c->fail(LOIP_ERR_INVALID, "fault kind");
+    if (kind == LOIP_FAULT_BARRIER && arg < 0) return c->fail(LOIP_ERR_INVALID, "fault block");
+    c->fault_kind = kind;
+    c->fault_arg = arg;
+    return LOIP_OK;
+}
+
+extern "C" int loip_poll_deadline_check(uint32_t timeout_ms, int32_t pending_polls, double* waited_ms) {
+    int32_t polls = 0;
+    bool timed_out = false;
+    const cudaError_t r = poll_until(
+        [&] {
+            if (pending_polls >= 0 && polls >= pending_polls) return cudaSuccess;
+            ++polls;
+            return cudaErrorNotReady;
+        },
+        timeout_ms, &timed_out, waited_ms);
+    if (timed_out) return LOIP_ERR_TIMEOUT;
+    return r == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA;
+}
+
 extern "C" int loip_replan(loip_ctx* c, int32_t lookahead_tokens) {
     CTX_GUARD(c);
     if (lookahead_tokens < 0) return c->fail(LOIP_ERR_INVALID, "lookahead");
@@ -1917,7 +2033,16 @@ extern "C" int loip_k_gemm_bf16(const uint16_t* A, const uint16_t* W, int32_t M,
                                 void* stream) {
     if (!A || !W || !x || M < 1 || N < 1 || K < 8 || K % 8 || !al16(A) || !al16(W) || !al16(x) || N % 4)
         return LOIP_ERR_INVALID;
-    cudaError_t e = launch_tc_gemm_resid(A, W, M, N, K, x, (cudaStream_t)stream);
+    cudaError_t e = launch_tc_gemm_resid(A, false, W, M, N, K, x, (cudaStream_t)stream);
+    return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA;
+}
+
+extern "C" int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t M, int32_t N, int32_t K, float* x,
+                                 void* stream) {
+    // the lo plane starts M * K elements after the hi plane: 16-byte aligned too
+    if (!A2 || !W || !x || M < 1 || N < 1 || K < 8 || K % 8 || !al16(A2) || !al16(W) || !al16(x) || N % 4)
+        return LOIP_ERR_INVALID;
+    cudaError_t e = launch_tc_gemm_resid(A2, true, W, M, N, K, x, (cudaStream_t)stream);
     return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA;
 }
 

@@ -17,6 +17,7 @@ LIB_PATH = os.path.join(_HERE, "libloip.so")
 
 OK, ERR_INVALID, ERR_OOM, ERR_INFEASIBLE, ERR_CUDA, ERR_TIMEOUT, ERR_STATE = range(7)
 MODE_OVERLAP, MODE_NAIVE, MODE_DIRECT = 0, 1, 2
+FAULT_NONE, FAULT_WAIT, FAULT_COPY, FAULT_HOST_ALLOC, FAULT_BARRIER = range(5)
 _NAMES = {1: "INVALID", 2: "OOM", 3: "INFEASIBLE", 4: "CUDA", 5: "TIMEOUT", 6: "STATE"}
 
 
@@ -60,7 +61,8 @@ class Stats(C.Structure):
                 ("copy_ms_total", C.c_double), ("copies_total", C.c_uint64),
                 ("pool_min_GBps", C.c_double), ("pool_median_GBps", C.c_double), ("pool_replaced", C.c_uint64),
                 ("n_ssd_layers", C.c_int32), ("ssd_read_bytes", C.c_uint64), ("ssd_wait_ms", C.c_double),
-                ("ssd_stage_wait_ms", C.c_double), ("ssd_copy_ms", C.c_double)]
+                ("ssd_stage_wait_ms", C.c_double), ("ssd_copy_ms", C.c_double), ("pool_numa_node", C.c_int32),
+                ("pool_blobs", C.c_int32), ("pool_blobs_on_node", C.c_int32)]
 
 
 P, U64, I32, U32, F32, F64, VP = C.c_void_p, C.c_uint64, C.c_int32, C.c_uint32, C.c_float, C.c_double, C.c_void_p
@@ -86,6 +88,10 @@ _SIGS = {
     "loip_decode_step_device": (C.c_int, [P, P, I32, P, P]),
     "loip_prefill": (C.c_int, [P, P, P, I32, P, P]),
     "loip_replan": (C.c_int, [P, I32]),
+    "loip_inject_fault": (C.c_int, [P, I32, I32]),
+    "loip_get_copy_log": (I32, [P, P, P, I32]),
+    "loip_get_pool_nodes": (C.c_int, [P, P]),
+    "loip_poll_deadline_check": (C.c_int, [C.c_uint32, I32, C.POINTER(C.c_double)]),
     "loip_get_stats": (C.c_int, [P, C.POINTER(Stats)]),
     "loip_synchronize": (C.c_int, [P]),
     "loip_set_kernel_timing": (C.c_int, [P, I32]),
@@ -106,6 +112,7 @@ _SIGS = {
     "loip_k_lm_head": (C.c_int, [P, P, P, I32, I32, I32, F32, P, P, P, P, P]),
     "loip_k_lm_head_scratch_bytes": (C.c_uint64, [I32, I32]),
     "loip_k_gemm_bf16": (C.c_int, [P, P, I32, I32, I32, P, P]),
+    "loip_k_gemm_split": (C.c_int, [P, P, I32, I32, I32, P, P]),
     "loip_k_tc_status": (C.c_int, []),
 }
 
@@ -328,6 +335,23 @@ class Context:
     def replan(self, lookahead_tokens: int = 0):
         self._c(lib().loip_replan(self.h, lookahead_tokens))
 
+    def copy_log(self, max_n: int = 8192):
+        """(ms, bytes) arrays of the most recent completed layer copies, oldest first."""
+        ms, by = np.zeros(max_n, dtype=np.float64), np.zeros(max_n, dtype=np.uint64)
+        n = lib().loip_get_copy_log(self.h, _ptr(ms), _ptr(by), max_n)
+        if n < 0:
+            raise LoipError(ERR_INVALID, "copy log")
+        return ms[:n], by[:n]
+
+    def pool_nodes(self):
+        nodes = np.zeros(self.model["n_layers"], dtype=np.int32)
+        self._c(lib().loip_get_pool_nodes(self.h, _ptr(nodes)))
+        return nodes
+
+    def inject_fault(self, kind: int, arg: int = 0):
+        """Arms one host-side (or bounded device-wait) fault for a test."""
+        self._c(lib().loip_inject_fault(self.h, kind, arg))
+
     def stats(self) -> dict:
         s = Stats()
         self._c(lib().loip_get_stats(self.h, C.byref(s)))
@@ -379,6 +403,14 @@ def loip_k_qkv_rope(x, g, wqkv, Hq, Hkv, d, eps, theta, positions, q_out, kv_bas
                                  layer_page_bytes, _s(stream)))
 
 
+def loip_poll_deadline_check(timeout_ms: int, pending_polls: int):
+    """(status, waited_ms) of the library's host deadline loop against a fake
+    device that stays pending for `pending_polls` polls (< 0: forever)."""
+    w = C.c_double(0.0)
+    rc = lib().loip_poll_deadline_check(timeout_ms, pending_polls, C.byref(w))
+    return rc, w.value
+
+
 def loip_k_attention_scratch_floats(B, Hq, d, max_ctx, page_tokens) -> int:
     return int(lib().loip_k_attention_scratch_floats(B, Hq, d, max_ctx, page_tokens))
 
@@ -421,6 +453,13 @@ def loip_k_gemm_bf16(A, W, x, stream=None):
     """x += A W^T on the tensor cores (A [M, K], W [N, K] bf16 as int16 tensors)."""
     M, K = A.shape
     _check(lib().loip_k_gemm_bf16(_ptr(A), _ptr(W), M, W.shape[0], K, _ptr(x), _s(stream)))
+
+
+def loip_k_gemm_split(A2, W, x, stream=None):
+    """x += (A2[0] + A2[1]) W^T on the tensor cores (A2 [2, M, K], W [N, K] bf16
+    as int16 tensors): the split-pair operand at fp32 activation precision."""
+    _, M, K = A2.shape
+    _check(lib().loip_k_gemm_split(_ptr(A2), _ptr(W), M, W.shape[0], K, _ptr(x), _s(stream)))
 
 
 def loip_k_tc_status() -> int:

@@ -20,7 +20,7 @@ def L():
 
 def test_exports_every_declared_symbol(L):
     text = open(HEADER).read()
-    declared = set(re.findall(r"^\s*(?:int|void|const char\*|uint64_t|void\*)\s+(loip_\w+)\s*\(", text, re.M))
+    declared = set(re.findall(r"^\s*(?:int|int32_t|void|const char\*|uint64_t|void\*)\s+(loip_\w+)\s*\(", text, re.M))
     assert len(declared) >= 30
     for name in declared:
         assert hasattr(L, name), name
@@ -182,3 +182,17 @@ def test_noalloc_attention_refusals_without_gpu(L):
     assert call(B=2, Hq=24, Hkv=8, d=64, max_ctx=100) == loip.ERR_INVALID  # 3 query heads per kv head
     assert call(B=2, Hq=48, Hkv=3, d=64, max_ctx=100) == loip.ERR_INVALID  # 16
     assert call(B=2, Hq=8, Hkv=2, d=96, max_ctx=100) == loip.ERR_INVALID   # head size
+
+
+def test_host_deadline_loop_without_gpu(L):
+    """The deadline loop of every host wait, against a fake device: done after
+    some polls well inside the limit, or never done and given up once the limit
+    has passed (not long after it)."""
+    rc, w = loip.loip_poll_deadline_check(5000, 0)
+    assert rc == loip.OK and w < 100
+    rc, w = loip.loip_poll_deadline_check(5000, 2000)
+    assert rc == loip.OK and w < 2000
+    rc, w = loip.loip_poll_deadline_check(60, -1)
+    assert rc == loip.ERR_TIMEOUT and 60 <= w < 2000
+    rc, w = loip.loip_poll_deadline_check(0, -1)
+    assert rc == loip.ERR_TIMEOUT and w < 1000

@@ -2,24 +2,19 @@
 
 * 8B-shaped stack, every layer resident (the resident decode benchmark's plan and
   batch-1 kernel routing): 68 tokens decoded from an empty cache, teacher forced (the
-  last ones attend over two KV pages), against the oracle within the decode
+  last ones attend over two KV pages), against the oracle within the north-star
   tolerances; greedy tokens equal, or at a near tie within what the hidden-state error
   allows.  Then a 66-token prompt through the tensor-core prefill and two decode steps
-  on its cache, against the oracle's bf16-activation prefill.
+  on its cache, against the oracle, to the same tolerances.
 * 70B-shaped stack under the 60 GB device budget (the default benchmark's plan: 50 of
   80 layers streamed through two slots, one layer keeping its MHA block): a prefill and
   a decode step bit for bit equal to the same stack with every layer resident, then
-  three tokens decoded from an empty cache against the oracle.
+  three tokens decoded from an empty cache and a 2-token prefill with a decode step on
+  its cache, against the oracle.
 
-Decode runs fp32 activations, so the oracle (fp64, bf16 KV cache) agrees to the decode
-tolerances at any depth.  The prefill feeds its GEMMs bf16 activations; the oracle
-rounds at the same points, but a value within fp32 accumulation error of a bf16
-rounding boundary can round the other way, and those one-ulp differences spread
-through the residual stream over the layers (about 6.6e-3 max-abs after one layer,
-growing roughly with the square root of the depth: 0.045 at 32 layers, 0.089 at 80).
-Rows of the prefill, and decode rows that attend over a prefilled cache, are
-therefore held to a looser bound here (to the decode tolerances in the shallow models
-of the other tests).
+Both paths run fp32 activations (the prefill hands them to the tensor cores as split
+pairs of bf16 planes, ~2^-17 relative), so the oracle (fp64, bf16 KV cache, the one
+storage rounding the device makes) agrees to the benchmark spec's tolerances at any depth.
 
 The oracle reads the 8B weights materialised once; the 70B weights it generates per
 element on the fly (a full copy would not fit the host beside the pinned pool), about
@@ -31,8 +26,7 @@ from gpu_util import need_gpu
 from paper_2512_21835_gb300 import configs, inputs
 
 pytestmark = pytest.mark.gpu
-HID_ABS, HID_REL = 3e-2, 1e-2          # decode (the benchmark spec's tolerances)
-PREFILL_ABS, PREFILL_REL = 0.2, 5e-2   # bf16-activation prefill at full depth
+HID_ABS, HID_REL = 3e-2, 1e-2  # the benchmark spec's tolerances, for decode and prefill rows alike
 
 
 @pytest.fixture(scope="module")
@@ -76,7 +70,7 @@ def _oracle(orc, m, seq, n_prefill, materialise):
     else:
         w = orc.Weights(desc, configs.WEIGHT_SEED)
     return orc.forward(desc, w, np.asarray(seq, dtype=np.int32), n_prefill=n_prefill,
-                       prefill_flags=orc.KV_BF16 | orc.ACT_BF16, decode_flags=orc.KV_BF16, want_logits=True)
+                       prefill_flags=orc.KV_BF16, decode_flags=orc.KV_BF16, want_logits=True)
 
 
 def _errors(got_hid, want):
@@ -120,9 +114,9 @@ def test_8b_resident_decode_matches_oracle(torch, L, orc):
     ref = _oracle(orc, m, seq, 0, materialise=True)
     exempt = sum(_check_row(orc, m, toks[t], hids[t], ref, t) for t in range(len(seq)))
     assert exempt <= 1
-    ref_p = _oracle(orc, m, seq, P, materialise=True)
-    exempt = sum(_check_row(orc, m, pre_tok[i], pre_hid[i], ref_p, P - 1 + i, PREFILL_ABS, PREFILL_REL)
-                 for i in range(len(pre_tok)))
+    # prefill and decode use the same oracle flags, so the prefilled rows compare with
+    # the same reference rows
+    exempt = sum(_check_row(orc, m, pre_tok[i], pre_hid[i], ref, P - 1 + i) for i in range(len(pre_tok)))
     assert exempt <= 1
 
 
@@ -148,4 +142,7 @@ def test_70b_offloaded_is_lossless_and_decode_matches_oracle(torch, L, orc):
     dec_tok, dec_hid = runs[0][1]
     ref = _oracle(orc, m, seq, 0, materialise=False)
     exempt = sum(_check_row(orc, m, dec_tok[t], dec_hid[t], ref, t) for t in range(len(seq)))
+    # the 2-token prefill (its last row) and the decode step on its cache
+    pre_tok, pre_hid = runs[0][0]
+    exempt += sum(_check_row(orc, m, pre_tok[i], pre_hid[i], ref, 1 + i) for i in range(len(pre_tok)))
     assert exempt <= 1

@@ -105,6 +105,18 @@ def _paged_cache(torch, n_pages, Hkv, P, d, seed):
 @pytest.mark.parametrize("Hq,Hkv,d", [(8, 2, 128), (4, 2, 64), (32, 8, 128), (64, 8, 128), (8, 8, 128),
                                       (4, 4, 64), (16, 4, 64)])
 def test_attention_parity(torch, L, orc, Hq, Hkv, d, max_ctx, ctx_list):
+    _attention_case(torch, L, orc, Hq, Hkv, d, max_ctx, ctx_list)
+
+
+# the batched decode workload's shape: 8 requests, contexts up to 4096 + 256 decode
+# steps (68 pages, the combine's sixteen-pages-in-flight loop runs five rounds),
+# ragged on and off page boundaries; 70B heads (G = 8) and G = 2
+@pytest.mark.parametrize("Hq,Hkv,d", [(64, 8, 128), (16, 8, 128)])
+def test_attention_parity_batch8_many_pages(torch, L, orc, Hq, Hkv, d):
+    _attention_case(torch, L, orc, Hq, Hkv, d, 4352, (4352, 128, 4097, 1, 2600, 64, 3333, 4290))
+
+
+def _attention_case(torch, L, orc, Hq, Hkv, d, max_ctx, ctx_list):
     P = 64
     ctx = np.array(ctx_list, dtype=np.int32)
     B = len(ctx)
@@ -143,15 +155,18 @@ def test_attention_parity(torch, L, orc, Hq, Hkv, d, max_ctx, ctx_list):
 
 # one row (batch-1 decode) runs the block-tile kernel up to 8192 QKV rows and the
 # persistent kernel above (64 x 128 query + 2 x 8 x 128 kv rows = 10240)
-@pytest.mark.parametrize("single", [False, True])
+# "batch8": the batched decode shape, 8 rows at positions up to 4351 (68 pages)
+@pytest.mark.parametrize("single", [False, True, "batch8"])
 @pytest.mark.parametrize("Hq,Hkv,d,H", [(4, 2, 64, 256), (32, 8, 128, 4096), (8, 8, 128, 1024), (64, 8, 128, 1024)])
 def test_qkv_rope_parity(torch, L, orc, Hq, Hkv, d, H, single):
     P, eps, theta = 64, 1e-5, 500000.0
     pos = np.array([0, 5, 130, 1000], dtype=np.int32)[: 3 if Hq == 8 else 4]
-    if single:
+    if single is True:
         pos = np.array([1000], dtype=np.int32)
+    elif single == "batch8":
+        pos = np.array([4351, 0, 4096, 64, 2599, 127, 3333, 4289], dtype=np.int32)
     B = len(pos)
-    max_pages = 1000 // P + 1
+    max_pages = int(pos.max()) // P + 1
     buf, order, lpb = _paged_cache(torch, B * max_pages, Hkv, P, d, 4)
     pt = (order.reshape(B, max_pages).astype(np.int64)) * lpb
     x = inputs.normal_f32(41 + H, (B, H), 1.0)

@@ -54,16 +54,36 @@ def _run(L, torch, m, prompts, cont, cfg_kw, resident_layers, want_logits=False)
     return np.array(toks), np.array(hids), plan, st
 
 
+_ORACLE_CACHE = {}
+
+
 def _oracle(orc, m, prompt, cont):
-    desc = orc.ModelDesc(**m)
-    seq = np.concatenate([prompt, cont]).astype(np.int32)
-    return orc.forward(desc, orc.Weights(desc, configs.WEIGHT_SEED), seq, n_prefill=len(prompt),
-                       prefill_flags=orc.KV_BF16 | orc.ACT_BF16, decode_flags=orc.KV_BF16, want_logits=True)
+    key = (tuple(sorted(m.items())), tuple(int(t) for t in prompt), tuple(int(t) for t in cont))
+    if key not in _ORACLE_CACHE:
+        desc = orc.ModelDesc(**m)
+        seq = np.concatenate([prompt, cont]).astype(np.int32)
+        _ORACLE_CACHE[key] = orc.forward(desc, orc.Weights(desc, configs.WEIGHT_SEED), seq, n_prefill=len(prompt),
+                                         prefill_flags=orc.KV_BF16, decode_flags=orc.KV_BF16,
+                                         want_logits=True)
+    return _ORACLE_CACHE[key]
 
 
 def _check_hidden(got, want):
     assert np.max(np.abs(got - want)) <= HID_ABS
     assert np.linalg.norm(got - want) <= HID_REL * np.linalg.norm(want)
+
+
+def _check_vs_oracle(orc, m, prompts, conts, toks, hids):
+    """Every row a run produced (the prefill's last row of each request, then
+    one row per teacher-forced decode step) against the oracle: final hidden
+    within the decode tolerances, greedy token equal.  toks [steps + 1][B],
+    hids [steps + 1][B][H]; conts[b] = the tokens fed to request b."""
+    for b in range(len(prompts)):
+        ref = _oracle(orc, m, prompts[b], conts[b])
+        for i in range(len(conts[b]) + 1):
+            t = len(prompts[b]) - 1 + i
+            _check_hidden(hids[i][b], ref["hidden"][t])
+            assert int(toks[i][b]) == int(ref["argmax"][t]), (b, i)
 
 
 def test_tiny_prefill_decode_matches_oracle(torch, L, orc):
@@ -191,6 +211,8 @@ def test_direct_access_decode_copies_nothing(torch, L, orc):
     assert np.array_equal(np.array(toks), base[0])
     assert np.array_equal(hids[0].view(np.uint32), base[1][0].view(np.uint32))
     assert np.max(np.abs(np.array(hids) - base[1])) <= 1e-4
+    # and every row of the direct-access run against the oracle itself
+    _check_vs_oracle(orc, m, prompts, [[c[0] for c in cont]], np.array(toks), np.array(hids))
 
 
 def _decode_with_timing(L, torch, m, prompt, cont, cfg_kw, resident_layers):
@@ -315,6 +337,8 @@ def test_block_level_residency_is_bitwise_lossless(torch, L, orc, extra, mode):
     ctx.close()
     assert np.array_equal(np.array(toks), base[0])
     assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
+    conts = [[c[b] for c in cont] for b in range(2)]
+    _check_vs_oracle(orc, m, prompts, conts, np.array(toks), np.array(hids))
 
 
 @pytest.mark.parametrize("whole", [0, 1])
@@ -354,6 +378,7 @@ def test_kv_growth_offloads_blocks_or_layers(torch, L, orc, whole):
         assert masks.count(0) == 2 and masks.count(2) == 1 and masks.count(3) == 3
     assert np.array_equal(np.array(toks), base[0])
     assert np.array_equal(np.array(hids).view(np.uint32), base[1].view(np.uint32))
+    _check_vs_oracle(orc, m, [prompt], [[c[0] for c in cont]], np.array(toks), np.array(hids))
 
 
 TINY_QK = configs.MODELS["tiny-qk"]
@@ -414,3 +439,25 @@ def test_ssd_tier_is_bitwise_lossless(torch, L, orc, tmp_path, mode, K):
     assert got[3]["n_ssd_layers"] == 7 and got[3]["ssd_read_bytes"] >= 7 * lay["l_size"] * len(cont)
     assert np.array_equal(base[0], got[0])
     assert np.array_equal(base[1].view(np.uint32), got[1].view(np.uint32))
+    conts = [[c[b] for c in cont] for b in range(2)]
+    _check_vs_oracle(orc, m, prompts, conts, got[0], got[1])
+
+
+def test_batch8_decode_over_many_pages_matches_oracle(torch, L, orc):
+    """The batched decode shape (8 requests, ragged contexts drawn uniformly, here
+    in [128, 1600]: 3 to 26 KV pages each) on the tiny layers, four of them, two
+    streamed through one slot: the prefill of all eight prompts in 512-row
+    chunks, then six teacher-forced decode steps at batch 8 (three requests cross
+    a page boundary), every row against the oracle."""
+    m = dict(TINY, n_layers=4)
+    lens = [int(n) for n in inputs.context_lengths(configs.CONTEXT_SEED, 8, 128, 1600)]
+    for b in (0, 3, 6):  # these requests cross into a new page during the decode steps
+        lens[b] = lens[b] // 64 * 64 - 3
+    prompts = [inputs.token_ids(300 + b, n, m["vocab"]) for b, n in enumerate(lens)]
+    assert max(lens) > 1200 and min(lens) < 600
+    conts = [inputs.token_ids(400 + b, 6, m["vocab"]) for b in range(8)]
+    cont = [[int(conts[b][s]) for b in range(8)] for s in range(6)]
+    kw = dict(max_batch=8, max_ctx=max(lens) + 8, n_slots=1)
+    toks, hids, plan, st = _run(L, torch, m, prompts, cont, kw, 2)
+    assert plan["n_offloaded"] == 2 and st["h2d_weight_bytes"] > 0
+    _check_vs_oracle(orc, m, prompts, conts, toks, hids)

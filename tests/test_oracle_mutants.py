@@ -47,6 +47,24 @@ MUTANTS = {
                                    "            for (int h = 0; h < Hq; ++h) orc_rope(q + (size_t)h * hd, hd, t, d->rope_theta);\n            for (int h = 0; h < Hkv; ++h) orc_rope(k + (size_t)h * hd, hd, t, d->rope_theta);\n            if (d->qk_norm) {"),
     "qk-norm uses the query gain for keys": ("orc_rmsnorm(k + (size_t)h * hd, &qk[1], hd,", "orc_rmsnorm(k + (size_t)h * hd, &qk[0], hd,"),
     "kv rounding skipped": ("Kl[(size_t)t * kvd + i] = maybe_bf16(k[i], kvb);", "Kl[(size_t)t * kvd + i] = k[i];"),
+    "value rounding skipped": ("Vl[(size_t)t * kvd + i] = maybe_bf16(v[i], kvb);", "Vl[(size_t)t * kvd + i] = v[i];"),
+    # the one storage rounding, moved: keys rounded before their rotation instead of after
+    "keys rounded before the rotation": (
+        "            for (int h = 0; h < Hkv; ++h) orc_rope(k + (size_t)h * hd, hd, t, d->rope_theta);\n"
+        "            for (int i = 0; i < kvd; ++i) {\n                Kl[(size_t)t * kvd + i] = maybe_bf16(k[i], kvb);",
+        "            for (int i = 0; i < kvd; ++i) k[i] = maybe_bf16(k[i], kvb);\n"
+        "            for (int h = 0; h < Hkv; ++h) orc_rope(k + (size_t)h * hd, hd, t, d->rope_theta);\n"
+        "            for (int i = 0; i < kvd; ++i) {\n                Kl[(size_t)t * kvd + i] = k[i];"),
+    # ... or spread to a value the device keeps in fp32: the rotated queries
+    "queries rounded like the cache": (
+        "            orc_attention(q, Kl, Vl, t + 1, Hq, Hkv, hd, o, NULL);",
+        "            for (int i = 0; i < qd; ++i) q[i] = maybe_bf16(q[i], kvb);\n"
+        "            orc_attention(q, Kl, Vl, t + 1, Hq, Hkv, hd, o, NULL);"),
+    # ... or to the attention output (the input of the output projection)
+    "attention output rounded like the cache": (
+        "            orc_gemv(&lt[L_WO], qd, NULL, H, o, r);",
+        "            for (int i = 0; i < qd; ++i) o[i] = maybe_bf16(o[i], kvb);\n"
+        "            orc_gemv(&lt[L_WO], qd, NULL, H, o, r);"),
 }
 
 
