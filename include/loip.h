@@ -92,6 +92,11 @@ typedef struct loip_config {
                                    * staging buffers taken out of this budget */
     const char* ssd_dir;          /* directory of the SSD tier's scratch file (caller-owned string,
                                    * read at create; NULL = /tmp) */
+    int32_t embed_on_host;        /* 1: the embedding table [vocab, hidden] stays in pinned host
+                                   * memory, mapped for the device, and the embedding gather reads
+                                   * each token's row over the host link (16 KB per token at the 70B
+                                   * shape); its vocab * hidden * 2 bytes of device budget go to
+                                   * resident weights instead.  0: in the device arena (default) */
 } loip_config;
 
 typedef struct loip_layer_layout_t {
@@ -210,8 +215,9 @@ int loip_create(const loip_model_desc* desc, const loip_config* cfg, void* devic
 
 void loip_destroy(loip_ctx* ctx);
 
-/* Message of the last failed call on ctx (or of the last failed create when
- * ctx is NULL).  Valid until the next call. */
+/* Message of the last failed call on ctx (or, when ctx is NULL, of the last
+ * failed create or kernel-level loip_k_* launch on this thread).  Valid until
+ * the next call. */
 const char* loip_last_error(const loip_ctx* ctx);
 
 /* Fills every weight with the seeded SplitMix64 generator (bf16 N(0, 0.02^2)
@@ -441,6 +447,28 @@ int loip_k_attention_noalloc(const float* q, const void* kv_base, const int64_t*
                              const int32_t* ctx_lens, int32_t B, int32_t Hq, int32_t Hkv, int32_t d,
                              int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes, int32_t max_ctx, float* o,
                              void* stream);
+
+/* Causal prefill attention on the tensor cores (the attention of a prefill
+ * pass, Sec. III-A's decoder layer on a prompt): n_prompts prompts of
+ * prompt_lens[i] tokens (host int32) whose rows are concatenated in q (fp32
+ * [M, Hq*d], M = sum of the lengths, 16-byte aligned); prompt i's rows sit at
+ * positions first_pos[i] .. first_pos[i] + len - 1 (host int32, NULL = 0) of
+ * request i, and each row attends over that request's cached positions 0 ..
+ * its own (keys and values already in the pages, layout as in
+ * loip_k_attention; request i's pages are row i of page_offsets).  Query and
+ * probability operands go to the tensor cores as split bf16 pairs (fp32
+ * accuracy).  Writes o2 (bf16 [2][M][Hq*d]: hi = bf16(o) then lo = bf16(o -
+ * hi), the next projection's split operand).  `tiles` is device scratch of at
+ * least (M + n_prompts) * 16 bytes (the query-tile list, uploaded on `stream`).
+ * d = 64 or 128, Hq / Hkv = 1, 2, 4 or 8, page_tokens = 64. */
+int loip_k_prefill_attention(const float* q, const void* kv_base, const int64_t* page_offsets, int32_t max_pages,
+                             const int32_t* prompt_lens, const int32_t* first_pos, int32_t n_prompts, int32_t Hq,
+                             int32_t Hkv, int32_t d, int32_t page_tokens, int32_t layer, uint64_t layer_page_bytes,
+                             void* tiles, uint16_t* o2, void* stream);
+
+/* 0 if no tensor-core attention launch has recorded a failure (a bounded wait
+ * that ran out); otherwise the first failure code.  -1 if unreadable. */
+int loip_k_attention_tc_status(void);
 
 /* x += wo o  (output projection with the residual add); o fp32 [B, Hq*d].  As in
  * decode, at batch 1 the blocks of the first wave also pull the later blocks'

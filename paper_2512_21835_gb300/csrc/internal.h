@@ -145,6 +145,16 @@ cudaError_t launch_tc_gemm_swiglu(const uint16_t* y, bool split, const uint16_t*
                                   int F, uint16_t* a, cudaStream_t st);
 // First failure code recorded by a tensor-core GEMM launch (0 = none).
 cudaError_t tc_error(int* code);
+// Causal prefill attention on the tensor cores (attn_tc.cu).  tiles[i] =
+// {first row, rows, request, position of the first row}: a run of at most
+// attention_tc_tile_positions(Hq, Hkv) = 128 / (Hq / Hkv) consecutive positions
+// of one request, rows of q (fp32 [M, Hq d]); each row attends over its
+// request's cached positions 0 .. its own.  o: split pair [2][M][Hq d].
+// d = 64 or 128, Hq / Hkv = 1, 2, 4 or 8, page_tokens = 64.
+int attention_tc_tile_positions(int Hq, int Hkv);
+cudaError_t launch_attention_tc(const float* q, KvView kv, const int4* tiles, int n_tiles, int M, int Hq, int Hkv,
+                                int d, uint16_t* o, cudaStream_t st);
+cudaError_t attention_tc_error(int* code);
 cudaError_t launch_gather_rows(const float* x, const int32_t* rows, int n, int H, float* out, cudaStream_t st);
 
 }  // namespace loip

@@ -76,7 +76,7 @@ struct Request {
 struct Fixed {  // offsets inside the fixed region
     uint64_t embed, lm_head, g_final, x, q, o, a, z, logits, attn_scratch, lm_scratch;
     uint64_t tokens, out_tokens, positions, ctx_lens, row_req, page_table, last_rows, dec_pos, run_sync, qk_raw;
-    uint64_t px, py, pq, po, pa;
+    uint64_t px, py, pq, po, pa, ptiles;
     uint64_t total;
 };
 
@@ -145,7 +145,7 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
         off = align_up(off + bytes);
         return o;
     };
-    f.embed = take(V * H * 2);
+    f.embed = c->embed_on_host ? UINT64_MAX : take(V * H * 2);  // on the host: no device bytes
     f.lm_head = take(V * H * 2);
     f.g_final = take(H * 2);
     f.x = take(B * H * 4);
@@ -172,6 +172,7 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     f.pq = take(Mp * qd * 4);
     f.po = take(2 * Mp * qd * 2);
     f.pa = take(2 * Mp * F * 2);
+    f.ptiles = take((Mp + (uint64_t)B + 16) * 16);  // tensor-core attention's query tiles (int4 each)
     f.total = off;
     return f;
 }
@@ -206,6 +207,24 @@ struct loip_ctx {
     std::vector<Request> reqs;
     int max_pages = 0;
     bool pt_dirty = true;
+    // embedding table in mapped pinned host memory (loip_config.embed_on_host)
+    HostBuf embed_host;
+    // the table the embedding gather reads: the arena's copy, or the device
+    // address of the mapped host copy (nullptr until it is allocated)
+    const uint16_t* embed_table() {
+        if (!cfg.embed_on_host) return fixed_ptr<uint16_t>(fx.embed);
+        return static_cast<const uint16_t*>(embed_host.dev);
+    }
+    int ensure_embed_host() {
+        if (!cfg.embed_on_host || embed_host.ptr) return LOIP_OK;
+        cudaError_t e = host_buf_alloc((size_t)V * H * 2, &embed_host);
+        if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned allocation of the embedding table failed");
+        if (!embed_host.dev) {
+            host_buf_free(&embed_host);
+            return fail(LOIP_ERR_CUDA, "the host embedding table cannot be mapped for the device");
+        }
+        return LOIP_OK;
+    }
     // host pool: blobs of offloaded layers inside pinned huge-page regions
     std::vector<void*> host_layer;
     std::vector<HostBuf> host_regions;
@@ -255,6 +274,7 @@ struct loip_ctx {
     std::deque<KEv> kernel_events;
     bool weights_loaded = false;
     bool failed = false;
+    int prefill_tiles = 0;  // query tiles of the current prefill chunk (tensor-core attention)
     // fault injection (loip_inject_fault): one armed fault, fired once
     int fault_kind = 0, fault_arg = 0;
     bool take_fault(int kind) {
@@ -728,8 +748,7 @@ struct loip_ctx {
             });
         if (e == cudaSuccess)
             e = timed(7, s, [&] {
-                return launch_attention(pq, kv, nullptr, pos, req, Mc, Hq, Hkv, d, cfg.max_ctx, false, nullptr, po,
-                                        true, s);
+                return launch_attention_tc(pq, kv, fixed_ptr<int4>(fx.ptiles), prefill_tiles, Mc, Hq, Hkv, d, po, s);
             });
         if (e == cudaSuccess)
             e = timed(8, s, [&] { return launch_tc_gemm_resid(po, true, wa + lay.off_wo / 2, Mc, H, qd, px, s); });
@@ -1148,6 +1167,7 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
     if (ctx->compute) cudaStreamSynchronize(ctx->compute);
     if (ctx->copy) cudaStreamSynchronize(ctx->copy);
     for (auto& hb : ctx->host_regions) host_buf_free(&hb);
+    host_buf_free(&ctx->embed_host);
     for (int b = 0; b < loip_ctx::kStages; ++b) {
         host_buf_free(&ctx->stage[b]);
         if (ctx->stage_done[b]) cudaEventDestroy(ctx->stage_done[b]);
@@ -1350,7 +1370,9 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_stage, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreate(&c->ev_step0);
     if (e == cudaSuccess) e = cudaEventCreate(&c->ev_step1);
-    c->h_stage_ints = 4 * (size_t)std::max(cfg.max_batch, cfg.max_prefill_tokens) + 64;
+    // staging: a prefill chunk's tokens, positions, requests and attention tiles;
+    // the second quarter also receives the output tokens
+    c->h_stage_ints = 8 * (size_t)std::max(cfg.max_batch, cfg.max_prefill_tokens) + 4 * (size_t)cfg.max_batch + 128;
     if (e == cudaSuccess) e = cudaHostAlloc(&c->h_stage, c->h_stage_ints * 4, cudaHostAllocDefault);
     if (e == cudaSuccess) e = cudaHostAlloc(&c->h_pt, (size_t)cfg.max_batch * c->max_pages * 8, cudaHostAllocDefault);
     if (e != cudaSuccess) {
@@ -1440,7 +1462,10 @@ extern "C" int loip_load_weights_generated(loip_ctx* c, uint64_t seed) {
     CTX_GUARD(c);
     int rc = c->sync_all();
     if (rc) return rc;
-    cudaError_t e = launch_generate(c->fixed_ptr<uint16_t>(c->fx.embed), (uint64_t)c->V * c->H, 0, seed, 1, 0,
+    rc = c->ensure_embed_host();
+    if (rc) return rc;
+    // (a host-resident table is written by the generator through its mapping)
+    cudaError_t e = launch_generate(const_cast<uint16_t*>(c->embed_table()), (uint64_t)c->V * c->H, 0, seed, 1, 0,
                                     c->compute);
     if (e == cudaSuccess)
         e = launch_generate(c->fixed_ptr<uint16_t>(c->fx.lm_head), (uint64_t)c->V * c->H, 0, seed, 2, 0, c->compute);
@@ -1511,7 +1536,13 @@ extern "C" int loip_load_globals(loip_ctx* c, const uint16_t* embed, const uint1
     CTX_GUARD(c);
     if (!embed || !lm_head || !g_final) return c->fail(LOIP_ERR_INVALID, "null pointer");
     size_t vh = (size_t)c->V * c->H * 2;
-    cudaError_t e = cudaMemcpy(c->arena + c->fx.embed, embed, vh, cudaMemcpyHostToDevice);
+    int rc = c->ensure_embed_host();
+    if (rc) return rc;
+    cudaError_t e = cudaSuccess;
+    if (c->cfg.embed_on_host)
+        memcpy(c->embed_host.ptr, embed, vh);
+    else
+        e = cudaMemcpy(c->arena + c->fx.embed, embed, vh, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(c->arena + c->fx.lm_head, lm_head, vh, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(c->arena + c->fx.g_final, g_final, (size_t)c->H * 2, cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return c->cuda_fail(e, "globals upload");
@@ -1594,7 +1625,7 @@ static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int3
     cudaEventRecord(c->ev_step0, s);
     c->chain = false;
     float* x = c->fixed_ptr<float>(c->fx.x);
-    e = launch_embed(c->fixed_ptr<uint16_t>(c->fx.embed), d_tokens, B, c->H, c->V, x, s, false);
+    e = launch_embed(c->embed_table(), d_tokens, B, c->H, c->V, x, s, false);
     if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
     c->chain = true;
     if (c->cfg.mode == LOIP_MODE_DIRECT)
@@ -1699,6 +1730,7 @@ extern "C" int loip_prefill(loip_ctx* c, const int32_t* tokens, const int32_t* p
     rc = c->upload_page_table(s);
     if (rc) return rc;
     const int Mp = c->cfg.max_prefill_tokens;
+    const int tile_pos = attention_tc_tile_positions(c->Hq, c->Hkv);  // positions per attention tile
     // per-token request and position
     std::vector<int32_t> req_of(M), pos_of(M);
     std::vector<int32_t> last_row(n_prompts);
@@ -1722,14 +1754,29 @@ extern "C" int loip_prefill(loip_ctx* c, const int32_t* tokens, const int32_t* p
         memcpy(h, tokens + c0, (size_t)Mc * 4);
         memcpy(h + Mc, pos_of.data() + c0, (size_t)Mc * 4);
         memcpy(h + 2 * Mc, req_of.data() + c0, (size_t)Mc * 4);
+        // attention query tiles: runs of at most P_T consecutive rows of one request
+        int32_t* ht = h + 3 * Mc;
+        c->prefill_tiles = 0;
+        for (int i = 0; i < Mc;) {
+            int n = 1;
+            while (i + n < Mc && n < tile_pos && req_of[c0 + i + n] == req_of[c0 + i]) ++n;
+            ht[4 * c->prefill_tiles + 0] = i;
+            ht[4 * c->prefill_tiles + 1] = n;
+            ht[4 * c->prefill_tiles + 2] = req_of[c0 + i];
+            ht[4 * c->prefill_tiles + 3] = pos_of[c0 + i];
+            ++c->prefill_tiles;
+            i += n;
+        }
         cudaError_t e = cudaMemcpyAsync(c->arena + c->fx.tokens, h, (size_t)Mc * 4, cudaMemcpyHostToDevice, s);
         if (e == cudaSuccess)
             e = cudaMemcpyAsync(c->arena + c->fx.positions, h + Mc, (size_t)Mc * 4, cudaMemcpyHostToDevice, s);
         if (e == cudaSuccess)
             e = cudaMemcpyAsync(c->arena + c->fx.row_req, h + 2 * Mc, (size_t)Mc * 4, cudaMemcpyHostToDevice, s);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(c->arena + c->fx.ptiles, ht, (size_t)c->prefill_tiles * 16, cudaMemcpyHostToDevice, s);
         if (e != cudaSuccess) return c->cuda_fail(e, "prefill upload");
         cudaEventRecord(c->ev_stage, s);
-        e = launch_embed(c->fixed_ptr<uint16_t>(c->fx.embed), c->fixed_ptr<int32_t>(c->fx.tokens), Mc, c->H, c->V,
+        e = launch_embed(c->embed_table(), c->fixed_ptr<int32_t>(c->fx.tokens), Mc, c->H, c->V,
                          c->fixed_ptr<float>(c->fx.px), s);
         if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
         rc = c->run_layers([&](int l, int slot) { return c->prefill_layer(l, Mc, s, slot); });
@@ -1756,10 +1803,14 @@ extern "C" int loip_prefill(loip_ctx* c, const int32_t* tokens, const int32_t* p
     rc = c->wait_event(c->ev_done);
     if (rc) return rc;
     c->collect_kernel_times();
-    int tcerr = 0;
+    int tcerr = 0, aterr = 0;
     if (tc_error(&tcerr) != cudaSuccess || tcerr != 0) {
         c->failed = true;
         return c->fail(LOIP_ERR_TIMEOUT, "tensor-core GEMM pipeline did not complete (code " + std::to_string(tcerr) + ")");
+    }
+    if (attention_tc_error(&aterr) != cudaSuccess || aterr != 0) {
+        c->failed = true;
+        return c->fail(LOIP_ERR_TIMEOUT, "tensor-core attention did not complete (code " + std::to_string(aterr) + ")");
     }
     memcpy(out_tokens, hout, (size_t)n_prompts * 4);
     for (int i = 0; i < n_prompts; ++i) c->reqs[i].len = prompt_lens[i];
@@ -1958,6 +2009,7 @@ extern "C" void* loip_copy_stream(loip_ctx* c) { return c ? (void*)c->copy : nul
 static bool al16(const void* p) { return ((uintptr_t)p & 15) == 0; }
 static int cerr(cudaError_t e) {
     if (e == cudaSuccess) return LOIP_OK;
+    g_create_error = std::string("kernel launch: ") + cudaGetErrorString(e);  // loip_last_error(NULL)
     cudaGetLastError();  // leave no non-sticky error behind for the next call
     return LOIP_ERR_CUDA;
 }
@@ -2009,6 +2061,40 @@ extern "C" int loip_k_attention(const float* q, const void* kv_base, const int64
                                  (cudaStream_t)stream, false, 0, true));
 }
 
+extern "C" int loip_k_prefill_attention(const float* q, const void* kv_base, const int64_t* page_offsets,
+                                        int32_t max_pages, const int32_t* prompt_lens, const int32_t* first_pos,
+                                        int32_t n_prompts, int32_t Hq, int32_t Hkv, int32_t d, int32_t page_tokens,
+                                        int32_t layer, uint64_t layer_page_bytes, void* tiles, uint16_t* o2,
+                                        void* stream) {
+    if (!q || !kv_base || !page_offsets || !prompt_lens || !tiles || !o2 || n_prompts < 1 || Hq < 1 || Hkv < 1 ||
+        (d != 64 && d != 128) || Hq % Hkv || page_tokens != 64 || max_pages < 1 || !al16(q) || !al16(kv_base) ||
+        !al16(o2) || !al16(tiles))
+        return LOIP_ERR_INVALID;
+    const int G = Hq / Hkv;
+    if (G != 1 && G != 2 && G != 4 && G != 8) return LOIP_ERR_INVALID;
+    const int tp = attention_tc_tile_positions(Hq, Hkv);
+    std::vector<int4> t;
+    int M = 0;
+    for (int i = 0; i < n_prompts; ++i) {
+        const int len = prompt_lens[i], p0 = first_pos ? first_pos[i] : 0;
+        if (len < 1 || p0 < 0 || (int64_t)p0 + len > (int64_t)max_pages * page_tokens) return LOIP_ERR_INVALID;
+        for (int j = 0; j < len; j += tp) t.push_back(make_int4(M + j, std::min(tp, len - j), i, p0 + j));
+        M += len;
+    }
+    KvView kv{(char*)kv_base, page_offsets, max_pages, page_tokens, layer, layer_page_bytes};
+    cudaError_t e = cudaMemcpyAsync(tiles, t.data(), t.size() * sizeof(int4), cudaMemcpyHostToDevice,
+                                    (cudaStream_t)stream);
+    if (e != cudaSuccess) return cerr(e);
+    return cerr(launch_attention_tc(q, kv, static_cast<const int4*>(tiles), (int)t.size(), M, Hq, Hkv, d, o2,
+                                    (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_attention_tc_status(void) {
+    int code = 0;
+    if (attention_tc_error(&code) != cudaSuccess) return -1;
+    return code;
+}
+
 extern "C" int loip_k_oproj(const float* o, const uint16_t* wo, int32_t B, int32_t H, int32_t K, float* x,
                             void* stream) {
     if (!o || !wo || !x || B < 1 || B > 8 || K % 8 || H < 1 || !al16(wo) || !al16(o)) return LOIP_ERR_INVALID;
@@ -2033,8 +2119,7 @@ extern "C" int loip_k_gemm_bf16(const uint16_t* A, const uint16_t* W, int32_t M,
                                 void* stream) {
     if (!A || !W || !x || M < 1 || N < 1 || K < 8 || K % 8 || !al16(A) || !al16(W) || !al16(x) || N % 4)
         return LOIP_ERR_INVALID;
-    cudaError_t e = launch_tc_gemm_resid(A, false, W, M, N, K, x, (cudaStream_t)stream);
-    return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA;
+    return cerr(launch_tc_gemm_resid(A, false, W, M, N, K, x, (cudaStream_t)stream));
 }
 
 extern "C" int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t M, int32_t N, int32_t K, float* x,
@@ -2042,8 +2127,7 @@ extern "C" int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t 
     // the lo plane starts M * K elements after the hi plane: 16-byte aligned too
     if (!A2 || !W || !x || M < 1 || N < 1 || K < 8 || K % 8 || !al16(A2) || !al16(W) || !al16(x) || N % 4)
         return LOIP_ERR_INVALID;
-    cudaError_t e = launch_tc_gemm_resid(A2, true, W, M, N, K, x, (cudaStream_t)stream);
-    return e == cudaSuccess ? LOIP_OK : LOIP_ERR_CUDA;
+    return cerr(launch_tc_gemm_resid(A2, true, W, M, N, K, x, (cudaStream_t)stream));
 }
 
 extern "C" int loip_k_tc_status(void) {

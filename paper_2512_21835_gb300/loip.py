@@ -38,7 +38,7 @@ class Config(C.Structure):
                 ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("layer_run_kernel", C.c_int32), ("mode", C.c_int32),
                 ("timeout_ms", C.c_uint32), ("hbm_Bps", C.c_double), ("link_Bps", C.c_double),
                 ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32), ("whole_layers", C.c_int32),
-                ("host_budget_bytes", C.c_uint64), ("ssd_dir", C.c_char_p)]
+                ("host_budget_bytes", C.c_uint64), ("ssd_dir", C.c_char_p), ("embed_on_host", C.c_int32)]
 
 
 class LayerLayout(C.Structure):
@@ -113,6 +113,8 @@ _SIGS = {
     "loip_k_lm_head_scratch_bytes": (C.c_uint64, [I32, I32]),
     "loip_k_gemm_bf16": (C.c_int, [P, P, I32, I32, I32, P, P]),
     "loip_k_gemm_split": (C.c_int, [P, P, I32, I32, I32, P, P]),
+    "loip_k_prefill_attention": (C.c_int, [P, P, P, I32, P, P, I32, I32, I32, I32, I32, I32, U64, P, P, P]),
+    "loip_k_attention_tc_status": (C.c_int, []),
     "loip_k_tc_status": (C.c_int, []),
 }
 
@@ -165,10 +167,11 @@ def model_desc(m: dict) -> ModelDesc:
 def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 2048, mode: int = MODE_OVERLAP,
            timeout_ms: int = 0, hbm_Bps: float = 6.7e12, link_Bps: float = 2.1e11, kv_reserve_bytes: int = 0,
            max_prefill_tokens: int = 512, page_tokens: int = 64, layer_run_kernel: int = 0,
-           whole_layers: int = 0, host_budget_bytes: int = 0, ssd_dir: str | None = None) -> Config:
+           whole_layers: int = 0, host_budget_bytes: int = 0, ssd_dir: str | None = None,
+           embed_on_host: int = 0) -> Config:
     return Config(budget, n_slots, page_tokens, max_batch, max_ctx, layer_run_kernel, mode, timeout_ms, hbm_Bps,
                   link_Bps, kv_reserve_bytes, max_prefill_tokens, whole_layers, host_budget_bytes,
-                  ssd_dir.encode() if ssd_dir else None)
+                  ssd_dir.encode() if ssd_dir else None, embed_on_host)
 
 
 # ----------------------------------------------------------------------------
@@ -432,6 +435,20 @@ def loip_k_attention_noalloc(q, kv_base, page_offsets, max_pages, ctx_lens, Hq, 
     B = q.shape[0]
     _check(lib().loip_k_attention_noalloc(_ptr(q), _ptr(kv_base), _ptr(page_offsets), max_pages, _ptr(ctx_lens), B, Hq,
                                           Hkv, d, page_tokens, layer, layer_page_bytes, max_ctx, _ptr(o), _s(stream)))
+
+
+def loip_k_prefill_attention(q, kv_base, page_offsets, max_pages, prompt_lens, first_pos, Hq, Hkv, d, page_tokens,
+                             layer, layer_page_bytes, tiles, o2, stream=None):
+    """Causal prefill attention on the tensor cores; o2: [2, M, Hq*d] int16 (bf16 hi, lo)."""
+    lens = np.ascontiguousarray(prompt_lens, dtype=np.int32)
+    fp = None if first_pos is None else np.ascontiguousarray(first_pos, dtype=np.int32)
+    _check(lib().loip_k_prefill_attention(_ptr(q), _ptr(kv_base), _ptr(page_offsets), max_pages, _ptr(lens), _ptr(fp),
+                                          len(lens), Hq, Hkv, d, page_tokens, layer, layer_page_bytes, _ptr(tiles),
+                                          _ptr(o2), _s(stream)))
+
+
+def loip_k_attention_tc_status() -> int:
+    return int(lib().loip_k_attention_tc_status())
 
 
 def loip_k_oproj(o, wo, x, stream=None):

@@ -226,3 +226,65 @@ def test_lm_head_parity(torch, L, orc, B, H, V):
         assert argmax_agrees(int(gt[b]), glg[b], ref)
         # the token is the argmax of the logits the kernel wrote (lowest index on ties)
         assert int(gt[b]) == int(np.argmax(glg[b]))
+
+
+def _split_to_f64(orc, o2):
+    """[2, M, n] bf16 pair (hi, lo) -> fp64 hi + lo."""
+    a = o2.cpu().numpy().view(np.uint16)
+    return orc.bf16_bits_to_f64(a[0]) + orc.bf16_bits_to_f64(a[1])
+
+
+# Tensor-core causal prefill attention: G = 8, 4, 2, 1 at d = 128 and 64; prompts of
+# one row, several query tiles and page boundaries; the last prompt continues a
+# request whose first 64 or 128 positions are already cached (first_pos > 0)
+@pytest.mark.parametrize("Hq,Hkv,d", [(64, 8, 128), (16, 4, 64), (8, 4, 128), (4, 4, 64), (8, 2, 64), (4, 2, 64),
+                                      (8, 1, 64), (4, 4, 128)])
+@pytest.mark.parametrize("lens,first", [([1, 70, 200, 37], [0, 0, 0, 128]), ([32], [0])])
+def test_prefill_attention_tc_parity(torch, L, orc, Hq, Hkv, d, lens, first):
+    P = 64
+    B = len(lens)
+    max_pages = max(f + n for f, n in zip(first, lens)) // P + 1
+    buf, order, lpb = _paged_cache(torch, B * max_pages, Hkv, P, d, 5)
+    pt = (order.reshape(B, max_pages).astype(np.int64)) * lpb
+    T = max_pages * P
+    Kall = inputs.bf16_bits(71 + d, (B, T, Hkv, d), 1.0)
+    Vall = inputs.bf16_bits(72 + d, (B, T, Hkv, d), 1.0)
+    # positions past each request's last row hold no key yet: NaN there, which the
+    # kernel must never let into a result
+    for b in range(B):
+        Kall[b, first[b] + lens[b]:] = 0x7FC0
+        Vall[b, first[b] + lens[b]:] = 0x7FC0
+    host = np.zeros(buf.numel(), dtype=np.uint8)
+    for b in range(B):
+        for pg in range(max_pages):
+            base = pt[b, pg]
+            kp = Kall[b, pg * P:(pg + 1) * P].transpose(1, 0, 2).copy()
+            vp = Vall[b, pg * P:(pg + 1) * P].transpose(1, 0, 2).copy()
+            host[base:base + kp.nbytes] = kp.view(np.uint8).ravel()
+            host[base + kp.nbytes:base + 2 * kp.nbytes] = vp.view(np.uint8).ravel()
+    buf.copy_(torch.from_numpy(host))
+    M = sum(lens)
+    q = inputs.normal_f32(73 + d, (M, Hq * d), 0.5)
+    tiles = torch.empty((M + B) * 4, dtype=torch.int32, device="cuda")
+    o2 = torch.full((2, M, Hq * d), -1, dtype=torch.int16, device="cuda")
+    L.loip_k_prefill_attention(dev_f32(q), buf, torch.from_numpy(pt).cuda(), max_pages, lens, first, Hq, Hkv, d, P, 0,
+                               lpb, tiles, o2)
+    torch.cuda.synchronize()
+    assert L.loip_k_attention_tc_status() == 0
+    got = _split_to_f64(orc, o2)
+    row = 0
+    worst = 0.0
+    for b in range(B):
+        for i in range(lens[b]):
+            pos = first[b] + i
+            K64 = orc.bf16_bits_to_f64(Kall[b, :pos + 1])
+            V64 = orc.bf16_bits_to_f64(Vall[b, :pos + 1])
+            want = orc.attention(q[row].reshape(Hq, d).astype(np.float64), K64, V64, Hkv).ravel()
+            vmax = np.max(np.abs(V64))
+            # fp32 scores and sums as in decode, plus the split pairs' 2^-17 residues
+            tol = (d + pos + 64) * U * 8.0 * vmax + 2.0 ** -15 * vmax + 1e-6
+            err = np.max(np.abs(got[row] - want))
+            worst = max(worst, err / tol)
+            assert err <= tol, (b, i, err, tol)
+            row += 1
+    print("worst err / tol", worst)

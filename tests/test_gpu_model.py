@@ -461,3 +461,31 @@ def test_batch8_decode_over_many_pages_matches_oracle(torch, L, orc):
     toks, hids, plan, st = _run(L, torch, m, prompts, cont, kw, 2)
     assert plan["n_offloaded"] == 2 and st["h2d_weight_bytes"] > 0
     _check_vs_oracle(orc, m, prompts, conts, toks, hids)
+
+
+def test_embedding_on_host_frees_a_block_and_is_lossless(torch, L, orc):
+    """loip_config.embed_on_host: the embedding table stays in mapped pinned host
+    memory and the gather reads rows over the host link.  With a vocabulary whose
+    table is larger than a layer block, the same budget then keeps one more layer
+    resident; prefill and decode stay bit-identical to the all-resident run."""
+    m = dict(TINY6, vocab=4096)
+    prompts = [inputs.token_ids(131, 20, m["vocab"]), inputs.token_ids(132, 9, m["vocab"])]
+    cont = [[int(a), int(b)] for a, b in zip(inputs.token_ids(133, 5, 4096), inputs.token_ids(134, 5, 4096))]
+    base = _run(L, torch, m, prompts, cont, dict(max_batch=2, max_ctx=64), 6)
+    kw = dict(max_batch=2, max_ctx=64, n_slots=2)
+    budget = _budget(L, m, kw, 2)  # 2 resident layers + 2 slots + half a block of slack
+    ctx_dev = L.Context(m, L.config(budget=budget, **kw))
+    assert ctx_dev.plan()["n_resident"] == 2
+    ctx_dev.close()
+    ctx = L.Context(m, L.config(budget=budget, embed_on_host=1, **kw))
+    assert ctx.plan()["n_resident"] == 3
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    hid = torch.empty(2, m["hidden"], dtype=torch.float32, device="cuda")
+    toks = [ctx.prefill(prompts, out_hidden=hid)]
+    hids = [hid.cpu().numpy().copy()]
+    for step in cont:
+        toks.append(ctx.decode_step(step, out_hidden=hid))
+        hids.append(hid.cpu().numpy().copy())
+    ctx.close()
+    assert np.array_equal(base[0], np.array(toks))
+    assert np.array_equal(base[1].view(np.uint32), np.array(hids).view(np.uint32))
