@@ -172,11 +172,14 @@ def run_ours(args, rank, world):
     # pinned host memory (one 2 x hidden byte row per token crosses the link) and
     # gives its device bytes to resident layers
     embed_host = 0 if args.embed_on_device or not w["budget"] else 1
+    # streamed layers cross the link losslessly packed unless asked otherwise
+    # (not in the direct-access mode or with the SSD tier, where they stay raw)
+    pack = 0 if args.raw_stream or not w["budget"] else 1
     cfg = loip.config(budget=budget, n_slots=w["n_slots"], max_batch=Bsz, max_ctx=max_ctx,
                       max_prefill_tokens=max_prefill, link_Bps=link_peak * 1e9, hbm_Bps=hbm_peak * 1e9,
                       kv_reserve_bytes=kv_reserve, mode=mode, layer_run_kernel=1 if args.layer_run_kernel else 0,
                       host_budget_bytes=w.get("host_budget", 0), ssd_dir=os.environ.get("LOIP_SSD_DIR"),
-                      embed_on_host=embed_host)
+                      embed_on_host=embed_host, pack_stream=pack)
     t0 = time.time()
     ctx = loip.Context(m, cfg)
     plan = ctx.plan()
@@ -334,6 +337,8 @@ def run_ours(args, rank, world):
                    "layer_kernels": "persistent runs at batch 1" if args.layer_run_kernel else "per-op",
                    "resident_layers": st1["n_resident"],
                    "embedding": "host (mapped)" if embed_host else "device",
+                   "stream": "packed (lossless)" if pack and args.mode != "direct" and not w.get("host_budget")
+                   else "raw",
                    "offloaded_layers": n_off, "offloaded_at_start": n_off0,
                    "offloaded_at_end": plan_end["n_offloaded"], "replans": st_end["n_replans"],
                    "blocks_at_end": {"whole_resident": int((masks == 3).sum()), "mha_streamed": int((masks == 2).sum()),
@@ -485,6 +490,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--mode", default="overlap", choices=sorted(MODES))
+    ap.add_argument("--raw-stream", action="store_true",
+                    help="stream the offloaded layers as raw bf16 blobs instead of losslessly packed")
     ap.add_argument("--embed-on-device", action="store_true",
                     help="keep the embedding table in the device budget even when layers are offloaded")
     ap.add_argument("--layer-run-kernel", action="store_true",

@@ -92,6 +92,12 @@ typedef struct loip_config {
                                    * staging buffers taken out of this budget */
     const char* ssd_dir;          /* directory of the SSD tier's scratch file (caller-owned string,
                                    * read at create; NULL = /tmp) */
+    int32_t pack_stream;          /* 1: streamed layers cross the host link losslessly packed
+                                   * (sign-and-mantissa bytes + 4-bit exponent codes per 1024-word
+                                   * superblock, ~77% of the bytes; unpacked into the slot on the
+                                   * device, bit for bit) -- see loip_k_pack.  Ignored in
+                                   * LOIP_MODE_DIRECT and with the SSD tier (host_budget_bytes > 0).
+                                   * 0: raw blobs (default) */
     int32_t embed_on_host;        /* 1: the embedding table [vocab, hidden] stays in pinned host
                                    * memory, mapped for the device, and the embedding gather reads
                                    * each token's row over the host link (16 KB per token at the 70B
@@ -497,6 +503,25 @@ int loip_k_gemm_bf16(const uint16_t* A, const uint16_t* W, int32_t M, int32_t N,
  * (the losslessness of Sec. IV-A: no weight is changed).  Same layout, sizes
  * and alignment rules as loip_k_gemm_bf16; M * K elements per plane. */
 int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t M, int32_t N, int32_t K, float* x, void* stream);
+
+/* Lossless packing of bf16 weights for the host link (the streamed layers'
+ * transport under loip_config.pack_stream): n_sb superblocks of 1024 words
+ * (in: bf16 [n_sb * 1024], dev, 16-byte aligned) become n_sb packed
+ * superblocks of LOIP_PACKED_SB bytes (out, dev, 16-byte aligned): the
+ * sign-and-mantissa byte of every word, a 4-bit code of its exponent relative
+ * to the superblock's largest exponent (15 binades; code 0 = an exception), and
+ * a 32-byte record (byte 0: that largest exponent; byte 1: the number of
+ * exceptions, <= 7; then the exceptions as uint32 index | exponent << 16).  A
+ * superblock with more than 7 exceptions is not packed: its record says 0xff,
+ * and its index (first_sb + i) is appended to raw_list (dev uint32
+ * [1 + raw_cap]: raw_list[0] counts every such superblock, the first raw_cap
+ * indices follow, in no particular order; raw_list may be NULL).
+ * loip_k_unpack restores every packed superblock bit for bit and leaves the
+ * words of the others untouched.  Lossless: no weight changes (Sec. IV-A). */
+#define LOIP_PACKED_SB 1568
+int loip_k_pack(const uint16_t* in, uint64_t n_sb, uint8_t* out, uint32_t* raw_list, uint32_t first_sb,
+                uint32_t raw_cap, void* stream);
+int loip_k_unpack(const uint8_t* in, uint64_t n_sb, uint16_t* out, void* stream);
 
 /* 0 if no tensor-core GEMM launch has recorded a failure (a bounded pipeline
  * wait that ran out); otherwise the first failure code.  -1 if unreadable. */

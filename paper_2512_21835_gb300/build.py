@@ -10,7 +10,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "libloip.so")
 BUILD = os.path.join(HERE, "_build")
-SOURCES = ["decode.cu", "prefill.cu", "gemm_tc.cu", "attn_tc.cu", "runtime.cu", "plan.cpp", "hostpool.cpp", "noalloc.cu",
+SOURCES = ["decode.cu", "prefill.cu", "gemm_tc.cu", "attn_tc.cu", "pack.cu", "runtime.cu", "plan.cpp", "hostpool.cpp", "noalloc.cu",
            "disktier.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

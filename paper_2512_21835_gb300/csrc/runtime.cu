@@ -76,7 +76,7 @@ struct Request {
 struct Fixed {  // offsets inside the fixed region
     uint64_t embed, lm_head, g_final, x, q, o, a, z, logits, attn_scratch, lm_scratch;
     uint64_t tokens, out_tokens, positions, ctx_lens, row_req, page_table, last_rows, dec_pos, run_sync, qk_raw;
-    uint64_t px, py, pq, po, pa, ptiles;
+    uint64_t px, py, pq, po, pa, ptiles, pack_stage, pack_list;
     uint64_t total;
 };
 
@@ -133,6 +133,21 @@ loip_config normalized(const loip_config* c) {
     return r;
 }
 
+// Packed streaming (loip_config.pack_stream): not with direct access (kernels
+// read the host blobs in place) nor with the SSD tier (its blobs stay raw).
+constexpr uint64_t kPackChunkSb = 32768;  // superblocks per staging chunk (51 MB packed)
+constexpr uint32_t kPackRawCap = 256;     // superblocks per layer that may travel unpacked
+bool packing_enabled(const loip_config* c) {
+    return c->pack_stream && c->mode != LOIP_MODE_DIRECT && c->host_budget_bytes == 0;
+}
+// superblocks per staging chunk: kPackChunkSb, or the larger block of a small layer
+uint64_t pack_chunk_sb(const loip_model_desc* d) {
+    loip_layer_layout_t y{};
+    layout_of(d, &y);
+    const uint64_t big = std::max(y.mha_bytes, y.mlp_bytes) / (2 * kPackWords);
+    return std::max<uint64_t>(1, std::min(kPackChunkSb, big));
+}
+
 Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     Fixed f{};
     const uint64_t H = d->hidden, V = d->vocab, F = d->ffn, qd = (uint64_t)d->n_heads * d->head_dim;
@@ -173,6 +188,10 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     f.po = take(2 * Mp * qd * 2);
     f.pa = take(2 * Mp * F * 2);
     f.ptiles = take((Mp + (uint64_t)B + 16) * 16);  // tensor-core attention's query tiles (int4 each)
+    if (packing_enabled(c)) {  // two staging chunks of packed superblocks, the raw-superblock list
+        f.pack_stage = take(2 * pack_chunk_sb(d) * (uint64_t)kPackedSb);
+        f.pack_list = take(4 * (kPackRawCap + 1));
+    }
     f.total = off;
     return f;
 }
@@ -275,6 +294,150 @@ struct loip_ctx {
     bool weights_loaded = false;
     bool failed = false;
     int prefill_tiles = 0;  // query tiles of the current prefill chunk (tensor-core attention)
+    // ---- packed streaming: each streamed layer's two blocks (units) in the host
+    // pool as packed superblocks; the copy stream moves them chunk by chunk into
+    // a two-chunk device staging ring and the unpack stream expands each chunk
+    // into the slot.  Host area of a layer: [unit 0 packed | unit 0 tail | unit 1
+    // packed | unit 1 tail | up to kPackRawCap raw superblocks of 2048 bytes].
+    struct PackUnit {
+        uint64_t off = 0, n_sb = 0, tail = 0;  // blob offset; packed superblocks; raw tail bytes after them
+        uint64_t host_off = 0;                  // offset of the unit inside the layer's host area
+    };
+    struct PackLayer {
+        bool on = false;
+        std::vector<std::pair<int, uint32_t>> raw;  // (unit, superblock) carried raw, in raw-area order
+    };
+    bool packing = false;
+    uint64_t chunk_sb = 1;  // superblocks per staging chunk
+    PackUnit pu[2];
+    uint64_t pack_area = 0;  // host bytes per packed layer
+    std::vector<PackLayer> pk;
+    cudaStream_t unpack_st = nullptr;
+    cudaEvent_t chunk_ready[2] = {}, chunk_free[2] = {};
+    uint64_t chunk_seq = 0;
+    bool packed(int l) const { return packing && l < (int)pk.size() && pk[l].on; }
+    uint64_t host_bytes(int l) const { return packed(l) ? pack_area : lay.l_size; }
+    void init_packing() {
+        packing = packing_enabled(&cfg);
+        pk.assign(L, PackLayer{});
+        if (!packing) return;
+        chunk_sb = pack_chunk_sb(&desc);
+        const uint64_t offs[2] = {0, lay.mha_bytes}, sizes[2] = {lay.mha_bytes, lay.mlp_bytes};
+        uint64_t at = 0;
+        for (int u = 0; u < 2; ++u) {
+            pu[u].off = offs[u];
+            pu[u].n_sb = sizes[u] / (2 * kPackWords);
+            pu[u].tail = sizes[u] - pu[u].n_sb * 2 * kPackWords;
+            pu[u].host_off = at;
+            at += pu[u].n_sb * kPackedSb + pu[u].tail;
+        }
+        pack_area = at + (uint64_t)kPackRawCap * 2 * kPackWords;
+    }
+    // Packs layer l's blob (device, blob layout at dev) into its host area.
+    // Returns LOIP_OK with pk[l].on set, or LOIP_OK with it cleared when more
+    // than kPackRawCap superblocks would travel raw (the layer then streams raw).
+    int pack_layer(int l, const char* dev) {
+        char* host = static_cast<char*>(host_layer[l]);
+        uint8_t* stage = fixed_ptr<uint8_t>(fx.pack_stage);
+        uint32_t* list = fixed_ptr<uint32_t>(fx.pack_list);
+        cudaStream_t s = compute;
+        std::vector<std::pair<int, uint32_t>> raw;
+        for (int u = 0; u < 2; ++u) {
+            const PackUnit& U = pu[u];
+            cudaError_t e = cudaMemsetAsync(list, 0, 4, s);
+            for (uint64_t c0 = 0; c0 < U.n_sb && e == cudaSuccess; c0 += chunk_sb) {
+                const uint64_t n = std::min<uint64_t>(chunk_sb, U.n_sb - c0);
+                uint8_t* st_c = stage + ((c0 / chunk_sb) & 1) * chunk_sb * kPackedSb;
+                e = launch_pack(reinterpret_cast<const uint16_t*>(dev + U.off) + c0 * kPackWords, n, st_c, list,
+                                (uint32_t)c0, kPackRawCap, s);
+                if (e == cudaSuccess)
+                    e = cudaMemcpyAsync(host + U.host_off + c0 * kPackedSb, st_c, n * kPackedSb,
+                                        cudaMemcpyDeviceToHost, s);
+            }
+            if (e == cudaSuccess && U.tail)
+                e = cudaMemcpyAsync(host + U.host_off + U.n_sb * kPackedSb, dev + U.off + U.n_sb * 2 * kPackWords,
+                                    U.tail, cudaMemcpyDeviceToHost, s);
+            uint32_t h_list[1 + kPackRawCap];
+            if (e == cudaSuccess) e = cudaMemcpyAsync(h_list, list, sizeof h_list, cudaMemcpyDeviceToHost, s);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+            if (e != cudaSuccess) return cuda_fail(e, "weight packing");
+            if (h_list[0] > kPackRawCap || raw.size() + h_list[0] > kPackRawCap) {
+                pk[l].on = false;
+                return LOIP_OK;
+            }
+            std::vector<uint32_t> idx(h_list + 1, h_list + 1 + h_list[0]);
+            std::sort(idx.begin(), idx.end());
+            for (uint32_t i : idx) raw.push_back({u, i});
+        }
+        // the raw superblocks' own bytes, after the units
+        char* raw_area = host + pu[1].host_off + pu[1].n_sb * kPackedSb + pu[1].tail;
+        for (size_t j = 0; j < raw.size(); ++j) {
+            cudaError_t e = cudaMemcpy(raw_area + j * 2 * kPackWords,
+                                       dev + pu[raw[j].first].off + (uint64_t)raw[j].second * 2 * kPackWords,
+                                       2 * kPackWords, cudaMemcpyDeviceToHost);
+            if (e != cudaSuccess) return cuda_fail(e, "weight packing");
+        }
+        pk[l].raw = std::move(raw);
+        pk[l].on = true;
+        return LOIP_OK;
+    }
+    // Stores layer l (device blob at dev) in the host pool packed; when it cannot
+    // be packed (too many raw superblocks) it gets a raw region of its own.
+    int store_packed(int l, const char* dev) {
+        int rc = pack_layer(l, dev);
+        if (rc || pk[l].on) return rc;
+        HostBuf hb;
+        if (host_buf_alloc(lay.l_size, &hb) != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned host allocation failed");
+        host_regions.push_back(hb);
+        host_layer[l] = hb.ptr;
+        cudaError_t e = cudaMemcpy(hb.ptr, dev, lay.l_size, cudaMemcpyDeviceToHost);
+        return e == cudaSuccess ? LOIP_OK : cuda_fail(e, "layer copy to the host pool");
+    }
+    // Enqueues the streamed units of packed layer l into slot `slot`: raw tails
+    // and raw superblocks straight into the slot, packed chunks through the
+    // staging ring (copy stream) and the unpack kernel (unpack stream), which
+    // records slot_full.  Returns the bytes that crossed the link.
+    int enqueue_packed(int l, int slot, cudaStream_t cs, uint64_t* bytes) {
+        const char* host = static_cast<const char*>(host_layer[l]);
+        char* dst = slot_ptr(slot);
+        uint8_t* stage = fixed_ptr<uint8_t>(fx.pack_stage);
+        const char* raw_area = host + pu[1].host_off + pu[1].n_sb * kPackedSb + pu[1].tail;
+        uint64_t moved = 0;
+        cudaError_t e = cudaSuccess;
+        for (int u = 0; u < 2 && e == cudaSuccess; ++u) {
+            if (res_mask[l] & (1 << u)) continue;  // this block is resident
+            const PackUnit& U = pu[u];
+            if (U.tail) {
+                e = cudaMemcpyAsync(dst + U.off + U.n_sb * 2 * kPackWords, host + U.host_off + U.n_sb * kPackedSb,
+                                    U.tail, cudaMemcpyHostToDevice, cs);
+                moved += U.tail;
+            }
+            for (size_t j = 0; j < pk[l].raw.size() && e == cudaSuccess; ++j) {
+                if (pk[l].raw[j].first != u) continue;
+                e = cudaMemcpyAsync(dst + U.off + (uint64_t)pk[l].raw[j].second * 2 * kPackWords,
+                                    raw_area + j * 2 * kPackWords, 2 * kPackWords, cudaMemcpyHostToDevice, cs);
+                moved += 2 * kPackWords;
+            }
+            for (uint64_t c0 = 0; c0 < U.n_sb && e == cudaSuccess; c0 += chunk_sb) {
+                const uint64_t n = std::min<uint64_t>(chunk_sb, U.n_sb - c0);
+                const int g = (int)(chunk_seq++ & 1);
+                uint8_t* st_c = stage + (uint64_t)g * chunk_sb * kPackedSb;
+                e = cudaStreamWaitEvent(cs, chunk_free[g], 0);  // its previous chunk has been unpacked
+                if (e == cudaSuccess)
+                    e = cudaMemcpyAsync(st_c, host + U.host_off + c0 * kPackedSb, n * kPackedSb, cudaMemcpyHostToDevice,
+                                        cs);
+                if (e == cudaSuccess) e = cudaEventRecord(chunk_ready[g], cs);
+                if (e == cudaSuccess) e = cudaStreamWaitEvent(unpack_st, chunk_ready[g], 0);
+                if (e == cudaSuccess)
+                    e = launch_unpack(st_c, n, reinterpret_cast<uint16_t*>(dst + U.off) + c0 * kPackWords, unpack_st);
+                if (e == cudaSuccess) e = cudaEventRecord(chunk_free[g], unpack_st);
+                moved += n * kPackedSb;
+            }
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "packed layer copy");
+        *bytes = moved;
+        return LOIP_OK;
+    }
     // fault injection (loip_inject_fault): one armed fault, fired once
     int fault_kind = 0, fault_arg = 0;
     bool take_fault(int kind) {
@@ -346,6 +509,12 @@ struct loip_ctx {
         if (e != cudaSuccess) return cuda_fail(e, "event record");
         int r = wait_event(ev_done);
         if (r) return r;
+        if (unpack_st) {
+            e = cudaEventRecord(ev_done, unpack_st);
+            if (e != cudaSuccess) return cuda_fail(e, "event record");
+            r = wait_event(ev_done);
+            if (r) return r;
+        }
         e = cudaEventRecord(ev_done, compute);
         if (e != cudaSuccess) return cuda_fail(e, "event record");
         return wait_event(ev_done);
@@ -361,7 +530,15 @@ struct loip_ctx {
         return reinterpret_cast<const uint16_t*>(mlp_at[l] ? mlp_at[l] - lay.mha_bytes : slot_ptr(slot));
     }
     // bytes layer l streams per pass
-    uint64_t stream_bytes(int l) const {
+    uint64_t stream_bytes(int l) const {  // bytes a step moves over the link for layer l
+        if (packed(l)) {
+            uint64_t b = 0;
+            for (int u = 0; u < 2; ++u)
+                if (!(res_mask[l] & (1 << u))) b += pu[u].n_sb * kPackedSb + pu[u].tail;
+            for (const auto& r : pk[l].raw)
+                if (!(res_mask[l] & (1 << r.first))) b += 2 * kPackWords;
+            return b;
+        }
         return ((res_mask[l] & 1) ? 0 : lay.mha_bytes) + ((res_mask[l] & 2) ? 0 : lay.mlp_bytes);
     }
     void set_resident_block(int l, int b) {  // whole layer in block b
@@ -559,6 +736,19 @@ struct loip_ctx {
         }
         cudaEvent_t e0 = take_event(), e1 = take_event();
         cudaEventRecord(e0, cs);
+        if (packed(layer)) {
+            uint64_t moved = 0;
+            int rc = enqueue_packed(layer, slot, cs, &moved);
+            if (rc) return rc;
+            cudaEventRecord(e1, cs);
+            copy_events.push_back({e0, e1, false, moved});
+            // the slot is full once every chunk is unpacked and the raw copies landed
+            e = cudaStreamWaitEvent(unpack_st, e1, 0);
+            if (e == cudaSuccess) e = cudaEventRecord(slot_full[slot], unpack_st);
+            if (e != cudaSuccess) return cuda_fail(e, "slot event");
+            st.h2d_weight_bytes += moved;
+            return LOIP_OK;
+        }
         // the blocks the layer streams, at their blob offsets
         const uint64_t off0 = (res_mask[layer] & 1) ? lay.mha_bytes : 0;
         const uint64_t off1 = (res_mask[layer] & 2) ? lay.mha_bytes : lay.l_size;
@@ -1044,20 +1234,20 @@ struct loip_ctx {
             if (host_layer[l]) pooled.push_back(l);
         if (pooled.empty()) return LOIP_OK;
         cudaEvent_t a = take_event(), b = take_event();
-        auto rate = [&](const void* src, double* gbps) -> int {
+        auto rate = [&](const void* src, double* gbps, uint64_t bytes) -> int {
             cudaEventRecord(a, compute);
-            cudaError_t e = cudaMemcpyAsync(slot_ptr(0), src, lay.l_size, cudaMemcpyHostToDevice, compute);
+            cudaError_t e = cudaMemcpyAsync(slot_ptr(0), src, bytes, cudaMemcpyHostToDevice, compute);
             cudaEventRecord(b, compute);
             if (e == cudaSuccess) e = cudaEventSynchronize(b);
             float ms = 0;
             if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, a, b);
             if (e != cudaSuccess) return cuda_fail(e, "pool qualification copy");
-            *gbps = ms > 0 ? (double)lay.l_size / (ms * 1e-3) / 1e9 : 0.0;
+            *gbps = ms > 0 ? (double)bytes / (ms * 1e-3) / 1e9 : 0.0;
             return LOIP_OK;
         };
         std::vector<double> r(L, 0.0);
         for (int l : pooled) {
-            int rc = rate(host_layer[l], &r[l]);
+            int rc = rate(host_layer[l], &r[l], host_bytes(l));
             if (rc) return rc;
         }
         std::vector<double> sorted;
@@ -1068,11 +1258,12 @@ struct loip_ctx {
         for (int l : pooled) {
             for (int attempt = 0; attempt < 3 && r[l] < 0.9 * median; ++attempt) {
                 HostBuf hb;
-                if (host_buf_alloc(lay.l_size, &hb) != cudaSuccess) break;
+                if (host_buf_alloc(host_bytes(l), &hb) != cudaSuccess) break;
                 double g = 0;
-                int rc = rate(hb.ptr, &g);
+                int rc = rate(hb.ptr, &g, host_bytes(l));
                 if (rc) return rc;
                 if (g > r[l]) {
+                    // (the pool is filled after qualification: nothing to move)
                     host_regions.push_back(hb);
                     host_layer[l] = hb.ptr;
                     r[l] = g;
@@ -1103,7 +1294,7 @@ struct loip_ctx {
         int on = 0;
         for (int l : pooled) {
             double frac = 0;
-            pool_node[l] = host_range_node(host_layer[l], lay.l_size, 32, &frac);
+            pool_node[l] = host_range_node(host_layer[l], host_bytes(l), 32, &frac);
             on += (want >= 0 && pool_node[l] == want) ? 1 : 0;
         }
         st.pool_numa_node = want;
@@ -1118,12 +1309,17 @@ struct loip_ctx {
             if (offloaded[l] && !host_layer[l] && disk_off[l] < 0) need.push_back(l);
         if (need.empty()) return LOIP_OK;
         HostBuf b;
+        // packed layers take their packed area; the layer is marked packed now
+        // and cleared by pack_layer if it has to travel raw after all
+        const uint64_t per = packing ? pack_area : lay.l_size;
         cudaError_t e = take_fault(LOIP_FAULT_HOST_ALLOC) ? cudaErrorMemoryAllocation
-                                                           : host_buf_alloc(need.size() * lay.l_size, &b);
+                                                           : host_buf_alloc(need.size() * per, &b);
         if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
         host_regions.push_back(b);
-        for (size_t i = 0; i < need.size(); ++i)
-            host_layer[need[i]] = static_cast<char*>(b.ptr) + i * lay.l_size;
+        for (size_t i = 0; i < need.size(); ++i) {
+            host_layer[need[i]] = static_cast<char*>(b.ptr) + i * per;
+            if (packing) pk[need[i]].on = true;
+        }
         return qualify_host_pool();
     }
 
@@ -1166,6 +1362,7 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
     if (!ctx) return;
     if (ctx->compute) cudaStreamSynchronize(ctx->compute);
     if (ctx->copy) cudaStreamSynchronize(ctx->copy);
+    if (ctx->unpack_st) cudaStreamSynchronize(ctx->unpack_st);
     for (auto& hb : ctx->host_regions) host_buf_free(&hb);
     host_buf_free(&ctx->embed_host);
     for (int b = 0; b < loip_ctx::kStages; ++b) {
@@ -1186,10 +1383,12 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
         cudaEventDestroy(k.b);
     }
     for (auto e : ctx->event_pool) cudaEventDestroy(e);
-    for (cudaEvent_t e : {ctx->ev_done, ctx->ev_step0, ctx->ev_step1, ctx->ev_reach, ctx->ev_stage})
+    for (cudaEvent_t e : {ctx->ev_done, ctx->ev_step0, ctx->ev_step1, ctx->ev_reach, ctx->ev_stage,
+                          ctx->chunk_ready[0], ctx->chunk_ready[1], ctx->chunk_free[0], ctx->chunk_free[1]})
         if (e) cudaEventDestroy(e);
     if (ctx->compute) cudaStreamDestroy(ctx->compute);
     if (ctx->copy) cudaStreamDestroy(ctx->copy);
+    if (ctx->unpack_st) cudaStreamDestroy(ctx->unpack_st);
     delete ctx;
 }
 
@@ -1216,6 +1415,7 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     c->cfg = cfg;
     layout_of(desc, &c->lay);
     c->L = desc->n_layers;
+    c->init_packing();
     c->H = desc->hidden;
     c->Hq = desc->n_heads;
     c->Hkv = desc->n_kv_heads;
@@ -1359,6 +1559,15 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
     cudaError_t e;
     e = cudaStreamCreateWithFlags(&c->compute, cudaStreamNonBlocking);
     if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->copy, cudaStreamNonBlocking);
+    if (e == cudaSuccess && c->packing) {  // unpack kernels: short, they gate the staging ring
+        int lo = 0, hi = 0;
+        e = cudaDeviceGetStreamPriorityRange(&lo, &hi);
+        if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&c->unpack_st, cudaStreamNonBlocking, hi);
+        for (int g = 0; g < 2 && e == cudaSuccess; ++g) {
+            e = cudaEventCreateWithFlags(&c->chunk_ready[g], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->chunk_free[g], cudaEventDisableTiming);
+        }
+    }
     c->slot_full.resize(cfg.n_slots);
     c->slot_free.resize(cfg.n_slots);
     for (int k = 0; k < cfg.n_slots && e == cudaSuccess; ++k) {
@@ -1480,9 +1689,16 @@ extern "C" int loip_load_weights_generated(loip_ctx* c, uint64_t seed) {
             rc = c->ensure_host_pool();
             if (rc) return rc;
             char* tmp = c->slot_ptr(0);
+            if (c->packed(l)) {  // defined padding between the tensors (it is packed too)
+                e = cudaMemsetAsync(tmp, 0, c->lay.l_size, c->compute);
+                if (e != cudaSuccess) return c->cuda_fail(e, "slot clear");
+            }
             rc = write_layer_generated(c, tmp, l, seed);
             if (rc) return rc;
-            if (c->disk_off[l] >= 0) {  // SSD tier: through a staging buffer to the file
+            if (c->packed(l)) {
+                rc = c->store_packed(l, tmp);
+                if (rc) return rc;
+            } else if (c->disk_off[l] >= 0) {  // SSD tier: through a staging buffer to the file
                 rc = c->sync_all();
                 if (rc) return rc;
                 rc = c->write_disk_blob(l, tmp, cudaMemcpyDeviceToHost);
@@ -1518,6 +1734,11 @@ extern "C" int loip_load_layer(loip_ctx* c, int32_t layer, const void* host_blob
     const char* hb = static_cast<const char*>(host_blob);
     if (c->res_mask[layer] != 3 && c->disk_off[layer] >= 0) {
         rc = c->write_disk_blob(layer, hb, cudaMemcpyHostToHost);
+        if (rc) return rc;
+    } else if (c->res_mask[layer] != 3 && c->packed(layer)) {
+        e = cudaMemcpy(c->slot_ptr(0), hb, bytes, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) return c->cuda_fail(e, "layer upload");
+        rc = c->store_packed(layer, c->slot_ptr(0));
         if (rc) return rc;
     } else if (c->res_mask[layer] != 3) {
         memcpy(c->host_layer[layer], host_blob, bytes);
@@ -2128,6 +2349,19 @@ extern "C" int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t 
     if (!A2 || !W || !x || M < 1 || N < 1 || K < 8 || K % 8 || !al16(A2) || !al16(W) || !al16(x) || N % 4)
         return LOIP_ERR_INVALID;
     return cerr(launch_tc_gemm_resid(A2, true, W, M, N, K, x, (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_pack(const uint16_t* in, uint64_t n_sb, uint8_t* out, uint32_t* raw_list, uint32_t first_sb,
+                           uint32_t raw_cap, void* stream) {
+    if ((!in || !out) && n_sb) return LOIP_ERR_INVALID;
+    if (!al16(in) || !al16(out) || n_sb > (1ull << 32)) return LOIP_ERR_INVALID;
+    return cerr(launch_pack(in, n_sb, out, raw_list, first_sb, raw_cap, (cudaStream_t)stream));
+}
+
+extern "C" int loip_k_unpack(const uint8_t* in, uint64_t n_sb, uint16_t* out, void* stream) {
+    if ((!in || !out) && n_sb) return LOIP_ERR_INVALID;
+    if (!al16(in) || !al16(out)) return LOIP_ERR_INVALID;
+    return cerr(launch_unpack(in, n_sb, out, (cudaStream_t)stream));
 }
 
 extern "C" int loip_k_tc_status(void) {

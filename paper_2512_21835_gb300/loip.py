@@ -38,7 +38,8 @@ class Config(C.Structure):
                 ("max_batch", C.c_int32), ("max_ctx", C.c_int32), ("layer_run_kernel", C.c_int32), ("mode", C.c_int32),
                 ("timeout_ms", C.c_uint32), ("hbm_Bps", C.c_double), ("link_Bps", C.c_double),
                 ("kv_reserve_bytes", C.c_uint64), ("max_prefill_tokens", C.c_int32), ("whole_layers", C.c_int32),
-                ("host_budget_bytes", C.c_uint64), ("ssd_dir", C.c_char_p), ("embed_on_host", C.c_int32)]
+                ("host_budget_bytes", C.c_uint64), ("ssd_dir", C.c_char_p), ("pack_stream", C.c_int32),
+                ("embed_on_host", C.c_int32)]
 
 
 class LayerLayout(C.Structure):
@@ -115,6 +116,8 @@ _SIGS = {
     "loip_k_gemm_split": (C.c_int, [P, P, I32, I32, I32, P, P]),
     "loip_k_prefill_attention": (C.c_int, [P, P, P, I32, P, P, I32, I32, I32, I32, I32, I32, U64, P, P, P]),
     "loip_k_attention_tc_status": (C.c_int, []),
+    "loip_k_pack": (C.c_int, [P, U64, P, P, C.c_uint32, C.c_uint32, P]),
+    "loip_k_unpack": (C.c_int, [P, U64, P, P]),
     "loip_k_tc_status": (C.c_int, []),
 }
 
@@ -168,10 +171,10 @@ def config(budget: int, n_slots: int = 2, max_batch: int = 1, max_ctx: int = 204
            timeout_ms: int = 0, hbm_Bps: float = 6.7e12, link_Bps: float = 2.1e11, kv_reserve_bytes: int = 0,
            max_prefill_tokens: int = 512, page_tokens: int = 64, layer_run_kernel: int = 0,
            whole_layers: int = 0, host_budget_bytes: int = 0, ssd_dir: str | None = None,
-           embed_on_host: int = 0) -> Config:
+           embed_on_host: int = 0, pack_stream: int = 0) -> Config:
     return Config(budget, n_slots, page_tokens, max_batch, max_ctx, layer_run_kernel, mode, timeout_ms, hbm_Bps,
                   link_Bps, kv_reserve_bytes, max_prefill_tokens, whole_layers, host_budget_bytes,
-                  ssd_dir.encode() if ssd_dir else None, embed_on_host)
+                  ssd_dir.encode() if ssd_dir else None, pack_stream, embed_on_host)
 
 
 # ----------------------------------------------------------------------------
@@ -477,6 +480,20 @@ def loip_k_gemm_split(A2, W, x, stream=None):
     as int16 tensors): the split-pair operand at fp32 activation precision."""
     _, M, K = A2.shape
     _check(lib().loip_k_gemm_split(_ptr(A2), _ptr(W), M, W.shape[0], K, _ptr(x), _s(stream)))
+
+
+PACKED_SB = 1568
+
+
+def loip_k_pack(words, packed, raw_list=None, first_sb=0, raw_cap=0, stream=None):
+    """Pack words (int16 [n_sb * 1024]) into packed (uint8 [n_sb * 1568])."""
+    n_sb = words.numel() // 1024
+    _check(lib().loip_k_pack(_ptr(words), n_sb, _ptr(packed), _ptr(raw_list), first_sb, raw_cap, _s(stream)))
+
+
+def loip_k_unpack(packed, words, stream=None):
+    n_sb = packed.numel() // PACKED_SB
+    _check(lib().loip_k_unpack(_ptr(packed), n_sb, _ptr(words), _s(stream)))
 
 
 def loip_k_tc_status() -> int:

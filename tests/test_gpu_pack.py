@@ -1,0 +1,209 @@
+"""Lossless packing of the streamed weights (loip_config.pack_stream).
+
+* Kernel level: loip_k_pack against a numpy packer written from the format's
+  definition (byte for byte, raw list as a set), and loip_k_unpack restoring
+  every packed superblock bit for bit while leaving the unpacked ones alone.
+  Inputs: weight-like bf16 words plus the awkward cases -- zeros and zero runs,
+  subnormals, infinities and NaNs, values far below their superblock's largest
+  (exceptions), norm gains near 1, and superblocks whose exponents are spread
+  so widely that they must travel raw.
+* Runtime: a context that streams packed layers gives bit-identical results to
+  one that streams raw blobs (several slot counts, naive mode, block-level
+  residency), moves fewer bytes over the link, and handles a layer with a few
+  raw superblocks and a layer that cannot be packed at all (loaded through
+  loip_load_layer)."""
+import numpy as np
+import pytest
+
+from gpu_util import need_gpu
+from paper_2512_21835_gb300 import configs, inputs
+
+pytestmark = pytest.mark.gpu
+SB, PACKED = 1024, 1568
+TINY6 = dict(configs.MODELS["tiny"], n_layers=6)
+
+
+@pytest.fixture(scope="module")
+def torch():
+    return need_gpu()
+
+
+@pytest.fixture(scope="module")
+def L(torch):
+    from paper_2512_21835_gb300 import loip
+    return loip
+
+
+def pack_ref(words):
+    """The packed format, from its definition: per 1024-word superblock the
+    sign-and-mantissa bytes, 4-bit exponent codes relative to the largest
+    exponent (code 0 = exception), a 32-byte record (base, exception count or
+    0xff, up to 7 exceptions index | exponent << 16)."""
+    W = words.reshape(-1, SB).astype(np.uint32)
+    n_sb = W.shape[0]
+    E = (W >> 7) & 0xFF
+    base = E.max(axis=1)
+    SM = (((W >> 8) & 0x80) | (W & 0x7F)).astype(np.uint8)
+    C = np.where(E.astype(np.int64) >= base[:, None].astype(np.int64) - 14, E - base[:, None] + 15, 0)
+    codes = (C[:, 0::2] | (C[:, 1::2] << 4)).astype(np.uint8)
+    exc = C == 0
+    nexc = exc.sum(axis=1)
+    rec = np.zeros((n_sb, 8), dtype=np.uint32)
+    rec[:, 0] = base | (np.where(nexc <= 7, nexc, 0xFF) << 8)
+    for sb in np.nonzero((nexc > 0) & (nexc <= 7))[0]:
+        idx = np.nonzero(exc[sb])[0]
+        rec[sb, 1:1 + len(idx)] = idx.astype(np.uint32) | (E[sb, idx] << 16)
+    out = np.concatenate([SM, codes, rec.view(np.uint8).reshape(n_sb, 32)], axis=1)
+    return out.reshape(-1), sorted(np.nonzero(nexc > 7)[0].tolist())
+
+
+def _awkward_words(seed, n_sb):
+    w = inputs.bf16_bits(seed, (n_sb * SB,), 0.02).astype(np.uint16)
+    rng = np.random.default_rng(seed)
+    w[5 * SB:5 * SB + 300] = 0                                  # a zero run (padding)
+    w[7 * SB + 3] = 0x0001                                      # a subnormal
+    w[8 * SB + 9] = 0x7F80                                      # +inf
+    w[8 * SB + 10] = 0xFFC1                                     # a NaN
+    w[9 * SB + rng.integers(0, SB, 5)] = 0x0300                 # 5 tiny values: exceptions
+    w[10 * SB:11 * SB] = inputs.bf16_bits(seed + 1, (SB,), 1.0)  # gains-like values near 1
+    w[10 * SB:11 * SB] = ((w[10 * SB:11 * SB] & 0x807F) | (127 << 7)).astype(np.uint16)
+    w[12 * SB:13 * SB] = rng.integers(0, 1 << 16, SB).astype(np.uint16)  # random patterns: raw
+    w[14 * SB:14 * SB + 8] = 0x0200                             # 8 exceptions: one too many, raw
+    w[15 * SB:15 * SB + 3] = 0x0200                             # 3 (+ any natural ones): packed
+    return w
+
+
+@pytest.mark.parametrize("n_sb", [16, 70001])
+def test_pack_matches_format_and_round_trips(torch, L, n_sb):
+    words = _awkward_words(7 + n_sb, n_sb)
+    want, want_raw = pack_ref(words)
+    dw = torch.from_numpy(words.view(np.int16)).cuda()
+    packed = torch.zeros(n_sb * PACKED, dtype=torch.uint8, device="cuda")
+    raw_list = torch.zeros(1 + 64, dtype=torch.int32, device="cuda")
+    L.loip_k_pack(dw, packed, raw_list, first_sb=1000, raw_cap=64)
+    torch.cuda.synchronize()
+    got = packed.cpu().numpy()
+    assert np.array_equal(got, want)
+    rl = raw_list.cpu().numpy().view(np.uint32)
+    assert rl[0] == len(want_raw) and sorted((rl[1:1 + rl[0]] - 1000).tolist()) == want_raw
+    assert 12 in want_raw and 14 in want_raw
+    nexc = (want.reshape(-1, PACKED)[:, 1537]).astype(int)
+    assert np.any((nexc >= 3) & (nexc <= 7))  # packed superblocks with exceptions are exercised
+    out = torch.full((n_sb * SB,), 0x5555, dtype=torch.int16, device="cuda")
+    L.loip_k_unpack(packed, out)
+    torch.cuda.synchronize()
+    back = out.cpu().numpy().view(np.uint16).reshape(-1, SB)
+    ref = words.reshape(-1, SB)
+    for sb in range(n_sb):
+        if sb in want_raw:
+            assert np.all(back[sb] == 0x5555)  # left for the raw copy
+        else:
+            assert np.array_equal(back[sb], ref[sb]), sb
+    # weight-like words pack to ~77 % of their bytes
+    assert PACKED / (2 * SB) < 0.77
+
+
+def _budget(L, m, kw, resident):
+    lay = L.loip_layer_layout(m)
+    fixed = L.loip_fixed_bytes(m, L.config(budget=1 << 40, **kw))
+    group = ((2 * m["n_kv_heads"] * 64 * m["head_dim"] * 2 * m["n_layers"]) + 255) // 256 * 256
+    blk = (lay["l_size"] + 255) // 256 * 256
+    pages = kw["max_batch"] * ((kw["max_ctx"] + 63) // 64)
+    slots = 0 if resident >= m["n_layers"] else kw.get("n_slots", 2)
+    return fixed + pages * group + 256 + (resident + slots) * blk + blk // 2
+
+
+PROMPTS = [inputs.token_ids(601, 21, 1024), inputs.token_ids(602, 9, 1024)]
+CONT = [[int(a), int(b)] for a, b in zip(inputs.token_ids(603, 5, 1024), inputs.token_ids(604, 5, 1024))]
+
+
+def _run(L, torch, kw, resident, blobs=None, budget=None):
+    m = TINY6
+    budget = budget or _budget(L, m, kw, resident)
+    ctx = L.Context(m, L.config(budget=budget, **kw))
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    for l, blob in (blobs or {}).items():
+        ctx.load_layer(l, blob)
+    hid = torch.empty(2, m["hidden"], dtype=torch.float32, device="cuda")
+    toks = [ctx.prefill(PROMPTS, out_hidden=hid)]
+    hids = [hid.cpu().numpy().copy()]
+    ctx.synchronize()
+    b0 = ctx.stats()["h2d_weight_bytes"]
+    for step in CONT:
+        toks.append(ctx.decode_step(step, out_hidden=hid))
+        hids.append(hid.cpu().numpy().copy())
+    ctx.synchronize()
+    st = ctx.stats()
+    plan = ctx.plan()
+    ctx.close()
+    return np.array(toks), np.array(hids), plan, (st["h2d_weight_bytes"] - b0) / len(CONT)
+
+
+@pytest.mark.parametrize("resident,K,mode", [(2, 2, 0), (0, 1, 0), (2, 3, 0), (2, 1, 1)])
+def test_packed_streaming_is_bitwise_lossless(torch, L, resident, K, mode):
+    kw = dict(max_batch=2, max_ctx=64, n_slots=K, mode=mode)
+    raw = _run(L, torch, kw, resident)
+    pk = _run(L, torch, dict(kw, pack_stream=1), resident)  # its budget counts the staging ring
+    assert pk[2]["n_resident"] == resident
+    assert np.array_equal(raw[0], pk[0])
+    assert np.array_equal(raw[1].view(np.uint32), pk[1].view(np.uint32))
+    assert 0.70 < pk[3] / raw[3] < 0.80, (pk[3], raw[3])  # bytes over the link per step
+
+
+def test_packed_streaming_with_block_residency(torch, L):
+    """One streamed layer keeps its MLP block resident (Algorithm 1's block step):
+    only its MHA unit streams, packed."""
+    m = TINY6
+    lay = L.loip_layer_layout(m)
+    kw = dict(max_batch=2, max_ctx=64, n_slots=2)
+    def budget(k):  # no slack beyond the whole blocks but one MLP block
+        return _budget(L, m, k, 2) - (lay["l_size"] + 255) // 256 * 256 // 2 + lay["mlp_bytes"] + 256
+    kp = dict(kw, pack_stream=1)
+    raw = _run(L, torch, kw, 2, budget=budget(kw))
+    pk = _run(L, torch, kp, 2, budget=budget(kp))
+    assert np.array_equal(raw[0], pk[0])
+    assert np.array_equal(raw[1].view(np.uint32), pk[1].view(np.uint32))
+
+
+def _layer_blob(L, orc, l, seed):
+    """Layer l's blob as loip_load_weights_generated fills it (zero padding)."""
+    m = TINY6
+    lay = L.loip_layer_layout(m)
+    H, F = m["hidden"], m["ffn"]
+    qd, kvd = m["n_heads"] * m["head_dim"], m["n_kv_heads"] * m["head_dim"]
+    blob = np.zeros(lay["l_size"] // 2, dtype=np.uint16)
+    parts = [("off_g_attn", H, 0, 1), ("off_wqkv", qd * H, 1, 0), ("off_wqkv", kvd * H, 2, 0),
+             ("off_wqkv", kvd * H, 3, 0), ("off_wo", H * qd, 4, 0), ("off_g_mlp", H, 5, 1),
+             ("off_wg", F * H, 6, 0), ("off_wu", F * H, 7, 0), ("off_wd", H * F, 8, 0)]
+    extra = {2: qd * H, 3: (qd + kvd) * H}
+    for key, n, which, kind in parts:
+        o = lay[key] // 2 + extra.get(which, 0)
+        blob[o:o + n] = orc.gen_tensor(seed, 16 + 16 * l + which, n, kind)
+    return blob
+
+
+def test_packed_streaming_with_raw_superblocks_and_an_unpackable_layer(torch, L, orc):
+    """Streamed layer 1 gets three superblocks of random bit patterns in its MLP
+    block (carried raw beside the packed stream); streamed layer 2's MLP block is
+    random patterns throughout (more raw superblocks than a layer may carry: the
+    layer streams as a raw blob).  Both contexts load the same blobs; results are
+    bit-identical."""
+    rng = np.random.default_rng(11)
+    lay = L.loip_layer_layout(TINY6)
+    blobs = {}
+    for l, n_bad in ((1, 3), (2, None)):  # offloaded at 2 of 6 resident: layers 1, 2, 4, 5
+        b = _layer_blob(L, orc, l, configs.WEIGHT_SEED)
+        o = lay["off_wd"] // 2
+        if n_bad is None:
+            span = b[lay["mha_bytes"] // 2:]
+        else:
+            span = b[o:o + n_bad * SB]
+        # random signs and mantissas, exponents spread over [100, 126]: finite, small
+        r = rng.integers(0, 1 << 16, span.size).astype(np.uint16)
+        span[:] = (r & 0x807F) | (rng.integers(100, 127, span.size).astype(np.uint16) << 7)
+        blobs[l] = b
+    kw = dict(max_batch=2, max_ctx=64, n_slots=2)
+    raw = _run(L, torch, kw, 2, blobs=blobs)
+    pk = _run(L, torch, dict(kw, pack_stream=1), 2, blobs=blobs)
+    assert np.array_equal(raw[0], pk[0])
+    assert np.array_equal(raw[1].view(np.uint32), pk[1].view(np.uint32))
