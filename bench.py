@@ -40,6 +40,7 @@ METRIC = "decode tokens/s, 70B-shaped bf16 w/ offload; HBM & host-link GB/s vs p
 KERNEL_NAMES = ["qkv_rope", "attention", "o_proj", "gate_up", "down", "lm_head"]
 MODES = {"overlap": 0, "naive": 1, "direct": 2}
 RUN_CLASS = 12  # kernel-timing class of the persistent layer-run kernel
+UNPACK_CLASS = 13  # kernel-timing class of the unpack of packed streamed chunks
 
 # DRAM bytes (read + write) per launch of the gate/up SwiGLU GEMV at batch 1
 # (the persistent kernel, at the 70B and the 8B shape), from an
@@ -59,6 +60,23 @@ def gate_up_traffic(model, batch):
         if hashlib.sha256(f.read()).hexdigest() != GATE_UP_TRAFFIC_SRC:
             return None
     return GATE_UP_TRAFFIC[model]
+
+
+# DRAM bytes (read + write) of the unpack kernel per algorithmic byte (packed
+# chunk read + words written), from an ncu capture of the kernel microbenchmark
+# (one 70B layer's worth of words); valid while pack.cu has this hash.
+UNPACK_TRAFFIC_RATIO = None
+UNPACK_TRAFFIC_SRC = None
+
+
+def unpack_traffic(bytes_per_launch):
+    src = os.path.join(ROOT, "paper_2512_21835_gb300", "csrc", "pack.cu")
+    if UNPACK_TRAFFIC_RATIO is None:
+        return None
+    with open(src, "rb") as f:
+        if hashlib.sha256(f.read()).hexdigest() != UNPACK_TRAFFIC_SRC:
+            return None
+    return int(UNPACK_TRAFFIC_RATIO * bytes_per_launch)
 
 
 def measured_peaks():
@@ -257,6 +275,7 @@ def run_ours(args, rank, world):
                       for i in range(0, per_step * (len(cp_ms) // per_step), per_step)]
     pool_nodes = ctx.pool_nodes()
     # ---- per-kernel durations (CUDA events around every launch, separate pass) ----
+    st_pre_kt = ctx.stats()
     ctx.set_kernel_timing(True)
     for _ in range(steps):
         ctx.decode_step_device(tok, tok2)
@@ -300,12 +319,20 @@ def run_ours(args, rank, world):
         dom_name = f"decode_run (persistent layer run, {per_launch_layers:g} layers per launch)"
         dom_traffic = None
     else:
-        # dominant kernel: the gate/up SwiGLU product (55% of a layer's bytes)
-        dom_bytes = 2 * m["ffn"] * m["hidden"] * 2
+        # dominant kernel: the gate/up SwiGLU product (55% of a layer's bytes), or
+        # the unpack of packed streamed chunks when it takes more of the step
         k = KERNEL_NAMES.index("gate_up")
+        dom_bytes = 2 * m["ffn"] * m["hidden"] * 2
         dom_ms = st["kernel_ms"][k] / max(1, st["kernel_launches"][k])
         dom_name = "gate_up (RMSNorm+SwiGLU GEMV)"
         dom_traffic = gate_up_traffic(w["model"], Bsz)
+        n_up = st["kernel_launches"][UNPACK_CLASS]
+        if n_up and st["kernel_ms"][UNPACK_CLASS] > st["kernel_ms"][k]:
+            # algorithmic bytes of one unpack launch: the packed chunk read plus the words written
+            dom_bytes = int((st["unpack_bytes"] - st_pre_kt["unpack_bytes"]) / n_up)
+            dom_ms = st["kernel_ms"][UNPACK_CLASS] / n_up
+            dom_name = "unpack (packed streamed chunk -> slot, lossless)"
+            dom_traffic = unpack_traffic(dom_bytes)
     dom_gbs = dom_bytes / (dom_ms / 1e3) / 1e9
     hbm_bytes = m["n_layers"] * lay["l_size"] + m["vocab"] * m["hidden"] * 2 + kv_bytes
     # direct access: the offloaded bytes cross the link as kernel reads, whose
@@ -317,7 +344,8 @@ def run_ours(args, rank, world):
     exposed = max(0.0, step_s - max(kernel_sum_ms / 1e3, t_copy_only))
     # embed, 5 per per-op layer or 1 per layer run, LM head + argmax, advance
     per_step_launches = (1 + (m["n_layers"] - (st1["n_resident"] if run_launches else 0)) * 5
-                         + run_launches // steps + 2 + 1)
+                         + run_launches // steps + 2 + 1
+                         + (st1["unpack_launches"] - st0["unpack_launches"]) // steps)
     line = {
         "metric": METRIC,
         "value": round(tokens / dev_s, 4),
@@ -367,6 +395,7 @@ def run_ours(args, rank, world):
                           "pool_blob_GBps_min_median": [round(st1["pool_min_GBps"], 1),
                                                         round(st1["pool_median_GBps"], 1)],
                           "pool_blobs_moved": st1["pool_replaced"],
+                          "pool_huge_page_share_min": round(st1["pool_huge_min"], 4),
                           "pool_numa": {"node": st1["pool_numa_node"], "blobs": st1["pool_blobs"],
                                         "blobs_on_node": st1["pool_blobs_on_node"],
                                         "nodes_seen": sorted({int(v) for v in pool_nodes if v >= 0})},

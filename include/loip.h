@@ -137,7 +137,7 @@ typedef struct loip_stats {
      * decode: 0 qkv+rope, 1 attention (+combine), 2 o-proj, 3 gate/up, 4 down, 5 lm head (+argmax);
      * prefill: 6 qkv GEMM, 7 attention, 8 o-proj GEMM, 9 gate/up GEMM, 10 down GEMM, 11 RMSNorm;
      * 12 persistent layer run (decode at batch 1, a run of resident layers in one launch);
-     * 13-15 unused */
+     * 13 unpack of packed streamed chunks (on the unpack stream); 14-15 unused */
     double kernel_ms[16];
     uint64_t kernel_launches[16];
     double copy_ms_total;      /* summed duration of every completed layer copy (events) */
@@ -153,6 +153,9 @@ typedef struct loip_stats {
     int32_t pool_numa_node;    /* host NUMA node the pool's pages were asked for (the GPU's, -1: none) */
     int32_t pool_blobs;        /* streamed layers with a blob in the host pool */
     int32_t pool_blobs_on_node;/* of those, blobs whose sampled pages are mostly on pool_numa_node */
+    double pool_huge_min;      /* smallest share of a host-pool region in huge pages (1 = all) */
+    uint64_t unpack_launches;  /* unpack kernels enqueued (packed streaming) */
+    uint64_t unpack_bytes;     /* packed bytes they read plus raw bytes they write */
 } loip_stats;
 
 typedef struct loip_ctx loip_ctx;

@@ -12,6 +12,7 @@ struct HostBuf {
     bool mapped = false;   // mmap + cudaHostRegister (else cudaHostAlloc)
     void* dev = nullptr;   // device address of ptr (registered mapped), or nullptr
     int node = -1;         // host NUMA node the pages were asked for (-1: none)
+    double huge = 0.0;     // share of the buffer in transparent huge pages (1 = all)
 };
 // Host NUMA node closest to the current device (cudaDevAttrHostNumaId), or -1
 // when the system reports none or the node does not exist on this host.

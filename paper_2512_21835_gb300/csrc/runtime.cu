@@ -429,9 +429,14 @@ struct loip_ctx {
                 if (e == cudaSuccess) e = cudaEventRecord(chunk_ready[g], cs);
                 if (e == cudaSuccess) e = cudaStreamWaitEvent(unpack_st, chunk_ready[g], 0);
                 if (e == cudaSuccess)
-                    e = launch_unpack(st_c, n, reinterpret_cast<uint16_t*>(dst + U.off) + c0 * kPackWords, unpack_st);
+                    e = timed(13, unpack_st, [&] {
+                        return launch_unpack(st_c, n, reinterpret_cast<uint16_t*>(dst + U.off) + c0 * kPackWords,
+                                             unpack_st);
+                    });
                 if (e == cudaSuccess) e = cudaEventRecord(chunk_free[g], unpack_st);
                 moved += n * kPackedSb;
+                st.unpack_launches += 1;
+                st.unpack_bytes += n * (uint64_t)(kPackedSb + 2 * kPackWords);
             }
         }
         if (e != cudaSuccess) return cuda_fail(e, "packed layer copy");
@@ -1308,18 +1313,43 @@ struct loip_ctx {
         for (int l = 0; l < L; ++l)
             if (offloaded[l] && !host_layer[l] && disk_off[l] < 0) need.push_back(l);
         if (need.empty()) return LOIP_OK;
-        HostBuf b;
         // packed layers take their packed area; the layer is marked packed now
         // and cleared by pack_layer if it has to travel raw after all
         const uint64_t per = packing ? pack_area : lay.l_size;
-        cudaError_t e = take_fault(LOIP_FAULT_HOST_ALLOC) ? cudaErrorMemoryAllocation
-                                                           : host_buf_alloc(need.size() * per, &b);
-        if (e != cudaSuccess) return fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
-        host_regions.push_back(b);
-        for (size_t i = 0; i < need.size(); ++i) {
-            host_layer[need[i]] = static_cast<char*>(b.ptr) + i * per;
-            if (packing) pk[need[i]].on = true;
+        if (take_fault(LOIP_FAULT_HOST_ALLOC)) return fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
+        // regions of about 8 GB, each entirely in huge pages: a region that comes
+        // back partly in base pages is held (so the next try gets other memory)
+        // and allocated again, up to three more times; the best one is kept
+        const size_t group = std::max<size_t>(1, (size_t)((8ull << 30) / per));
+        std::vector<HostBuf> spare;
+        double huge_min = 1.0;
+        for (size_t g0 = 0; g0 < need.size(); g0 += group) {
+            const size_t n = std::min(group, need.size() - g0);
+            HostBuf best;
+            for (int attempt = 0; attempt < 4; ++attempt) {
+                HostBuf b;
+                if (host_buf_alloc(n * per, &b) != cudaSuccess) break;
+                if (!best.ptr || b.huge > best.huge) {
+                    if (best.ptr) spare.push_back(best);
+                    best = b;
+                } else {
+                    spare.push_back(b);
+                }
+                if (best.huge >= 0.999) break;
+            }
+            if (!best.ptr) {
+                for (auto& hb : spare) host_buf_free(&hb);
+                return fail(LOIP_ERR_OOM, "pinned host pool allocation failed");
+            }
+            huge_min = std::min(huge_min, best.huge);
+            host_regions.push_back(best);
+            for (size_t i = 0; i < n; ++i) {
+                host_layer[need[g0 + i]] = static_cast<char*>(best.ptr) + i * per;
+                if (packing) pk[need[g0 + i]].on = true;
+            }
         }
+        for (auto& hb : spare) host_buf_free(&hb);
+        st.pool_huge_min = huge_min;
         return qualify_host_pool();
     }
 

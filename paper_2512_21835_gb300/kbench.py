@@ -118,6 +118,40 @@ def run_tc(iters):
         torch.cuda.empty_cache()
 
 
+def run_pack(iters):
+    """Lossless pack / unpack of one 70B layer's worth of weight-like words
+    (855.6 M words); GB/s over the bytes each kernel reads plus writes."""
+    n_sb = 855654400 // 1024
+    w = _gen(n_sb * 1024, 80)
+    packed = torch.empty(n_sb * L.PACKED_SB, dtype=torch.uint8, device="cuda")
+    out = torch.empty_like(w)
+    tp = _time(lambda i: L.loip_k_pack(w, packed), iters)
+    tu = _time(lambda i: L.loip_k_unpack(packed, out), iters)
+    rw = n_sb * (2048 + L.PACKED_SB)
+    print(f"pack   {n_sb} superblocks: {tp * 1e6:9.1f} us  {rw / tp / 1e9:8.1f} GB/s (read + write)")
+    print(f"unpack {n_sb} superblocks: {tu * 1e6:9.1f} us  {rw / tu / 1e9:8.1f} GB/s (read + write)")
+    del w, packed, out
+    torch.cuda.empty_cache()
+
+
+def run_attn_tc(iters):
+    """Tensor-core causal prefill attention, 70B heads (64 query, 8 kv, d 128), 4
+    prompts x 512 tokens; TFLOP/s over 4 B_r L_q L_k d / 2 (causal half of QK^T and PV)."""
+    Hq, Hkv, d, P, B, n = 64, 8, 128, 64, 4, 512
+    pages = n // P
+    lpb = 2 * Hkv * P * d * 2
+    kv = (torch.randn(B * pages * lpb // 4, device="cuda") * 0.1).view(torch.uint8)
+    pt = (torch.arange(B * pages, device="cuda", dtype=torch.int64) * lpb).view(B, pages)
+    q = torch.randn(B * n, Hq * d, device="cuda") * 0.3
+    tiles = torch.empty((B * n + B) * 4, dtype=torch.int32, device="cuda")
+    o2 = torch.empty(2, B * n, Hq * d, dtype=torch.int16, device="cuda")
+    t = _time(lambda i: L.loip_k_prefill_attention(q, kv, pt, pages, [n] * B, None, Hq, Hkv, d, P, 0, lpb, tiles,
+                                                   o2), iters)
+    flops = 2 * 2 * B * Hq * d * (n * (n + 1) / 2)
+    print(f"prefill attention 4 x 512, 70B heads: {t * 1e6:9.1f} us  {flops / t / 1e12:7.1f} TFLOP/s "
+          f"(x80 layers: {80 * t * 1e3:.1f} ms)  status {L.loip_k_attention_tc_status()}")
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--only", default="")
@@ -131,6 +165,10 @@ def main():
             run_shape(name, a.only, a.B, a.iters)
     if a.only in ("", "tc"):
         run_tc(max(3, min(a.iters, 10)))
+    if a.only in ("", "pack"):
+        run_pack(max(3, min(a.iters, 10)))
+    if a.only in ("", "attn_tc"):
+        run_attn_tc(max(3, min(a.iters, 10)))
 
 
 if __name__ == "__main__":

@@ -63,7 +63,8 @@ class Stats(C.Structure):
                 ("pool_min_GBps", C.c_double), ("pool_median_GBps", C.c_double), ("pool_replaced", C.c_uint64),
                 ("n_ssd_layers", C.c_int32), ("ssd_read_bytes", C.c_uint64), ("ssd_wait_ms", C.c_double),
                 ("ssd_stage_wait_ms", C.c_double), ("ssd_copy_ms", C.c_double), ("pool_numa_node", C.c_int32),
-                ("pool_blobs", C.c_int32), ("pool_blobs_on_node", C.c_int32)]
+                ("pool_blobs", C.c_int32), ("pool_blobs_on_node", C.c_int32), ("pool_huge_min", C.c_double),
+                ("unpack_launches", C.c_uint64), ("unpack_bytes", C.c_uint64)]
 
 
 P, U64, I32, U32, F32, F64, VP = C.c_void_p, C.c_uint64, C.c_int32, C.c_uint32, C.c_float, C.c_double, C.c_void_p
