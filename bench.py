@@ -65,8 +65,8 @@ def gate_up_traffic(model, batch):
 # DRAM bytes (read + write) of the unpack kernel per algorithmic byte (packed
 # chunk read + words written), from an ncu capture of the kernel microbenchmark
 # (one 70B layer's worth of words); valid while pack.cu has this hash.
-UNPACK_TRAFFIC_RATIO = None
-UNPACK_TRAFFIC_SRC = None
+UNPACK_TRAFFIC_RATIO = 0.98104  # 2,964,243,968 B over 3,021,529,600 algorithmic (writes still in L2 at exit)
+UNPACK_TRAFFIC_SRC = "59744d91fc9014212e37fb8037237312cf69d5807563fd24e7e4c209eebad4fb"
 
 
 def unpack_traffic(bytes_per_launch):

@@ -18,7 +18,8 @@
 //                       more than 7 exceptions -- and its 2048 raw bytes travel
 //                       separately), bytes 4 + 4k: exception k = index | exponent << 16
 //
-// One warp per superblock in both directions; lane j handles words 32 j .. 32 j + 31.
+// One warp per superblock in both directions; in the pack kernel lane j handles
+// words 32 j .. 32 j + 31.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -98,45 +99,67 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint16_t* __restrict__ 
     }
 }
 
+// Unpack: lane j of the warp takes words 8j .. 8j + 7 of each quarter (256
+// words) of the superblock, so every load and store of the warp is one
+// contiguous run (256 sign-and-mantissa bytes, 128 code bytes, 512 output
+// bytes); the words are rebuilt two at a time in 32-bit registers.
+__device__ __forceinline__ uint32_t unpack_pair(uint32_t sm4, uint32_t sel, uint32_t code_byte, uint32_t add) {
+    const uint32_t t = __byte_perm(sm4, 0u, sel);                // byte b0 | byte b1 << 16
+    const uint32_t n = __byte_perm(code_byte, 0u, 0x4040u);      // the two codes, in both halves
+    uint32_t e = (n & 0x0000000fu) | ((n >> 4) & 0x000f0000u);   // code of word 0 | code of word 1 << 16
+    e = (e + add) & 0x00ff00ffu;                                 // base + code - 15, modulo 256, per half
+    return ((t & 0x00800080u) << 8) | (e << 7) | (t & 0x007f007fu);
+}
+
+// Exception k of the superblock (word index | exponent << 16) into the register
+// of the lane that holds the word.
+__device__ __forceinline__ void unpack_patch(uint4 (&o)[4], int lane, uint32_t x) {
+    const int idx = (int)(x & 0xffffu);
+    if (((idx >> 3) & 31) != lane) return;
+    const int quarter = idx >> 8, q = idx & 7;
+    const int sh = 7 + 16 * (q & 1);
+    const uint32_t keep = ~(0xffu << sh), v = ((x >> 16) & 0xffu) << sh;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        if (k != quarter) continue;
+        if ((q >> 1) == 0) o[k].x = (o[k].x & keep) | v;
+        if ((q >> 1) == 1) o[k].y = (o[k].y & keep) | v;
+        if ((q >> 1) == 2) o[k].z = (o[k].z & keep) | v;
+        if ((q >> 1) == 3) o[k].w = (o[k].w & keep) | v;
+    }
+}
+
 __global__ void __launch_bounds__(256) unpack_kernel(const uint8_t* __restrict__ in, uint64_t n_sb,
                                                      uint16_t* __restrict__ out) {
     const uint64_t sb = (uint64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
     if (sb >= n_sb) return;
     const int lane = threadIdx.x & 31;
     const uint8_t* src = in + sb * kPackedSb;
-    const uint32_t r = lane < 8 ? reinterpret_cast<const uint32_t*>(src + 1536)[lane] : 0u;
-    const uint32_t head = __shfl_sync(0xffffffffu, r, 0);
-    const int base = (int)(head & 0xffu), n_exc = (int)((head >> 8) & 0xffu);
-    if (n_exc == 0xff) return;  // carried raw
-    const uint4 s0 = reinterpret_cast<const uint4*>(src + lane * 32)[0];
-    const uint4 s1 = reinterpret_cast<const uint4*>(src + lane * 32)[1];
-    const uint4 cv = *reinterpret_cast<const uint4*>(src + 1024 + lane * 16);
-    const uint32_t sm[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-    const uint32_t codes[4] = {cv.x, cv.y, cv.z, cv.w};
-    uint32_t exc[kPackMaxExc];
+    // every load first: read once, evict first
+    uint2 sm[4];
+    uint32_t codes[4];
 #pragma unroll
-    for (int k = 0; k < kPackMaxExc; ++k) exc[k] = __shfl_sync(0xffffffffu, r, 1 + k);
-    uint32_t o[16];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-        const uint32_t b = (sm[i >> 2] >> ((i & 3) * 8)) & 0xffu;
-        const int c = (int)((codes[i >> 3] >> ((i & 7) * 4)) & 0xfu);
-        uint32_t e = (uint32_t)(base + c - 15);
-        if (c == 0) {
-            e = 0;
-#pragma unroll
-            for (int k = 0; k < kPackMaxExc; ++k)
-                if (k < n_exc && (exc[k] & 0xffffu) == (uint32_t)(lane * 32 + i)) e = exc[k] >> 16;
-        }
-        const uint32_t x = ((b & 0x80u) << 8) | ((e & 0xffu) << 7) | (b & 0x7fu);
-        if (i & 1)
-            o[i >> 1] |= x << 16;
-        else
-            o[i >> 1] = x;
+    for (int k = 0; k < 4; ++k) {
+        sm[k] = __ldcs(reinterpret_cast<const uint2*>(src + 256 * k) + lane);
+        codes[k] = __ldcs(reinterpret_cast<const uint32_t*>(src + 1024 + 128 * k) + lane);
     }
-    uint4* dst = reinterpret_cast<uint4*>(out + sb * kPackWords + lane * 32);
+    const uint32_t r = lane < 8 ? __ldcs(reinterpret_cast<const uint32_t*>(src + 1536) + lane) : 0u;
+    const uint32_t head = __shfl_sync(0xffffffffu, r, 0);
+    const uint32_t base = head & 0xffu, n_exc = (head >> 8) & 0xffu;
+    if (n_exc == 0xffu) return;  // carried raw
+    const uint32_t add = ((base + 241u) & 0xffu) * 0x10001u;  // 241 = -15 modulo 256
+    uint4 o[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+    for (int k = 0; k < 4; ++k) {
+        o[k].x = unpack_pair(sm[k].x, 0x4140u, codes[k], add);
+        o[k].y = unpack_pair(sm[k].x, 0x4342u, codes[k] >> 8, add);
+        o[k].z = unpack_pair(sm[k].y, 0x4140u, codes[k] >> 16, add);
+        o[k].w = unpack_pair(sm[k].y, 0x4342u, codes[k] >> 24, add);
+    }
+    for (uint32_t k = 0; k < n_exc; ++k) unpack_patch(o, lane, __shfl_sync(0xffffffffu, r, 1 + k));
+    uint4* dst = reinterpret_cast<uint4*>(out + sb * kPackWords) + lane;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) __stcs(dst + 32 * k, o[k]);  // streamed out: not read again soon
 }
 
 }  // namespace

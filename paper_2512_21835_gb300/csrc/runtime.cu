@@ -140,6 +140,16 @@ constexpr uint32_t kPackRawCap = 256;     // superblocks per layer that may trav
 bool packing_enabled(const loip_config* c) {
     return c->pack_stream && c->mode != LOIP_MODE_DIRECT && c->host_budget_bytes == 0;
 }
+// Chunks in the device staging ring.  A chunk is unpacked by a kernel on its
+// own stream, which only gets SMs when a compute kernel ends: during a prefill
+// pass the tensor-core GEMMs hold every SM for up to a few ms (the gate/up GEMM
+// of 2048 rows at the 70B shape: ~2.3 ms, ten chunks' worth of link time), so
+// the ring grows with the prefill rows to keep the copy engine busy: two chunks
+// up to 512 rows, one more per 256 rows above, at most kPackRingMax.
+constexpr int kPackRingMax = 8;
+int pack_ring_chunks(const loip_config* c) {
+    return std::max(2, std::min(kPackRingMax, c->max_prefill_tokens / 256));
+}
 // superblocks per staging chunk: kPackChunkSb, or the larger block of a small layer
 uint64_t pack_chunk_sb(const loip_model_desc* d) {
     loip_layer_layout_t y{};
@@ -188,8 +198,8 @@ Fixed fixed_layout(const loip_model_desc* d, const loip_config* c) {
     f.po = take(2 * Mp * qd * 2);
     f.pa = take(2 * Mp * F * 2);
     f.ptiles = take((Mp + (uint64_t)B + 16) * 16);  // tensor-core attention's query tiles (int4 each)
-    if (packing_enabled(c)) {  // two staging chunks of packed superblocks, the raw-superblock list
-        f.pack_stage = take(2 * pack_chunk_sb(d) * (uint64_t)kPackedSb);
+    if (packing_enabled(c)) {  // the staging ring of packed superblocks, the raw-superblock list
+        f.pack_stage = take((uint64_t)pack_ring_chunks(c) * pack_chunk_sb(d) * (uint64_t)kPackedSb);
         f.pack_list = take(4 * (kPackRawCap + 1));
     }
     f.total = off;
@@ -296,7 +306,7 @@ struct loip_ctx {
     int prefill_tiles = 0;  // query tiles of the current prefill chunk (tensor-core attention)
     // ---- packed streaming: each streamed layer's two blocks (units) in the host
     // pool as packed superblocks; the copy stream moves them chunk by chunk into
-    // a two-chunk device staging ring and the unpack stream expands each chunk
+    // a device staging ring (pack_ring_chunks) and the unpack stream expands each chunk
     // into the slot.  Host area of a layer: [unit 0 packed | unit 0 tail | unit 1
     // packed | unit 1 tail | up to kPackRawCap raw superblocks of 2048 bytes].
     struct PackUnit {
@@ -309,12 +319,50 @@ struct loip_ctx {
     };
     bool packing = false;
     uint64_t chunk_sb = 1;  // superblocks per staging chunk
+    int ring = 2;           // chunks in the staging ring
     PackUnit pu[2];
     uint64_t pack_area = 0;  // host bytes per packed layer
     std::vector<PackLayer> pk;
     cudaStream_t unpack_st = nullptr;
-    cudaEvent_t chunk_ready[2] = {}, chunk_free[2] = {};
-    uint64_t chunk_seq = 0;
+    cudaEvent_t chunk_ready[kPackRingMax] = {}, chunk_free[kPackRingMax] = {};
+    // The pieces of packed layer copies wait in pack_fifo, in ring order, until
+    // pump() enqueues them.  A packed chunk takes staging entry seq % ring; the
+    // pump hands out sequence number seq only once the unpack of seq - ring, the
+    // entry's previous chunk, has been enqueued (so that every wait on
+    // chunk_free / chunk_ready refers to the right record).  A layer's pieces are
+    // its chunks, then one end job: the raw tails and raw superblocks, copied
+    // straight into the slot after the slot is free.
+    //
+    // Where a chunk is unpacked is fixed when its layer's copy is issued: by a
+    // kernel on the unpack stream (prefill passes, explicit stream_layer calls,
+    // naive mode; slot_full is recorded there), or inline, on the compute stream
+    // right before the layer computes (decode passes: the step waits on the link
+    // anyway, and an unpack on its own stream would queue behind the decode
+    // GEMVs, whose persistent blocks hold every SM).
+    struct PackJob {
+        int layer, slot, unit;  // unit 0 / 1: a chunk of that block; 2: the end job
+        uint64_t c0, n;         // chunk: first superblock and count
+        bool inl;               // unpacked inline by the compute stream
+        bool first;             // the layer's first piece (copy timing starts)
+        cudaStream_t cs;        // copy stream
+    };
+    struct InlineChunk {
+        uint64_t seq;
+        int unit;
+        uint64_t c0, n;
+    };
+    std::deque<PackJob> pack_fifo;
+    uint64_t ring_next = 0, ring_done = 0;  // sequence numbers handed out; below ring_done: unpack enqueued
+    std::deque<bool> ring_unpacked;         // seq in [ring_done, ring_next): unpack enqueued
+    bool inline_unpack = false;             // copies issued now unpack inline (decode passes)
+    // per slot: the layer it is being filled with unpacks inline; its pumped
+    // chunks awaiting their unpack; chunks not yet unpack-enqueued; end job pumped
+    std::vector<uint8_t> slot_inline, raw_pumped;
+    std::vector<std::deque<InlineChunk>> inl_chunks;
+    std::vector<int> inl_left;
+    std::vector<cudaEvent_t> raw_done;      // per slot: the end job's copies landed (copy stream)
+    cudaEvent_t pump_e0 = nullptr;          // copy timing of the layer being pumped
+    uint64_t pump_bytes = 0;
     bool packed(int l) const { return packing && l < (int)pk.size() && pk[l].on; }
     uint64_t host_bytes(int l) const { return packed(l) ? pack_area : lay.l_size; }
     void init_packing() {
@@ -322,6 +370,7 @@ struct loip_ctx {
         pk.assign(L, PackLayer{});
         if (!packing) return;
         chunk_sb = pack_chunk_sb(&desc);
+        ring = pack_ring_chunks(&cfg);
         const uint64_t offs[2] = {0, lay.mha_bytes}, sizes[2] = {lay.mha_bytes, lay.mlp_bytes};
         uint64_t at = 0;
         for (int u = 0; u < 2; ++u) {
@@ -393,55 +442,189 @@ struct loip_ctx {
         cudaError_t e = cudaMemcpy(hb.ptr, dev, lay.l_size, cudaMemcpyDeviceToHost);
         return e == cudaSuccess ? LOIP_OK : cuda_fail(e, "layer copy to the host pool");
     }
-    // Enqueues the streamed units of packed layer l into slot `slot`: raw tails
-    // and raw superblocks straight into the slot, packed chunks through the
-    // staging ring (copy stream) and the unpack kernel (unpack stream), which
-    // records slot_full.  Returns the bytes that crossed the link.
-    int enqueue_packed(int l, int slot, cudaStream_t cs, uint64_t* bytes) {
-        const char* host = static_cast<const char*>(host_layer[l]);
-        char* dst = slot_ptr(slot);
-        uint8_t* stage = fixed_ptr<uint8_t>(fx.pack_stage);
-        const char* raw_area = host + pu[1].host_off + pu[1].n_sb * kPackedSb + pu[1].tail;
-        uint64_t moved = 0;
-        cudaError_t e = cudaSuccess;
-        for (int u = 0; u < 2 && e == cudaSuccess; ++u) {
+    // Queues the pieces of packed layer l (streamed units only) for slot `slot`
+    // and pumps what the ring allows.
+    int queue_packed(int l, int slot, cudaStream_t cs, bool inl) {
+        bool first = true;
+        int chunks = 0;
+        uint64_t bytes = 0;  // what the layer's copies will move over the link
+        for (int u = 0; u < 2; ++u) {
             if (res_mask[l] & (1 << u)) continue;  // this block is resident
-            const PackUnit& U = pu[u];
-            if (U.tail) {
-                e = cudaMemcpyAsync(dst + U.off + U.n_sb * 2 * kPackWords, host + U.host_off + U.n_sb * kPackedSb,
-                                    U.tail, cudaMemcpyHostToDevice, cs);
-                moved += U.tail;
-            }
-            for (size_t j = 0; j < pk[l].raw.size() && e == cudaSuccess; ++j) {
-                if (pk[l].raw[j].first != u) continue;
-                e = cudaMemcpyAsync(dst + U.off + (uint64_t)pk[l].raw[j].second * 2 * kPackWords,
-                                    raw_area + j * 2 * kPackWords, 2 * kPackWords, cudaMemcpyHostToDevice, cs);
-                moved += 2 * kPackWords;
-            }
-            for (uint64_t c0 = 0; c0 < U.n_sb && e == cudaSuccess; c0 += chunk_sb) {
-                const uint64_t n = std::min<uint64_t>(chunk_sb, U.n_sb - c0);
-                const int g = (int)(chunk_seq++ & 1);
-                uint8_t* st_c = stage + (uint64_t)g * chunk_sb * kPackedSb;
-                e = cudaStreamWaitEvent(cs, chunk_free[g], 0);  // its previous chunk has been unpacked
-                if (e == cudaSuccess)
-                    e = cudaMemcpyAsync(st_c, host + U.host_off + c0 * kPackedSb, n * kPackedSb, cudaMemcpyHostToDevice,
-                                        cs);
-                if (e == cudaSuccess) e = cudaEventRecord(chunk_ready[g], cs);
-                if (e == cudaSuccess) e = cudaStreamWaitEvent(unpack_st, chunk_ready[g], 0);
-                if (e == cudaSuccess)
-                    e = timed(13, unpack_st, [&] {
-                        return launch_unpack(st_c, n, reinterpret_cast<uint16_t*>(dst + U.off) + c0 * kPackWords,
-                                             unpack_st);
-                    });
-                if (e == cudaSuccess) e = cudaEventRecord(chunk_free[g], unpack_st);
-                moved += n * kPackedSb;
-                st.unpack_launches += 1;
-                st.unpack_bytes += n * (uint64_t)(kPackedSb + 2 * kPackWords);
+            bytes += pu[u].n_sb * kPackedSb + pu[u].tail;
+            for (const auto& r : pk[l].raw) bytes += r.first == u ? 2 * kPackWords : 0;
+            // equal chunks of at most chunk_sb superblocks (no short last chunk)
+            const uint64_t nc = (pu[u].n_sb + chunk_sb - 1) / chunk_sb;
+            const uint64_t per = nc ? (pu[u].n_sb + nc - 1) / nc : 1;
+            for (uint64_t c0 = 0; c0 < pu[u].n_sb; c0 += per) {
+                pack_fifo.push_back({l, slot, u, c0, std::min<uint64_t>(per, pu[u].n_sb - c0), inl, first, cs});
+                first = false;
+                ++chunks;
             }
         }
+        pack_fifo.push_back({l, slot, 2, 0, 0, inl, first, cs});
+        slot_inline[slot] = inl;
+        inl_left[slot] = inl ? chunks : 0;
+        raw_pumped[slot] = 0;
+        st.h2d_weight_bytes += bytes;  // counted when issued, like raw layer copies
+        return pump();
+    }
+    void mark_unpacked(uint64_t seq) {
+        ring_unpacked[seq - ring_done] = true;
+        while (!ring_unpacked.empty() && ring_unpacked.front()) {
+            ring_unpacked.pop_front();
+            ++ring_done;
+        }
+    }
+    // Unpack of one staged chunk into its slot, on stream s.
+    cudaError_t enqueue_unpack(uint64_t seq, int slot, int unit, uint64_t c0, uint64_t n, cudaStream_t s) {
+        const int g = (int)(seq % (uint64_t)ring);
+        const uint8_t* st_c = fixed_ptr<uint8_t>(fx.pack_stage) + (uint64_t)g * chunk_sb * kPackedSb;
+        uint16_t* out = reinterpret_cast<uint16_t*>(slot_ptr(slot) + pu[unit].off) + c0 * kPackWords;
+        cudaError_t e = cudaStreamWaitEvent(s, chunk_ready[g], 0);
+        if (e == cudaSuccess) e = timed(13, s, [&] { return launch_unpack(st_c, n, out, s); });
+        if (e == cudaSuccess) e = cudaEventRecord(chunk_free[g], s);
+        mark_unpacked(seq);
+        st.unpack_launches += 1;
+        st.unpack_bytes += n * (uint64_t)(kPackedSb + 2 * kPackWords);
+        return e;
+    }
+    // Enqueues queued pieces in order while the staging ring has room.
+    int pump() {
+        cudaError_t e = cudaSuccess;
+        while (!pack_fifo.empty() && e == cudaSuccess) {
+            const PackJob j = pack_fifo.front();
+            const char* host = static_cast<const char*>(host_layer[j.layer]);
+            char* dst = slot_ptr(j.slot);
+            if (j.unit < 2 && ring_next >= ring_done + (uint64_t)ring) break;  // entry still in use
+            if (j.first) {
+                pump_e0 = take_event();
+                pump_bytes = 0;
+                e = cudaEventRecord(pump_e0, j.cs);
+                if (e != cudaSuccess) break;
+                if (!j.inl) e = cudaStreamWaitEvent(unpack_st, slot_free[j.slot], 0);  // unpacks write the slot
+                if (e != cudaSuccess) break;
+            }
+            if (j.unit < 2) {
+                const PackUnit& U = pu[j.unit];
+                const uint64_t seq = ring_next++;
+                ring_unpacked.push_back(false);
+                const int g = (int)(seq % (uint64_t)ring);
+                uint8_t* st_c = fixed_ptr<uint8_t>(fx.pack_stage) + (uint64_t)g * chunk_sb * kPackedSb;
+                e = cudaStreamWaitEvent(j.cs, chunk_free[g], 0);  // the entry's previous chunk has been unpacked
+                if (e == cudaSuccess)
+                    e = cudaMemcpyAsync(st_c, host + U.host_off + j.c0 * kPackedSb, j.n * kPackedSb,
+                                        cudaMemcpyHostToDevice, j.cs);
+                if (e == cudaSuccess) e = cudaEventRecord(chunk_ready[g], j.cs);
+                pump_bytes += j.n * kPackedSb;
+                if (e == cudaSuccess) {
+                    if (j.inl)
+                        inl_chunks[j.slot].push_back({seq, j.unit, j.c0, j.n});
+                    else
+                        e = enqueue_unpack(seq, j.slot, j.unit, j.c0, j.n, unpack_st);
+                }
+            } else {  // end job: raw tails and raw superblocks into the slot once it is free
+                const char* raw_area = host + pu[1].host_off + pu[1].n_sb * kPackedSb + pu[1].tail;
+                e = cudaStreamWaitEvent(j.cs, slot_free[j.slot], 0);
+                for (int u = 0; u < 2 && e == cudaSuccess; ++u) {
+                    if (res_mask[j.layer] & (1 << u)) continue;
+                    const PackUnit& U = pu[u];
+                    if (U.tail) {
+                        e = cudaMemcpyAsync(dst + U.off + U.n_sb * 2 * kPackWords,
+                                            host + U.host_off + U.n_sb * kPackedSb, U.tail, cudaMemcpyHostToDevice,
+                                            j.cs);
+                        pump_bytes += U.tail;
+                    }
+                    for (size_t r = 0; r < pk[j.layer].raw.size() && e == cudaSuccess; ++r) {
+                        if (pk[j.layer].raw[r].first != u) continue;
+                        e = cudaMemcpyAsync(dst + U.off + (uint64_t)pk[j.layer].raw[r].second * 2 * kPackWords,
+                                            raw_area + r * 2 * kPackWords, 2 * kPackWords, cudaMemcpyHostToDevice,
+                                            j.cs);
+                        pump_bytes += 2 * kPackWords;
+                    }
+                }
+                cudaEvent_t e1 = take_event();
+                if (e == cudaSuccess) e = cudaEventRecord(e1, j.cs);
+                if (e == cudaSuccess) {
+                    copy_events.push_back({pump_e0, e1, false, pump_bytes});
+                    if (j.inl) {
+                        e = cudaEventRecord(raw_done[j.slot], j.cs);
+                    } else {  // the slot is full once every chunk is unpacked and the raw copies landed
+                        e = cudaStreamWaitEvent(unpack_st, e1, 0);
+                        if (e == cudaSuccess) e = cudaEventRecord(slot_full[j.slot], unpack_st);
+                    }
+                }
+                raw_pumped[j.slot] = 1;
+            }
+            pack_fifo.pop_front();
+        }
         if (e != cudaSuccess) return cuda_fail(e, "packed layer copy");
-        *bytes = moved;
         return LOIP_OK;
+    }
+    // Before a packed layer in `slot` computes on stream s: its inline unpacks
+    // (each after its chunk landed) and the wait for its raw pieces, or the wait
+    // for slot_full.
+    int wait_packed_slot(int slot, cudaStream_t s) {
+        cudaError_t e = cudaSuccess;
+        while (inl_left[slot] > 0) {
+            if (inl_chunks[slot].empty()) {
+                int rc = pump();
+                if (rc) return rc;
+                if (inl_chunks[slot].empty()) return fail(LOIP_ERR_STATE, "packed copy queue out of order");
+            }
+            const InlineChunk c = inl_chunks[slot].front();
+            inl_chunks[slot].pop_front();
+            --inl_left[slot];
+            e = enqueue_unpack(c.seq, slot, c.unit, c.c0, c.n, s);
+            if (e != cudaSuccess) return cuda_fail(e, "unpack kernel");
+            chain = false;
+            int rc = pump();  // the freed entry lets the next chunk's copy go
+            if (rc) return rc;
+        }
+        while (!raw_pumped[slot]) {
+            const size_t before = pack_fifo.size();
+            int rc = pump();
+            if (rc) return rc;
+            if (pack_fifo.size() == before) return fail(LOIP_ERR_STATE, "packed copy queue stalled");
+        }
+        e = cudaStreamWaitEvent(s, slot_inline[slot] ? raw_done[slot] : slot_full[slot], 0);
+        if (e != cudaSuccess) return cuda_fail(e, "compute wait");
+        return LOIP_OK;
+    }
+    // Hands every inline unpack still pending to the unpack stream (before a
+    // prefill pass or an explicit stream_layer call), so that those layers'
+    // slots get slot_full without the compute stream's help.
+    int flush_inline() {
+        if (!packing) return LOIP_OK;
+        for (auto& j : pack_fifo) j.inl = false;
+        for (int s = 0; s < cfg.n_slots; ++s) {
+            if (!slot_inline[s]) continue;
+            cudaError_t e = cudaStreamWaitEvent(unpack_st, slot_free[s], 0);
+            while (e == cudaSuccess && !inl_chunks[s].empty()) {
+                const InlineChunk c = inl_chunks[s].front();
+                inl_chunks[s].pop_front();
+                e = enqueue_unpack(c.seq, s, c.unit, c.c0, c.n, unpack_st);
+            }
+            if (e == cudaSuccess && raw_pumped[s]) {  // end job already enqueued: slot_full after it
+                e = cudaStreamWaitEvent(unpack_st, raw_done[s], 0);
+                if (e == cudaSuccess) e = cudaEventRecord(slot_full[s], unpack_st);
+            }
+            if (e != cudaSuccess) return cuda_fail(e, "unpack kernel");
+            slot_inline[s] = 0;
+            inl_left[s] = 0;
+        }
+        return pump();
+    }
+    // Forgets queued and staged pieces (the streams are idle: after sync_all).
+    void reset_pack_queue() {
+        pack_fifo.clear();
+        ring_done = ring_next;
+        ring_unpacked.clear();
+        for (int s = 0; s < (int)slot_inline.size(); ++s) {
+            slot_inline[s] = 0;
+            raw_pumped[s] = 1;
+            inl_left[s] = 0;
+            inl_chunks[s].clear();
+        }
     }
     // fault injection (loip_inject_fault): one armed fault, fired once
     int fault_kind = 0, fault_arg = 0;
@@ -727,9 +910,10 @@ struct loip_ctx {
     }
 
     // ---- streaming ------------------------------------------------------------
-    int enqueue_copy(int layer, int slot, cudaStream_t cs) {
+    int enqueue_copy(int layer, int slot, cudaStream_t cs, bool inl = false) {
         if (take_fault(LOIP_FAULT_COPY))  // as if the copy call had failed; nothing is enqueued
             return cuda_fail(cudaErrorInvalidValue, "layer copy (injected fault)");
+        if (packed(layer)) return queue_packed(layer, slot, cs, inl);
         cudaError_t e = cudaStreamWaitEvent(cs, slot_free[slot], 0);
         if (e != cudaSuccess) return cuda_fail(e, "copy wait");
         const char* src = static_cast<const char*>(host_layer[layer]);
@@ -741,19 +925,6 @@ struct loip_ctx {
         }
         cudaEvent_t e0 = take_event(), e1 = take_event();
         cudaEventRecord(e0, cs);
-        if (packed(layer)) {
-            uint64_t moved = 0;
-            int rc = enqueue_packed(layer, slot, cs, &moved);
-            if (rc) return rc;
-            cudaEventRecord(e1, cs);
-            copy_events.push_back({e0, e1, false, moved});
-            // the slot is full once every chunk is unpacked and the raw copies landed
-            e = cudaStreamWaitEvent(unpack_st, e1, 0);
-            if (e == cudaSuccess) e = cudaEventRecord(slot_full[slot], unpack_st);
-            if (e != cudaSuccess) return cuda_fail(e, "slot event");
-            st.h2d_weight_bytes += moved;
-            return LOIP_OK;
-        }
         // the blocks the layer streams, at their blob offsets
         const uint64_t off0 = (res_mask[layer] & 1) ? lay.mha_bytes : 0;
         const uint64_t off1 = (res_mask[layer] & 2) ? lay.mha_bytes : lay.l_size;
@@ -775,14 +946,15 @@ struct loip_ctx {
 
     int issue_next_copy() {  // ring order over offloaded layers, across steps
         const int m = (int)off_order.size();
-        int rc = enqueue_copy(off_order[copy_seq % m], (int)(copy_seq % cfg.n_slots), copy);
+        int rc = enqueue_copy(off_order[copy_seq % m], (int)(copy_seq % cfg.n_slots), copy, inline_unpack);
         if (rc) return rc;
         ++copy_seq;
         return LOIP_OK;
     }
 
-    int prime_slots() {
+    int prime_slots() {  // the streams are idle (callers synchronise first)
         copy_seq = compute_seq = 0;
+        if (packing) reset_pack_queue();
         if (off_order.empty() || cfg.mode == LOIP_MODE_NAIVE) return LOIP_OK;
         for (int k = 0; k < cfg.n_slots; ++k) {
             int rc = issue_next_copy();
@@ -1044,8 +1216,13 @@ struct loip_ctx {
                     if (off_order[compute_seq % off_order.size()] != l)
                         return fail(LOIP_ERR_STATE, "slot ring out of order");
                 }
-                cudaError_t e = cudaStreamWaitEvent(compute, slot_full[slot], 0);
-                if (e != cudaSuccess) return cuda_fail(e, "compute wait");
+                if (packed(l)) {
+                    int rc = wait_packed_slot(slot, compute);
+                    if (rc) return rc;
+                } else {
+                    cudaError_t e = cudaStreamWaitEvent(compute, slot_full[slot], 0);
+                    if (e != cudaSuccess) return cuda_fail(e, "compute wait");
+                }
                 chain = false;
             }
             int rc = fn(l, slot);
@@ -1403,6 +1580,8 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
     if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
     if (ctx->h_pt) cudaFreeHost(ctx->h_pt);
     for (auto e : ctx->slot_full) cudaEventDestroy(e);
+    for (auto e : ctx->raw_done)
+        if (e) cudaEventDestroy(e);
     for (auto e : ctx->slot_free) cudaEventDestroy(e);
     for (auto& pr : ctx->copy_events) {
         cudaEventDestroy(pr.a);
@@ -1413,9 +1592,12 @@ extern "C" void loip_destroy(loip_ctx* ctx) {
         cudaEventDestroy(k.b);
     }
     for (auto e : ctx->event_pool) cudaEventDestroy(e);
-    for (cudaEvent_t e : {ctx->ev_done, ctx->ev_step0, ctx->ev_step1, ctx->ev_reach, ctx->ev_stage,
-                          ctx->chunk_ready[0], ctx->chunk_ready[1], ctx->chunk_free[0], ctx->chunk_free[1]})
+    for (cudaEvent_t e : {ctx->ev_done, ctx->ev_step0, ctx->ev_step1, ctx->ev_reach, ctx->ev_stage})
         if (e) cudaEventDestroy(e);
+    for (int g = 0; g < kPackRingMax; ++g) {
+        if (ctx->chunk_ready[g]) cudaEventDestroy(ctx->chunk_ready[g]);
+        if (ctx->chunk_free[g]) cudaEventDestroy(ctx->chunk_free[g]);
+    }
     if (ctx->compute) cudaStreamDestroy(ctx->compute);
     if (ctx->copy) cudaStreamDestroy(ctx->copy);
     if (ctx->unpack_st) cudaStreamDestroy(ctx->unpack_st);
@@ -1593,10 +1775,17 @@ extern "C" int loip_create(const loip_model_desc* desc, const loip_config* cfg_i
         int lo = 0, hi = 0;
         e = cudaDeviceGetStreamPriorityRange(&lo, &hi);
         if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&c->unpack_st, cudaStreamNonBlocking, hi);
-        for (int g = 0; g < 2 && e == cudaSuccess; ++g) {
+        for (int g = 0; g < c->ring && e == cudaSuccess; ++g) {
             e = cudaEventCreateWithFlags(&c->chunk_ready[g], cudaEventDisableTiming);
             if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->chunk_free[g], cudaEventDisableTiming);
         }
+        c->slot_inline.assign(cfg.n_slots, 0);
+        c->raw_pumped.assign(cfg.n_slots, 1);
+        c->inl_left.assign(cfg.n_slots, 0);
+        c->inl_chunks.assign(cfg.n_slots, {});
+        c->raw_done.assign(cfg.n_slots, nullptr);
+        for (int k = 0; k < cfg.n_slots && e == cudaSuccess; ++k)
+            e = cudaEventCreateWithFlags(&c->raw_done[k], cudaEventDisableTiming);
     }
     c->slot_full.resize(cfg.n_slots);
     c->slot_free.resize(cfg.n_slots);
@@ -1807,7 +1996,8 @@ extern "C" int loip_stream_layer(loip_ctx* c, int32_t layer, int32_t slot, void*
         c->off_order.empty() || !c->host_layer[layer])
         return c->fail(LOIP_ERR_INVALID, "layer is not offloaded or slot out of range");
     cudaStream_t s = copy_stream ? reinterpret_cast<cudaStream_t>(copy_stream) : c->copy;
-    return c->enqueue_copy(layer, slot, s);
+    int rc = c->flush_inline();
+    return rc ? rc : c->enqueue_copy(layer, slot, s);
 }
 
 extern "C" int loip_set_batch(loip_ctx* c, int32_t batch, const int32_t* ctx_lens) {
@@ -1838,7 +2028,11 @@ extern "C" int loip_layer_forward(loip_ctx* c, int32_t layer, int32_t slot, floa
     float* x = c->fixed_ptr<float>(c->fx.x);
     cudaError_t e = cudaMemcpyAsync(x, hidden, (size_t)batch * c->H * 4, cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess) return c->cuda_fail(e, "hidden copy");
-    if (c->offloaded[layer]) {
+    if (c->offloaded[layer] && c->packed(layer)) {
+        rc = c->flush_inline();
+        if (rc == LOIP_OK) rc = c->wait_packed_slot(slot, s);
+        if (rc) return rc;
+    } else if (c->offloaded[layer]) {
         e = cudaStreamWaitEvent(s, c->slot_full[slot], 0);
         if (e != cudaSuccess) return c->cuda_fail(e, "slot wait");
     }
@@ -1879,6 +2073,8 @@ static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int3
     e = launch_embed(c->embed_table(), d_tokens, B, c->H, c->V, x, s, false);
     if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
     c->chain = true;
+    // streamed layers unpack inline, on the compute stream (see pump())
+    c->inline_unpack = c->packing && c->cfg.mode == LOIP_MODE_OVERLAP;
     if (c->cfg.mode == LOIP_MODE_DIRECT)
         rc = c->run_layers_direct(B, pos, s);
     else
@@ -1971,6 +2167,10 @@ extern "C" int loip_prefill(loip_ctx* c, const int32_t* tokens, const int32_t* p
         if (tokens[t] < 0 || tokens[t] >= c->V) return c->fail(LOIP_ERR_INVALID, "token id out of range");
     auto t0 = std::chrono::steady_clock::now();
     int rc = c->sync_all();
+    if (rc) return rc;
+    // the GEMMs hold every SM for ms at a time: streamed layers unpack on their own stream
+    c->inline_unpack = false;
+    rc = c->flush_inline();
     if (rc) return rc;
     for (int i = 0; i < n_prompts; ++i) {
         c->release_pages(i);

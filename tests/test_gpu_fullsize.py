@@ -6,8 +6,9 @@
   tolerances; greedy tokens equal, or at a near tie within what the hidden-state error
   allows.  Then a 66-token prompt through the tensor-core prefill and two decode steps
   on its cache, against the oracle, to the same tolerances.
-* 70B-shaped stack under the 60 GB device budget (the default benchmark's plan: 50 of
-  80 layers streamed through two slots, one layer keeping its MHA block): a prefill and
+* 70B-shaped stack under the 60 GB device budget (the default benchmark's plan and
+  streaming path: 49 of 80 layers streamed losslessly packed through two slots, two
+  of them keeping their MHA block; embedding table in host memory): a prefill and
   a decode step bit for bit equal to the same stack with every layer resident, then
   three tokens decoded from an empty cache and a 2-token prefill with a decode step on
   its cache, against the oracle.
@@ -123,11 +124,14 @@ def test_8b_resident_decode_matches_oracle(torch, L, orc):
 def test_70b_offloaded_is_lossless_and_decode_matches_oracle(torch, L, orc):
     m = configs.MODELS["llama3-70b"]
     seq = inputs.token_ids(configs.PROMPT_SEED, 3, m["vocab"])
-    # the default benchmark's context and prefill sizes (1024-token prompt, 12 + 3
-    # steps), so that the residency plan is the benchmarked one
-    kw = dict(n_slots=2, max_batch=1, max_ctx=1079, max_prefill_tokens=1024)
+    # the default benchmark's configuration: its context and prefill sizes
+    # (1024-token prompt, 12 + 3 steps), the embedding table in mapped host
+    # memory and the streamed layers packed, so that the residency plan (49
+    # streamed layers, two of them keeping their MHA block) and the streaming
+    # path are the benchmarked ones
+    kw = dict(n_slots=2, max_batch=1, max_ctx=1079, max_prefill_tokens=1024, embed_on_host=1, pack_stream=1)
     runs = []
-    for budget, n_off in ((60_000_000_000, 50), (200_000_000_000, 0)):
+    for budget, n_off in ((60_000_000_000, 49), (200_000_000_000, 0)):
         ctx = L.Context(m, L.config(budget=budget, **kw))
         assert ctx.plan()["n_offloaded"] == n_off
         ctx.load_weights_generated(configs.WEIGHT_SEED)

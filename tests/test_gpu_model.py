@@ -341,15 +341,16 @@ def test_block_level_residency_is_bitwise_lossless(torch, L, orc, extra, mode):
     _check_vs_oracle(orc, m, prompts, conts, np.array(toks), np.array(hids))
 
 
-@pytest.mark.parametrize("whole", [0, 1])
-def test_kv_growth_offloads_blocks_or_layers(torch, L, orc, whole):
+@pytest.mark.parametrize("whole,pack", [(0, 0), (1, 0), (0, 1)])
+def test_kv_growth_offloads_blocks_or_layers(torch, L, orc, whole, pack):
     """KV growth past the reserve: block granularity (Eq. 7) offloads one MHA
     block (the smallest resident block covering a page group); whole-layer mode
-    offloads a layer.  Results stay bit-identical either way."""
+    offloads a layer.  Results stay bit-identical either way, also when the
+    demoted weights then stream packed (the re-plan drops the queued copies)."""
     m = TINY6
     prompt = inputs.token_ids(41, 60, m["vocab"])
     cont = [[int(t)] for t in inputs.token_ids(42, 10, m["vocab"])]
-    kw = dict(max_batch=1, max_ctx=128, n_slots=2, whole_layers=whole)
+    kw = dict(max_batch=1, max_ctx=128, n_slots=2, whole_layers=whole, pack_stream=pack)
     base = _run(L, torch, m, [prompt], cont, dict(max_batch=1, max_ctx=128, n_slots=2), 6)
     lay = L.loip_layer_layout(m)
     cfg0 = L.config(budget=1 << 40, **kw)

@@ -207,3 +207,50 @@ def test_packed_streaming_with_raw_superblocks_and_an_unpackable_layer(torch, L,
     pk = _run(L, torch, dict(kw, pack_stream=1), 2, blobs=blobs)
     assert np.array_equal(raw[0], pk[0])
     assert np.array_equal(raw[1].view(np.uint32), pk[1].view(np.uint32))
+
+
+LLAMA8B = configs.MODELS["llama3-8b"]
+
+
+def _passes(L, torch, m, cfg, prompts_a, conts_a, prompts_b, conts_b):
+    """prefill -> decode steps -> prefill of new prompts -> decode steps; tokens
+    and final hidden rows of every call."""
+    ctx = L.Context(m, cfg)
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    hid = torch.empty(len(prompts_a), m["hidden"], dtype=torch.float32, device="cuda")
+    toks, hids = [], []
+    for prompts, conts in ((prompts_a, conts_a), (prompts_b, conts_b)):
+        toks.append(ctx.prefill(prompts, out_hidden=hid))
+        hids.append(hid.cpu().numpy().copy())
+        for step in conts:
+            toks.append(ctx.decode_step(step, out_hidden=hid))
+            hids.append(hid.cpu().numpy().copy())
+    plan, st = ctx.plan(), ctx.stats()
+    ctx.close()
+    torch.cuda.empty_cache()
+    return np.array(toks), np.array(hids), plan, st
+
+
+@pytest.mark.parametrize("max_prefill", [512, 1024, 2048])
+def test_packed_streaming_8b_layers_many_chunks(torch, L, max_prefill):
+    """8B-shaped layers (each streamed layer is 8 staging chunks: 2 of its MHA
+    block, 6 of its MLP block) with staging rings of 2, 4 and 8 chunks: decode
+    steps unpack on the compute stream, prefill passes on the unpack stream, and
+    the two alternate (decode -> prefill -> decode hands pending unpacks over).
+    Embedding table in mapped host memory, as in the offloaded benchmarks.
+    Bit-identical to the same calls with every layer resident."""
+    m = LLAMA8B
+    V = m["vocab"]
+    pa = [inputs.token_ids(701, 70, V), inputs.token_ids(702, 33, V)]
+    pb = [inputs.token_ids(703, 41, V), inputs.token_ids(704, 90, V)]
+    ca = [[int(a), int(b)] for a, b in zip(inputs.token_ids(705, 3, V), inputs.token_ids(706, 3, V))]
+    cb = [[int(a), int(b)] for a, b in zip(inputs.token_ids(707, 2, V), inputs.token_ids(708, 2, V))]
+    kw = dict(max_batch=2, max_ctx=160, n_slots=2, max_prefill_tokens=max_prefill)
+    ref = _passes(L, torch, m, L.config(budget=40_000_000_000, **kw), pa, ca, pb, cb)
+    assert ref[2]["n_offloaded"] == 0
+    kp = dict(kw, pack_stream=1, embed_on_host=1)
+    got = _passes(L, torch, m, L.config(budget=_budget(L, m, kp, 12), **kp), pa, ca, pb, cb)
+    assert 16 <= got[2]["n_offloaded"] <= 20, got[2]
+    assert got[3]["unpack_launches"] > 0
+    assert np.array_equal(ref[0], got[0])
+    assert np.array_equal(ref[1].view(np.uint32), got[1].view(np.uint32))
