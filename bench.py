@@ -185,7 +185,10 @@ def run_ours(args, rank, world):
     kv_reserve = 0
     if "ctx_lo" in w:  # KV reserved for the prompts only: decoding grows it (online re-planning)
         kv_reserve = sum((n + 63) // 64 for n in lens) * kv_group_bytes(m)
-    max_prefill = sum(lens) if prefill_mode else min(4096, sum(lens))
+    # decode workloads prefill their prompts as untimed set-up; at batch 1 in
+    # passes of at most 512 rows, so that the prefill workspace (and the staging
+    # ring sized by it) leaves the device bytes to weights
+    max_prefill = sum(lens) if prefill_mode else min(4096 if Bsz > 1 else 512, sum(lens))
     # a device budget that cannot hold every layer keeps the embedding table in
     # pinned host memory (one 2 x hidden byte row per token crosses the link) and
     # gives its device bytes to resident layers

@@ -23,9 +23,10 @@
 // Shared memory (bf16, K-major, 128-byte swizzle: 16-byte chunk c of row r at
 // r * 128 + ((c ^ (r & 7)) * 16), 8-row atoms of 1024 bytes):
 //   Q_hi, Q_lo   [128 rows][D]        D/64 slabs of 16 KB each
-//   K            [64 keys][D]         D/64 slabs of 8 KB
+//   K            [64 keys][D]         D/64 slabs of 8 KB, two buffers (the next
+//                                     page loads while this one is used)
 //   V^T          [D rows][64 keys]    one slab of D * 128 bytes (transposed by
-//                                     the threads while loading)
+//                                     the threads, 8 x 8 blocks in registers)
 //   P_hi, P_lo   [128 rows][64 keys]  one slab of 16 KB each
 // Tensor memory: S [128 x 64] fp32 at column 0, O_blk [128 x D] at column 128.
 //
@@ -59,8 +60,9 @@ struct AttnTcSmem {
     static constexpr int K_SLAB = 64 * 128;
     static constexpr int QHI = 0;
     static constexpr int QLO = QHI + SLABS * Q_SLAB;
-    static constexpr int KB = QLO + SLABS * Q_SLAB;
-    static constexpr int VT = KB + SLABS * K_SLAB;
+    static constexpr int KB = QLO + SLABS * Q_SLAB;  // two K buffers: page kb and page kb + 1
+    static constexpr int KBUF = SLABS * K_SLAB;
+    static constexpr int VT = KB + 2 * KBUF;
     static constexpr int PHI = VT + D * 128;
     static constexpr int PLO = PHI + Q_SLAB;
     static constexpr int RED = PLO + Q_SLAB;  // float [2][128] row maxima of the two column halves
@@ -223,50 +225,86 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
     const int nkb = last_pos / kKeys + 1;
     const char* kv_layer = p.kv.base + (uint64_t)p.kv.layer * p.kv.layer_page_bytes;
 
-    for (int kb = 0; kb < nkb && ok; ++kb) {
-        // ---- K page -> K-major slabs (cp.async); V page -> V^T slab (threads).
-        // Positions past the tile's last one hold no key yet (the page may keep
-        // anything there): they are zero-filled, so that their zero weights in P
-        // meet finite values (0 x NaN would spoil the row).
-        const char* page = kv_layer + p.kv.page_offsets[(int64_t)req * p.kv.max_pages + kb];
-        const char* kp = page + (size_t)g * kKeys * D * 2;
-        const char* vp = page + (size_t)(p.Hkv + g) * kKeys * D * 2;
+    // Positions past the tile's last one hold no key yet (the page may keep
+    // anything there): their K and V are zero-filled, so that their zero
+    // weights in P meet finite values (0 x NaN would spoil the row).
+    auto page_at = [&](int kb) { return kv_layer + p.kv.page_offsets[(int64_t)req * p.kv.max_pages + kb]; };
+    // K page kb -> K buffer b, K-major slabs (cp.async)
+    auto load_k = [&](int kb, int b) {
+        const char* kp = page_at(kb) + (size_t)g * kKeys * D * 2;
         const int n_keys = last_pos - kb * kKeys + 1;  // valid keys in this page (>= 1)
         for (int i = tid; i < kKeys * (D / 8); i += kAttnThreads) {
             const int key = i / (D / 8), c = i - key * (D / 8);  // 16-byte chunk c of the key's row
-            cp_async16(sbase + S::KB + (uint32_t)((c >> 3) * S::K_SLAB) + swz(key, c & 7),
+            cp_async16(sbase + S::KB + (uint32_t)(b * S::KBUF + (c >> 3) * S::K_SLAB) + swz(key, c & 7),
                        kp + (size_t)key * D * 2 + c * 16, key < n_keys ? 16u : 0u);
         }
         asm volatile("cp.async.commit_group;" ::: "memory");
-        for (int i = tid; i < kKeys * (D / 8); i += kAttnThreads) {
-            const int key = i % kKeys, c = i / kKeys;  // keys fastest: a warp reads 32 rows' chunk c
-            const uint4 w = key < n_keys ? *reinterpret_cast<const uint4*>(vp + (size_t)key * D * 2 + c * 16)
-                                         : make_uint4(0u, 0u, 0u, 0u);
-            const uint16_t* e = reinterpret_cast<const uint16_t*>(&w);
+    };
+    // V page kb -> registers.  The page is cut into 8 x 8 blocks (keys 8 kc ..,
+    // dims 8 c ..); thread 2 blk + h holds dims 4h .. 4h+3 of block blk's 8 keys.
+    constexpr int kVThreads = 2 * 8 * (D / 8);
+    uint2 vin[8];
+    auto load_v = [&](int kb) {
+        if (tid >= kVThreads) return;
+        const int blk = tid >> 1, h = tid & 1, kc = blk & 7, c = blk >> 3;
+        const char* vp = page_at(kb) + (size_t)(p.Hkv + g) * kKeys * D * 2 + c * 16 + h * 8;
+        const int n_keys = last_pos - kb * kKeys + 1;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const int dd = c * 8 + j;  // V^T row
-                *reinterpret_cast<uint16_t*>(sm + S::VT + swz(dd, key >> 3) + (key & 7) * 2) = e[j];
-            }
+        for (int i = 0; i < 8; ++i) {
+            const int key = 8 * kc + i;
+            vin[i] = key < n_keys ? *reinterpret_cast<const uint2*>(vp + (size_t)key * D * 2) : make_uint2(0u, 0u);
         }
-        asm volatile("cp.async.wait_all;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic-proxy writes -> the tensor core
-        __syncthreads();
+    };
+    // registers -> V^T slab: row dd = 8 c + j holds the 8 keys of block blk as
+    // one 16-byte chunk (kc)
+    auto store_vt = [&]() {
+        if (tid >= kVThreads) return;
+        const int blk = tid >> 1, h = tid & 1, kc = blk & 7, c = blk >> 3;
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+            const uint32_t sel = (jj & 1) ? 0x7632u : 0x5410u;  // high or low halves of the two words
+            uint32_t w[4];
+#pragma unroll
+            for (int k2 = 0; k2 < 4; ++k2) {
+                const uint32_t a = (jj >> 1) ? vin[2 * k2].y : vin[2 * k2].x;
+                const uint32_t b = (jj >> 1) ? vin[2 * k2 + 1].y : vin[2 * k2 + 1].x;
+                w[k2] = __byte_perm(a, b, sel);  // keys 2 k2, 2 k2 + 1 of dim 4h + jj
+            }
+            *reinterpret_cast<uint4*>(sm + S::VT + swz(8 * c + 4 * h + jj, kc)) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    };
+    load_k(0, 0);
+    load_v(0);
+    store_vt();
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic-proxy writes -> the tensor core
+    __syncthreads();
+
+    for (int kb = 0; kb < nkb && ok; ++kb) {
+        const int kbuf = kb & 1;
         // ---- S = (Q_hi + Q_lo) K^T
         if (tid == 0) {
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
             for (int k = 0; k < D / 16; ++k) {
-                const uint32_t qo = (uint32_t)((k >> 2) * S::Q_SLAB), ko = (uint32_t)((k >> 2) * S::K_SLAB);
+                const uint32_t qo = (uint32_t)((k >> 2) * S::Q_SLAB);
+                const uint32_t ko = (uint32_t)(kbuf * S::KBUF + (k >> 2) * S::K_SLAB);
                 const uint64_t bd = sdesc(sbase + S::KB + ko) + 2 * (k & 3);
                 umma(tmem, sdesc(sbase + S::QHI + qo) + 2 * (k & 3), bd, idesc(kKeys), k != 0);
                 umma(tmem, sdesc(sbase + S::QLO + qo) + 2 * (k & 3), bd, idesc(kKeys), 1u);
             }
             umma_commit(mbar);
-            if (!mbar_wait(mbar, phase)) {
-                atomicCAS(&g_attn_tc_error, 0, 1);
-                ok = false;
-            }
+        }
+        // the next page's K (into the other buffer, free since S of the last
+        // page completed) and V (into registers) load under this page's work
+        const bool more = kb + 1 < nkb;
+        if (more) {
+            load_k(kb + 1, kbuf ^ 1);
+            load_v(kb + 1);
+        }
+        if (tid == 0 && !mbar_wait(mbar, phase)) {
+            atomicCAS(&g_attn_tc_error, 0, 1);
+            ok = false;
         }
         phase ^= 1;
         ok = __syncthreads_and(ok);
@@ -346,9 +384,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
 #pragma unroll
             for (int j = 0; j < 16; ++j) o[j0 + j] = fmaf(o[j0 + j], alpha, v[j]);
         }
+        // ---- the next page's V^T (the slab is free: this page's P V completed)
+        if (more) {
+            store_vt();
+            asm volatile("cp.async.wait_all;" ::: "memory");
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        __syncthreads();  // S, P and the K/V slabs are reused by the next page
+        __syncthreads();  // S, P, K and V^T are reused by the next page
     }
+    // a wait that gave up can leave the next page's copies in flight
+    asm volatile("cp.async.wait_all;" ::: "memory");
     if (ok) {
         // l of the row = both halves' sums
         red[hh * 128 + r] = l_run;

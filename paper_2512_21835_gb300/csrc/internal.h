@@ -157,6 +157,9 @@ constexpr int kPackMaxExc = 7;
 cudaError_t launch_pack(const uint16_t* in, uint64_t n_sb, uint8_t* out, uint32_t* raw_list, uint32_t first_sb,
                         uint32_t raw_cap, cudaStream_t st);
 cudaError_t launch_unpack(const uint8_t* in, uint64_t n_sb, uint16_t* out, cudaStream_t st);
+// two segments in one launch (either may be empty)
+cudaError_t launch_unpack2(const uint8_t* in0, uint64_t n0, uint16_t* out0, const uint8_t* in1, uint64_t n1,
+                           uint16_t* out1, cudaStream_t st);
 
 // First failure code recorded by a tensor-core GEMM launch (0 = none).
 cudaError_t tc_error(int* code);

@@ -129,10 +129,23 @@ __device__ __forceinline__ void unpack_patch(uint4 (&o)[4], int lane, uint32_t x
     }
 }
 
-__global__ void __launch_bounds__(256) unpack_kernel(const uint8_t* __restrict__ in, uint64_t n_sb,
-                                                     uint16_t* __restrict__ out) {
-    const uint64_t sb = (uint64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
-    if (sb >= n_sb) return;
+// One launch unpacks one or two segments (runs of superblocks, each with its
+// own input and output): blocks [0, s0.blocks) take the first, the rest the
+// second.  Two chunks per launch halve the launches, whose start-up after an
+// idle wait for the host link costs about as much as the unpack itself.
+struct UnpackSeg {
+    const uint8_t* in;
+    uint16_t* out;
+    uint64_t n_sb;
+    uint32_t blocks;
+};
+
+__global__ void __launch_bounds__(256) unpack_kernel(UnpackSeg s0, UnpackSeg s1) {
+    const bool second = blockIdx.x >= s0.blocks;
+    const uint8_t* __restrict__ in = second ? s1.in : s0.in;
+    uint16_t* __restrict__ out = second ? s1.out : s0.out;
+    const uint64_t sb = (uint64_t)(blockIdx.x - (second ? s0.blocks : 0u)) * kWarps + (threadIdx.x >> 5);
+    if (sb >= (second ? s1.n_sb : s0.n_sb)) return;
     const int lane = threadIdx.x & 31;
     const uint8_t* src = in + sb * kPackedSb;
     // every load first: read once, evict first
@@ -173,9 +186,17 @@ cudaError_t launch_pack(const uint16_t* in, uint64_t n_sb, uint8_t* out, uint32_
 }
 
 cudaError_t launch_unpack(const uint8_t* in, uint64_t n_sb, uint16_t* out, cudaStream_t st) {
-    if (n_sb == 0) return cudaSuccess;
-    if (((uintptr_t)in & 15) || ((uintptr_t)out & 15)) return cudaErrorInvalidValue;
-    unpack_kernel<<<(unsigned)((n_sb + kWarps - 1) / kWarps), 256, 0, st>>>(in, n_sb, out);
+    return launch_unpack2(in, n_sb, out, nullptr, 0, nullptr, st);
+}
+
+cudaError_t launch_unpack2(const uint8_t* in0, uint64_t n0, uint16_t* out0, const uint8_t* in1, uint64_t n1,
+                           uint16_t* out1, cudaStream_t st) {
+    if (n0 + n1 == 0) return cudaSuccess;
+    if (((uintptr_t)in0 & 15) || ((uintptr_t)out0 & 15) || ((uintptr_t)in1 & 15) || ((uintptr_t)out1 & 15))
+        return cudaErrorInvalidValue;
+    const UnpackSeg s0{in0, out0, n0, (uint32_t)((n0 + kWarps - 1) / kWarps)};
+    const UnpackSeg s1{in1, out1, n1, (uint32_t)((n1 + kWarps - 1) / kWarps)};
+    unpack_kernel<<<s0.blocks + s1.blocks, 256, 0, st>>>(s0, s1);
     return cudaGetLastError();
 }
 

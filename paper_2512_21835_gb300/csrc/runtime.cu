@@ -140,15 +140,19 @@ constexpr uint32_t kPackRawCap = 256;     // superblocks per layer that may trav
 bool packing_enabled(const loip_config* c) {
     return c->pack_stream && c->mode != LOIP_MODE_DIRECT && c->host_budget_bytes == 0;
 }
-// Chunks in the device staging ring.  A chunk is unpacked by a kernel on its
-// own stream, which only gets SMs when a compute kernel ends: during a prefill
-// pass the tensor-core GEMMs hold every SM for up to a few ms (the gate/up GEMM
-// of 2048 rows at the 70B shape: ~2.3 ms, ten chunks' worth of link time), so
-// the ring grows with the prefill rows to keep the copy engine busy: two chunks
-// up to 512 rows, one more per 256 rows above, at most kPackRingMax.
+// Chunks in the device staging ring.  In decode the compute stream unpacks
+// two landed chunks per launch while the copy engine fills two more, and a
+// layer's compute (up to ~0.9 ms for a streamed layer and its resident
+// neighbour at the 70B shape, about four chunks' worth of link time) must not
+// stall the copies: six chunks.  In a
+// prefill pass a chunk is unpacked by a kernel on its own stream, which only
+// gets SMs when a compute kernel ends, and the tensor-core GEMMs hold every SM
+// for up to a few ms (the gate/up GEMM of 2048 rows at the 70B shape: ~2.1 ms,
+// nine chunks' worth of link time): one chunk per 256 prefill rows, at most
+// kPackRingMax.
 constexpr int kPackRingMax = 8;
 int pack_ring_chunks(const loip_config* c) {
-    return std::max(2, std::min(kPackRingMax, c->max_prefill_tokens / 256));
+    return std::max(6, std::min(kPackRingMax, c->max_prefill_tokens / 256));
 }
 // superblocks per staging chunk: kPackChunkSb, or the larger block of a small layer
 uint64_t pack_chunk_sb(const loip_model_desc* d) {
@@ -377,6 +381,7 @@ struct loip_ctx {
             pu[u].off = offs[u];
             pu[u].n_sb = sizes[u] / (2 * kPackWords);
             pu[u].tail = sizes[u] - pu[u].n_sb * 2 * kPackWords;
+            at = (at + 4095) / 4096 * 4096;  // each unit's packed data on a 4 KB boundary
             pu[u].host_off = at;
             at += pu[u].n_sb * kPackedSb + pu[u].tail;
         }
@@ -452,9 +457,12 @@ struct loip_ctx {
             if (res_mask[l] & (1 << u)) continue;  // this block is resident
             bytes += pu[u].n_sb * kPackedSb + pu[u].tail;
             for (const auto& r : pk[l].raw) bytes += r.first == u ? 2 * kPackWords : 0;
-            // equal chunks of at most chunk_sb superblocks (no short last chunk)
+            // chunks of about equal size, at most chunk_sb superblocks (no short
+            // last chunk), a multiple of 128 superblocks so that each copy starts
+            // on a 4 KB boundary of the host area (the copy engine read
+            // 32-byte-aligned chunks ~4% slower)
             const uint64_t nc = (pu[u].n_sb + chunk_sb - 1) / chunk_sb;
-            const uint64_t per = nc ? (pu[u].n_sb + nc - 1) / nc : 1;
+            const uint64_t per = nc ? std::min(chunk_sb, ((pu[u].n_sb + nc - 1) / nc + 127) / 128 * 128) : 1;
             for (uint64_t c0 = 0; c0 < pu[u].n_sb; c0 += per) {
                 pack_fifo.push_back({l, slot, u, c0, std::min<uint64_t>(per, pu[u].n_sb - c0), inl, first, cs});
                 first = false;
@@ -475,17 +483,29 @@ struct loip_ctx {
             ++ring_done;
         }
     }
-    // Unpack of one staged chunk into its slot, on stream s.
-    cudaError_t enqueue_unpack(uint64_t seq, int slot, int unit, uint64_t c0, uint64_t n, cudaStream_t s) {
-        const int g = (int)(seq % (uint64_t)ring);
-        const uint8_t* st_c = fixed_ptr<uint8_t>(fx.pack_stage) + (uint64_t)g * chunk_sb * kPackedSb;
-        uint16_t* out = reinterpret_cast<uint16_t*>(slot_ptr(slot) + pu[unit].off) + c0 * kPackWords;
-        cudaError_t e = cudaStreamWaitEvent(s, chunk_ready[g], 0);
-        if (e == cudaSuccess) e = timed(13, s, [&] { return launch_unpack(st_c, n, out, s); });
-        if (e == cudaSuccess) e = cudaEventRecord(chunk_free[g], s);
-        mark_unpacked(seq);
+    // Unpack of one staged chunk (or two: b != nullptr, one launch) into the
+    // slot, on stream s, after their copies landed.
+    cudaError_t enqueue_unpack(int slot, const InlineChunk& a, const InlineChunk* b, cudaStream_t s) {
+        const InlineChunk* c[2] = {&a, b};
+        const uint8_t* in[2] = {nullptr, nullptr};
+        uint16_t* out[2] = {nullptr, nullptr};
+        uint64_t n[2] = {0, 0};
+        cudaError_t e = cudaSuccess;
+        for (int i = 0; i < 2 && c[i] && e == cudaSuccess; ++i) {
+            const int g = (int)(c[i]->seq % (uint64_t)ring);
+            in[i] = fixed_ptr<uint8_t>(fx.pack_stage) + (uint64_t)g * chunk_sb * kPackedSb;
+            out[i] = reinterpret_cast<uint16_t*>(slot_ptr(slot) + pu[c[i]->unit].off) + c[i]->c0 * kPackWords;
+            n[i] = c[i]->n;
+            e = cudaStreamWaitEvent(s, chunk_ready[g], 0);
+        }
+        if (e == cudaSuccess)
+            e = timed(13, s, [&] { return launch_unpack2(in[0], n[0], out[0], in[1], n[1], out[1], s); });
+        for (int i = 0; i < 2 && c[i]; ++i) {
+            if (e == cudaSuccess) e = cudaEventRecord(chunk_free[c[i]->seq % (uint64_t)ring], s);
+            mark_unpacked(c[i]->seq);
+        }
         st.unpack_launches += 1;
-        st.unpack_bytes += n * (uint64_t)(kPackedSb + 2 * kPackWords);
+        st.unpack_bytes += (n[0] + n[1]) * (uint64_t)(kPackedSb + 2 * kPackWords);
         return e;
     }
     // Enqueues queued pieces in order while the staging ring has room.
@@ -517,10 +537,11 @@ struct loip_ctx {
                 if (e == cudaSuccess) e = cudaEventRecord(chunk_ready[g], j.cs);
                 pump_bytes += j.n * kPackedSb;
                 if (e == cudaSuccess) {
+                    const InlineChunk c{seq, j.unit, j.c0, j.n};
                     if (j.inl)
-                        inl_chunks[j.slot].push_back({seq, j.unit, j.c0, j.n});
+                        inl_chunks[j.slot].push_back(c);
                     else
-                        e = enqueue_unpack(seq, j.slot, j.unit, j.c0, j.n, unpack_st);
+                        e = enqueue_unpack(j.slot, c, nullptr, unpack_st);
                 }
             } else {  // end job: raw tails and raw superblocks into the slot once it is free
                 const char* raw_area = host + pu[1].host_off + pu[1].n_sb * kPackedSb + pu[1].tail;
@@ -561,23 +582,33 @@ struct loip_ctx {
         return LOIP_OK;
     }
     // Before a packed layer in `slot` computes on stream s: its inline unpacks
-    // (each after its chunk landed) and the wait for its raw pieces, or the wait
-    // for slot_full.
+    // (after their chunks landed; two chunks per launch when the ring leaves the
+    // copy engine four more meanwhile) and the wait for its raw pieces, or the
+    // wait for slot_full.
     int wait_packed_slot(int slot, cudaStream_t s) {
         cudaError_t e = cudaSuccess;
+        const size_t per_launch = ring >= 6 ? 2 : 1;
         while (inl_left[slot] > 0) {
-            if (inl_chunks[slot].empty()) {
+            const size_t want = std::min<size_t>(per_launch, (size_t)inl_left[slot]);
+            while (inl_chunks[slot].size() < want) {
+                const size_t have = inl_chunks[slot].size();
                 int rc = pump();
                 if (rc) return rc;
-                if (inl_chunks[slot].empty()) return fail(LOIP_ERR_STATE, "packed copy queue out of order");
+                if (inl_chunks[slot].size() == have) return fail(LOIP_ERR_STATE, "packed copy queue out of order");
             }
             const InlineChunk c = inl_chunks[slot].front();
             inl_chunks[slot].pop_front();
-            --inl_left[slot];
-            e = enqueue_unpack(c.seq, slot, c.unit, c.c0, c.n, s);
+            InlineChunk c2{};
+            const bool two = want == 2;
+            if (two) {
+                c2 = inl_chunks[slot].front();
+                inl_chunks[slot].pop_front();
+            }
+            inl_left[slot] -= two ? 2 : 1;
+            e = enqueue_unpack(slot, c, two ? &c2 : nullptr, s);
             if (e != cudaSuccess) return cuda_fail(e, "unpack kernel");
             chain = false;
-            int rc = pump();  // the freed entry lets the next chunk's copy go
+            int rc = pump();  // the freed entries let the next chunks' copies go
             if (rc) return rc;
         }
         while (!raw_pumped[slot]) {
@@ -602,7 +633,7 @@ struct loip_ctx {
             while (e == cudaSuccess && !inl_chunks[s].empty()) {
                 const InlineChunk c = inl_chunks[s].front();
                 inl_chunks[s].pop_front();
-                e = enqueue_unpack(c.seq, s, c.unit, c.c0, c.n, unpack_st);
+                e = enqueue_unpack(s, c, nullptr, unpack_st);
             }
             if (e == cudaSuccess && raw_pumped[s]) {  // end job already enqueued: slot_full after it
                 e = cudaStreamWaitEvent(unpack_st, raw_done[s], 0);

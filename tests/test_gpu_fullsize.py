@@ -125,11 +125,11 @@ def test_70b_offloaded_is_lossless_and_decode_matches_oracle(torch, L, orc):
     m = configs.MODELS["llama3-70b"]
     seq = inputs.token_ids(configs.PROMPT_SEED, 3, m["vocab"])
     # the default benchmark's configuration: its context and prefill sizes
-    # (1024-token prompt, 12 + 3 steps), the embedding table in mapped host
-    # memory and the streamed layers packed, so that the residency plan (49
-    # streamed layers, two of them keeping their MHA block) and the streaming
-    # path are the benchmarked ones
-    kw = dict(n_slots=2, max_batch=1, max_ctx=1079, max_prefill_tokens=1024, embed_on_host=1, pack_stream=1)
+    # (1024-token prompt prefilled in passes of 512 rows, 12 + 3 steps), the
+    # embedding table in mapped host memory and the streamed layers packed, so
+    # that the residency plan (49 streamed layers, two of them keeping their MHA
+    # block) and the streaming path are the benchmarked ones
+    kw = dict(n_slots=2, max_batch=1, max_ctx=1079, max_prefill_tokens=512, embed_on_host=1, pack_stream=1)
     runs = []
     for budget, n_off in ((60_000_000_000, 49), (200_000_000_000, 0)):
         ctx = L.Context(m, L.config(budget=budget, **kw))

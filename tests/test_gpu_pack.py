@@ -231,12 +231,13 @@ def _passes(L, torch, m, cfg, prompts_a, conts_a, prompts_b, conts_b):
     return np.array(toks), np.array(hids), plan, st
 
 
-@pytest.mark.parametrize("max_prefill", [512, 1024, 2048])
+@pytest.mark.parametrize("max_prefill", [512, 2048])
 def test_packed_streaming_8b_layers_many_chunks(torch, L, max_prefill):
     """8B-shaped layers (each streamed layer is 8 staging chunks: 2 of its MHA
-    block, 6 of its MLP block) with staging rings of 2, 4 and 8 chunks: decode
-    steps unpack on the compute stream, prefill passes on the unpack stream, and
-    the two alternate (decode -> prefill -> decode hands pending unpacks over).
+    block, 6 of its MLP block) with staging rings of 6 and 8 chunks: decode
+    steps unpack on the compute stream, two chunks per launch, prefill passes
+    on the unpack stream, and the two alternate (decode -> prefill -> decode
+    hands pending unpacks over).
     Embedding table in mapped host memory, as in the offloaded benchmarks.
     Bit-identical to the same calls with every layer resident."""
     m = LLAMA8B
