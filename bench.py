@@ -65,8 +65,8 @@ def gate_up_traffic(model, batch):
 # DRAM bytes (read + write) of the unpack kernel per algorithmic byte (packed
 # chunk read + words written), from an ncu capture of the kernel microbenchmark
 # (one 70B layer's worth of words); valid while pack.cu has this hash.
-UNPACK_TRAFFIC_RATIO = 0.98104  # 2,964,243,968 B over 3,021,529,600 algorithmic (writes still in L2 at exit)
-UNPACK_TRAFFIC_SRC = "59744d91fc9014212e37fb8037237312cf69d5807563fd24e7e4c209eebad4fb"
+UNPACK_TRAFFIC_RATIO = 0.98088  # 2,963,747,584 B over 3,021,529,600 algorithmic (writes still in L2 at exit)
+UNPACK_TRAFFIC_SRC = "fe8993707ec6e43a29784b48cbf80378dcf189aa5693129747548bc7730e9b93"
 
 
 def unpack_traffic(bytes_per_launch):
