@@ -2104,8 +2104,12 @@ static int decode_step_enqueue(loip_ctx* c, const int32_t* d_tokens, int B, int3
     e = launch_embed(c->embed_table(), d_tokens, B, c->H, c->V, x, s, false);
     if (e != cudaSuccess) return c->cuda_fail(e, "embed kernel");
     c->chain = true;
-    // streamed layers unpack inline, on the compute stream (see pump())
-    c->inline_unpack = c->packing && c->cfg.mode == LOIP_MODE_OVERLAP;
+    // At batch 1 streamed layers unpack inline, on the compute stream (see
+    // pump()).  Batched steps compute for much longer per layer (70B, batch 8:
+    // 108 ms of kernels per step against 34 ms at batch 1), and inline unpacks
+    // would hold the copies back behind them (the link fell to 166 GB/s): their
+    // chunks unpack on the unpack stream, between the compute kernels.
+    c->inline_unpack = c->packing && c->cfg.mode == LOIP_MODE_OVERLAP && B == 1;
     if (c->cfg.mode == LOIP_MODE_DIRECT)
         rc = c->run_layers_direct(B, pos, s);
     else

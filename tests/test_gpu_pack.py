@@ -231,22 +231,22 @@ def _passes(L, torch, m, cfg, prompts_a, conts_a, prompts_b, conts_b):
     return np.array(toks), np.array(hids), plan, st
 
 
-@pytest.mark.parametrize("max_prefill", [512, 2048])
-def test_packed_streaming_8b_layers_many_chunks(torch, L, max_prefill):
+@pytest.mark.parametrize("max_prefill,batch", [(512, 1), (512, 2), (2048, 1)])
+def test_packed_streaming_8b_layers_many_chunks(torch, L, max_prefill, batch):
     """8B-shaped layers (each streamed layer is 8 staging chunks: 2 of its MHA
-    block, 6 of its MLP block) with staging rings of 6 and 8 chunks: decode
-    steps unpack on the compute stream, two chunks per launch, prefill passes
-    on the unpack stream, and the two alternate (decode -> prefill -> decode
-    hands pending unpacks over).
+    block, 6 of its MLP block) with staging rings of 6 and 8 chunks: batch-1
+    decode steps unpack on the compute stream, two chunks per launch; batch-2
+    decode steps and prefill passes unpack on the unpack stream; and the passes
+    alternate (decode -> prefill -> decode hands pending unpacks over).
     Embedding table in mapped host memory, as in the offloaded benchmarks.
     Bit-identical to the same calls with every layer resident."""
     m = LLAMA8B
     V = m["vocab"]
-    pa = [inputs.token_ids(701, 70, V), inputs.token_ids(702, 33, V)]
-    pb = [inputs.token_ids(703, 41, V), inputs.token_ids(704, 90, V)]
-    ca = [[int(a), int(b)] for a, b in zip(inputs.token_ids(705, 3, V), inputs.token_ids(706, 3, V))]
-    cb = [[int(a), int(b)] for a, b in zip(inputs.token_ids(707, 2, V), inputs.token_ids(708, 2, V))]
-    kw = dict(max_batch=2, max_ctx=160, n_slots=2, max_prefill_tokens=max_prefill)
+    pa = [inputs.token_ids(701, 70, V), inputs.token_ids(702, 33, V)][:batch]
+    pb = [inputs.token_ids(703, 41, V), inputs.token_ids(704, 90, V)][:batch]
+    ca = [[int(a), int(b)][:batch] for a, b in zip(inputs.token_ids(705, 3, V), inputs.token_ids(706, 3, V))]
+    cb = [[int(a), int(b)][:batch] for a, b in zip(inputs.token_ids(707, 2, V), inputs.token_ids(708, 2, V))]
+    kw = dict(max_batch=batch, max_ctx=160, n_slots=2, max_prefill_tokens=max_prefill)
     ref = _passes(L, torch, m, L.config(budget=40_000_000_000, **kw), pa, ca, pb, cb)
     assert ref[2]["n_offloaded"] == 0
     kp = dict(kw, pack_stream=1, embed_on_host=1)
