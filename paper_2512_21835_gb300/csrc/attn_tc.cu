@@ -25,8 +25,9 @@
 //   Q_hi, Q_lo   [128 rows][D]        D/64 slabs of 16 KB each
 //   K            [64 keys][D]         D/64 slabs of 8 KB, two buffers (the next
 //                                     page loads while this one is used)
-//   V^T          [D rows][64 keys]    one slab of D * 128 bytes (transposed by
-//                                     the threads, 8 x 8 blocks in registers)
+//   V^T          [D rows][64 keys]    slabs of D * 128 bytes, two buffers
+//                                     (transposed by the threads, 8 x 8 blocks
+//                                     in registers)
 //   P_hi, P_lo   [128 rows][64 keys]  one slab of 16 KB each
 // Tensor memory: S [128 x 64] fp32 at column 0, O_blk [128 x D] at column 128.
 //
@@ -62,8 +63,9 @@ struct AttnTcSmem {
     static constexpr int QLO = QHI + SLABS * Q_SLAB;
     static constexpr int KB = QLO + SLABS * Q_SLAB;  // two K buffers: page kb and page kb + 1
     static constexpr int KBUF = SLABS * K_SLAB;
-    static constexpr int VT = KB + 2 * KBUF;
-    static constexpr int PHI = VT + D * 128;
+    static constexpr int VT = KB + 2 * KBUF;  // two V^T slabs: page kb and page kb + 1
+    static constexpr int VTBUF = D * 128;
+    static constexpr int PHI = VT + 2 * VTBUF;
     static constexpr int PLO = PHI + Q_SLAB;
     static constexpr int RED = PLO + Q_SLAB;  // float [2][128] row maxima of the two column halves
     static constexpr int BAR = RED + 2 * 128 * 4;
@@ -155,8 +157,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     float* red = reinterpret_cast<float*>(sm + S::RED);
     uint64_t* bar = reinterpret_cast<uint64_t*>(sm + S::BAR);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + S::BAR + 8);
-    const uint32_t sbase = smem_u32(sm), mbar = smem_u32(bar);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + S::BAR + 24);
+    // completion of: S = Q K^T; O_blk = P V; everything issued (error path)
+    const uint32_t sbase = smem_u32(sm), mbar_s = smem_u32(bar), mbar_pv = smem_u32(bar + 1),
+                   mbar_end = smem_u32(bar + 2);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int4 tile = p.tiles[blockIdx.x];
     const int g = blockIdx.y;  // kv head
@@ -164,7 +168,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
     const int qd = p.Hq * D;
 
     if (tid == 0) {
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar) : "memory");
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar_s) : "memory");
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar_pv) : "memory");
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar_end) : "memory");
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 0) {
@@ -219,7 +225,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
 #pragma unroll
     for (int j = 0; j < DH; ++j) o[j] = 0.f;
     float m_run = -INFINITY, l_run = 0.f;
-    uint32_t phase = 0;
+    uint32_t phase_s = 0, phase_pv = 0;
     bool ok = true;
     const int last_pos = pos0 + nrows - 1;
     const int nkb = last_pos / kKeys + 1;
@@ -257,7 +263,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
     };
     // registers -> V^T slab: row dd = 8 c + j holds the 8 keys of block blk as
     // one 16-byte chunk (kc)
-    auto store_vt = [&]() {
+    auto store_vt = [&](int b) {
         if (tid >= kVThreads) return;
         const int blk = tid >> 1, h = tid & 1, kc = blk & 7, c = blk >> 3;
 #pragma unroll
@@ -270,43 +276,45 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
                 const uint32_t b = (jj >> 1) ? vin[2 * k2 + 1].y : vin[2 * k2 + 1].x;
                 w[k2] = __byte_perm(a, b, sel);  // keys 2 k2, 2 k2 + 1 of dim 4h + jj
             }
-            *reinterpret_cast<uint4*>(sm + S::VT + swz(8 * c + 4 * h + jj, kc)) = make_uint4(w[0], w[1], w[2], w[3]);
+            *reinterpret_cast<uint4*>(sm + S::VT + b * S::VTBUF + swz(8 * c + 4 * h + jj, kc)) =
+                make_uint4(w[0], w[1], w[2], w[3]);
         }
     };
+    // S = (Q_hi + Q_lo) K^T of page kb (K buffer kb & 1), completion on mbar_s
+    auto issue_s = [&](int kb) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k) {
+            const uint32_t qo = (uint32_t)((k >> 2) * S::Q_SLAB);
+            const uint32_t ko = (uint32_t)((kb & 1) * S::KBUF + (k >> 2) * S::K_SLAB);
+            const uint64_t bd = sdesc(sbase + S::KB + ko) + 2 * (k & 3);
+            umma(tmem, sdesc(sbase + S::QHI + qo) + 2 * (k & 3), bd, idesc(kKeys), k != 0);
+            umma(tmem, sdesc(sbase + S::QLO + qo) + 2 * (k & 3), bd, idesc(kKeys), 1u);
+        }
+        umma_commit(mbar_s);
+    };
+    // Pipeline: while the CUDA cores run page kb's softmax and O update, the
+    // tensor core runs S of page kb + 1 (issued right behind P V of page kb),
+    // and the loads of page kb + 2 are in flight.
     load_k(0, 0);
     load_v(0);
-    store_vt();
+    store_vt(0);
     asm volatile("cp.async.wait_all;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // generic-proxy writes -> the tensor core
     __syncthreads();
+    if (tid == 0) issue_s(0);
+    if (nkb > 1) {
+        load_k(1, 1);
+        load_v(1);
+    }
 
     for (int kb = 0; kb < nkb && ok; ++kb) {
-        const int kbuf = kb & 1;
-        // ---- S = (Q_hi + Q_lo) K^T
-        if (tid == 0) {
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k) {
-                const uint32_t qo = (uint32_t)((k >> 2) * S::Q_SLAB);
-                const uint32_t ko = (uint32_t)(kbuf * S::KBUF + (k >> 2) * S::K_SLAB);
-                const uint64_t bd = sdesc(sbase + S::KB + ko) + 2 * (k & 3);
-                umma(tmem, sdesc(sbase + S::QHI + qo) + 2 * (k & 3), bd, idesc(kKeys), k != 0);
-                umma(tmem, sdesc(sbase + S::QLO + qo) + 2 * (k & 3), bd, idesc(kKeys), 1u);
-            }
-            umma_commit(mbar);
-        }
-        // the next page's K (into the other buffer, free since S of the last
-        // page completed) and V (into registers) load under this page's work
         const bool more = kb + 1 < nkb;
-        if (more) {
-            load_k(kb + 1, kbuf ^ 1);
-            load_v(kb + 1);
-        }
-        if (tid == 0 && !mbar_wait(mbar, phase)) {
+        if (tid == 0 && !mbar_wait(mbar_s, phase_s)) {
             atomicCAS(&g_attn_tc_error, 0, 1);
             ok = false;
         }
-        phase ^= 1;
+        phase_s ^= 1;
         ok = __syncthreads_and(ok);
         if (!ok) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -355,28 +363,43 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
             *reinterpret_cast<uint4*>(sm + S::PLO + off) =
                 make_uint4(plo[4 * c], plo[4 * c + 1], plo[4 * c + 2], plo[4 * c + 3]);
         }
+        // ---- the next page's V^T (its slab was last read by P V of page kb - 1,
+        // complete) and K (landed)
+        if (more) {
+            store_vt((kb + 1) & 1);
+            asm volatile("cp.async.wait_all;" ::: "memory");
+        }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncthreads();
-        // ---- O_blk = (P_hi + P_lo) V
+        // ---- O_blk = (P_hi + P_lo) V, then S of the next page behind it
         if (tid == 0) {
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t vt = sbase + S::VT + (uint32_t)((kb & 1) * S::VTBUF);
 #pragma unroll
             for (int k = 0; k < kKeys / 16; ++k) {
-                const uint64_t bd = sdesc(sbase + S::VT) + 2 * k;
+                const uint64_t bd = sdesc(vt) + 2 * k;
                 umma(tmem + kOCol, sdesc(sbase + S::PHI) + 2 * k, bd, idesc(D), k != 0);
                 umma(tmem + kOCol, sdesc(sbase + S::PLO) + 2 * k, bd, idesc(D), 1u);
             }
-            umma_commit(mbar);
-            if (!mbar_wait(mbar, phase)) {
-                atomicCAS(&g_attn_tc_error, 0, 2);
-                ok = false;
-            }
+            umma_commit(mbar_pv);
+            if (more) issue_s(kb + 1);
         }
-        phase ^= 1;
+        // ---- page kb + 2 into the K buffer S of page kb used (complete) and registers
+        if (kb + 2 < nkb) {
+            load_k(kb + 2, kb & 1);
+            load_v(kb + 2);
+        }
+        if (tid == 0 && !mbar_wait(mbar_pv, phase_pv)) {
+            atomicCAS(&g_attn_tc_error, 0, 2);
+            ok = false;
+        }
+        phase_pv ^= 1;
         ok = __syncthreads_and(ok);
         if (!ok) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        // ---- O = O * alpha + O_blk (my D/2 columns), in fp32 registers
+        // ---- O = O * alpha + O_blk (my D/2 columns), in fp32 registers.  The next
+        // P V writes O_blk only after the barriers of the next page's softmax.
 #pragma unroll
         for (int j0 = 0; j0 < DH; j0 += 16) {
             float v[16];
@@ -384,14 +407,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
 #pragma unroll
             for (int j = 0; j < 16; ++j) o[j0 + j] = fmaf(o[j0 + j], alpha, v[j]);
         }
-        // ---- the next page's V^T (the slab is free: this page's P V completed)
-        if (more) {
-            store_vt();
-            asm volatile("cp.async.wait_all;" ::: "memory");
-        }
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        __syncthreads();  // S, P, K and V^T are reused by the next page
     }
     // a wait that gave up can leave the next page's copies in flight
     asm volatile("cp.async.wait_all;" ::: "memory");
@@ -420,8 +436,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const AttnTcPa
     } else if (tid == 0) {
         // a commit of everything issued so far, so no MMA is in flight when the
         // tensor memory is released (bounded like every other wait)
-        umma_commit(mbar);
-        mbar_wait(mbar, phase);
+        umma_commit(mbar_end);
+        mbar_wait(mbar_end, 0);
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
