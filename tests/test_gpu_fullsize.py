@@ -150,3 +150,56 @@ def test_70b_offloaded_is_lossless_and_decode_matches_oracle(torch, L, orc):
     pre_tok, pre_hid = runs[0][0]
     exempt += sum(_check_row(orc, m, pre_tok[i], pre_hid[i], ref, 1 + i) for i in range(len(pre_tok)))
     assert exempt <= 1
+
+
+def _prefill_rows(ctx, torch, m, prompts):
+    hid = torch.empty(len(prompts), m["hidden"], dtype=torch.float32, device="cuda")
+    toks = ctx.prefill(prompts, out_hidden=hid)
+    return np.array(toks), hid.cpu().numpy().copy()
+
+
+def test_8b_prefill_4x512_matches_token_by_token_decode(torch, L):
+    """The prefill benchmark's launch shape (4 prompts x 512 tokens in one
+    2048-row pass: several query tiles per prompt, every page boundary) on the
+    8B stack, against decoding each prompt one token at a time (the decode path,
+    checked against the oracle at full depth above): final hidden rows within
+    the benchmark spec's tolerances, greedy tokens equal.  (The fp64 oracle itself
+    cannot run 2048 tokens through the stack in a test's time.)"""
+    m = configs.MODELS["llama3-8b"]
+    prompts = [np.asarray(p) for p in inputs.prompts(configs.PROMPT_SEED, 4, 512, m["vocab"])]
+    ctx = L.Context(m, L.config(budget=40_000_000_000, n_slots=2, max_batch=4, max_ctx=520,
+                                max_prefill_tokens=2048))
+    assert ctx.plan()["n_offloaded"] == 0
+    ctx.load_weights_generated(configs.WEIGHT_SEED)
+    pre_tok, pre_hid = _prefill_rows(ctx, torch, m, prompts)
+    for i, p in enumerate(prompts):
+        toks, hids = _decode_from_empty(ctx, torch, m, p)
+        ea, er = _errors(pre_hid[i].astype(np.float64), hids[-1].astype(np.float64))
+        print(f"prompt {i}: max-abs {ea:.3e} rel-L2 {er:.3e}")
+        assert ea <= HID_ABS and er <= HID_REL, (i, ea, er)
+        assert int(pre_tok[i]) == int(toks[-1]), i
+    ctx.close()
+    torch.cuda.empty_cache()
+
+
+def test_70b_prefill_4x512_offloaded_is_lossless(torch, L):
+    """The prefill benchmark's exact configuration (60 GB budget, 50 layers
+    streamed losslessly packed through an 8-chunk staging ring, 4 x 512 tokens
+    in one pass, embedding table in host memory) gives the same tokens and final
+    hidden rows, bit for bit, as the same pass with every layer resident."""
+    m = configs.MODELS["llama3-70b"]
+    prompts = [np.asarray(p) for p in inputs.prompts(configs.PROMPT_SEED, 4, 512, m["vocab"])]
+    kw = dict(n_slots=2, max_batch=4, max_ctx=512, max_prefill_tokens=2048, embed_on_host=1, pack_stream=1)
+    runs = []
+    for budget, n_off in ((60_000_000_000, 50), (200_000_000_000, 0)):
+        ctx = L.Context(m, L.config(budget=budget, **kw))
+        assert ctx.plan()["n_offloaded"] == n_off
+        ctx.load_weights_generated(configs.WEIGHT_SEED)
+        runs.append(_prefill_rows(ctx, torch, m, prompts))
+        runs.append(_prefill_rows(ctx, torch, m, prompts))  # a second pass on the same context
+        ctx.close()
+        torch.cuda.empty_cache()
+    for tok, hid in runs[1:]:
+        assert np.array_equal(tok, runs[0][0])
+        assert np.array_equal(hid.view(np.uint32), runs[0][1].view(np.uint32))
+    assert np.all(np.isfinite(runs[0][1]))
