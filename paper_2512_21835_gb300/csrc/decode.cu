@@ -1190,12 +1190,19 @@ __global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int chunk = blockIdx.x, kvh = blockIdx.y, row = blockIdx.z;
     pdl_trigger();
-    pdl_wait();
+    // Lengths, positions, the page table and every cached key and value but the
+    // newest position's were written before this step's first (non-overlapped)
+    // launch: their loads go out before the wait for the kernel that wrote the
+    // newest position's key and value (and the queries).
     const int ctx = p.ctx_lens ? p.ctx_lens[row] : p.positions[row] + 1;
     const int npages = (ctx + P - 1) / P;
-    if (chunk >= npages) return;
+    if (chunk >= npages) {
+        pdl_wait();
+        return;
+    }
     const int req = p.row_req ? p.row_req[row] : row;
     const int nvalid = min(P, ctx - chunk * P);
+    const int newest = ctx - 1 - chunk * P;  // row of the newest position in this page (< 0 or >= P: none)
     {
         const char* page = p.kv.base + p.kv.page_offsets[(int64_t)req * p.kv.max_pages + chunk] +
                            (uint64_t)p.kv.layer * p.kv.layer_page_bytes;
@@ -1203,9 +1210,16 @@ __global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
         const uint16_t* Vh = reinterpret_cast<const uint16_t*>(page) + ((size_t)p.Hkv + kvh) * P * D;
         for (int i = tid; i < nvalid * CH; i += NT) {
             const int t = i / CH, c = i - t * CH;
+            if (t == newest) continue;
             cp_async16(&sm.sK[(t * CH + ((c + t) & (CH - 1))) * 8], Kh + (size_t)t * D + c * 8);
             cp_async16(&sm.sV[(t * CH + c) * 8], Vh + (size_t)t * D + c * 8);
         }
+        pdl_wait();
+        if (newest >= 0 && newest < P)
+            for (int c = tid; c < CH; c += NT) {
+                cp_async16(&sm.sK[(newest * CH + ((c + newest) & (CH - 1))) * 8], Kh + (size_t)newest * D + c * 8);
+                cp_async16(&sm.sV[(newest * CH + c) * 8], Vh + (size_t)newest * D + c * 8);
+            }
         const float* qs = p.q + (size_t)row * p.Hq * D + (size_t)kvh * G * D;
         for (int i = tid; i < G * D / 4; i += NT)
             reinterpret_cast<float4*>(&sm.sq[0][0])[i] = ld_act4<false>(qs + 4 * i);
