@@ -65,8 +65,8 @@ def gate_up_traffic(model, batch):
 # DRAM bytes (read + write) of the unpack kernel per algorithmic byte (packed
 # chunk read + words written), from an ncu capture of the kernel microbenchmark
 # (one 70B layer's worth of words); valid while pack.cu has this hash.
-UNPACK_TRAFFIC_RATIO = 0.98088  # 2,963,747,584 B over 3,021,529,600 algorithmic (writes still in L2 at exit)
-UNPACK_TRAFFIC_SRC = "fe8993707ec6e43a29784b48cbf80378dcf189aa5693129747548bc7730e9b93"
+UNPACK_TRAFFIC_RATIO = 0.98091  # 2,858,929,152 B over 2,914,572,800 algorithmic (writes still in L2 at exit)
+UNPACK_TRAFFIC_SRC = "8064b4d9eb77121cd3bf37bcaa7a385968f4df26fe5cbd463d23af30b9506087"
 
 
 def unpack_traffic(bytes_per_launch):

@@ -510,18 +510,28 @@ int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t M, int32_t 
 /* Lossless packing of bf16 weights for the host link (the streamed layers'
  * transport under loip_config.pack_stream): n_sb superblocks of 1024 words
  * (in: bf16 [n_sb * 1024], dev, 16-byte aligned) become n_sb packed
- * superblocks of LOIP_PACKED_SB bytes (out, dev, 16-byte aligned): the
- * sign-and-mantissa byte of every word, a 4-bit code of its exponent relative
- * to the superblock's largest exponent (15 binades; code 0 = an exception), and
- * a 32-byte record (byte 0: that largest exponent; byte 1: the number of
- * exceptions, <= 7; then the exceptions as uint32 index | exponent << 16).  A
- * superblock with more than 7 exceptions is not packed: its record says 0xff,
- * and its index (first_sb + i) is appended to raw_list (dev uint32
- * [1 + raw_cap]: raw_list[0] counts every such superblock, the first raw_cap
- * indices follow, in no particular order; raw_list may be NULL).
- * loip_k_unpack restores every packed superblock bit for bit and leaves the
- * words of the others untouched.  Lossless: no weight changes (Sec. IV-A). */
-#define LOIP_PACKED_SB 1568
+ * superblocks of LOIP_PACKED_SB bytes (out, dev, 16-byte aligned):
+ *   bytes 0..1023     the sign-and-mantissa byte of every word;
+ *   bytes 1024..1279  2 bits per word: with k = (the superblock's largest
+ *                     exponent) - (the word's exponent), codes 0..2 name the
+ *                     three most frequent k of the superblock, 3 escapes;
+ *   bytes 1280..1367  2 bits per level-1 escape, in word order: codes 0..2 name
+ *                     the next three most frequent k, 3 escapes (at most 352);
+ *   bytes 1368..1407  4 bits per level-2 escape, in word order: k itself (0..14)
+ *                     or 15, an exception (at most 80);
+ *   bytes 1408..1439  a record of 8 uint32: [0] largest exponent | flag << 8 |
+ *                     rank[0] << 16 | rank[1] << 24, [1] rank[2..5], [2] the
+ *                     escape counts n1 | n2 << 16 | the exception count << 24,
+ *                     [3..7] up to 5 exceptions as index | exponent << 16.
+ * rank[] lists the six most frequent k in 0..14, most frequent first, ties to
+ * the smaller k.  A superblock over one of the limits is not packed: its flag
+ * is 0xff, every other byte of it 0, and its index (first_sb + i) is appended
+ * to raw_list (dev uint32 [1 + raw_cap]: raw_list[0] counts every such
+ * superblock, the first raw_cap indices follow, in no particular order;
+ * raw_list may be NULL).  loip_k_unpack restores every packed superblock bit
+ * for bit and leaves the words of the others untouched.  Lossless: no weight
+ * changes (Sec. IV-A). */
+#define LOIP_PACKED_SB 1440
 int loip_k_pack(const uint16_t* in, uint64_t n_sb, uint8_t* out, uint32_t* raw_list, uint32_t first_sb,
                 uint32_t raw_cap, void* stream);
 int loip_k_unpack(const uint8_t* in, uint64_t n_sb, uint16_t* out, void* stream);

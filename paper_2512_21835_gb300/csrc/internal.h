@@ -144,14 +144,17 @@ cudaError_t launch_tc_gemm_resid(const uint16_t* a, bool split, const uint16_t* 
 cudaError_t launch_tc_gemm_swiglu(const uint16_t* y, bool split, const uint16_t* wg, const uint16_t* wu, int M, int H,
                                   int F, uint16_t* a, cudaStream_t st);
 // Lossless packing of bf16 weights for the host link (pack.cu): superblocks of
-// kPackWords words become kPackedSb bytes (sign-and-mantissa bytes, 4-bit
-// exponent codes relative to the superblock's largest exponent, a record with
-// up to kPackMaxExc exceptions).  A superblock with more exceptions is marked
-// unpacked (record byte 1 = 0xff): unpack leaves its words untouched and they
-// travel raw.  in / out 16-byte aligned.
+// kPackWords words become kPackedSb bytes (sign-and-mantissa bytes, exponents
+// as codes of one, two or three levels relative to the superblock's largest
+// exponent, a record with up to kPackMaxExc exceptions).  A superblock over
+// one of the limits (kPackEsc1 level-1 escapes, kPackEsc2 level-2 escapes,
+// kPackMaxExc exceptions) is marked unpacked (record byte 1 = 0xff): unpack
+// leaves its words untouched and they travel raw.  in / out 16-byte aligned.
 constexpr int kPackWords = 1024;
-constexpr int kPackedSb = 1568;
-constexpr int kPackMaxExc = 7;
+constexpr int kPackedSb = 1440;
+constexpr int kPackEsc1 = 352;
+constexpr int kPackEsc2 = 80;
+constexpr int kPackMaxExc = 5;
 // raw_list (may be null): [0] counts the superblocks left unpacked, then their
 // indices (first_sb + i), at most raw_cap of them.
 cudaError_t launch_pack(const uint16_t* in, uint64_t n_sb, uint8_t* out, uint32_t* raw_list, uint32_t first_sb,

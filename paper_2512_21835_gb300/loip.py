@@ -275,6 +275,7 @@ class Context:
         if getattr(self, "h", None):
             lib().loip_destroy(self.h)
             self.h = None
+        self.arena = None  # the device arena goes back to the allocator now, not at collection
 
     def __del__(self):
         try:
@@ -483,11 +484,11 @@ def loip_k_gemm_split(A2, W, x, stream=None):
     _check(lib().loip_k_gemm_split(_ptr(A2), _ptr(W), M, W.shape[0], K, _ptr(x), _s(stream)))
 
 
-PACKED_SB = 1568
+PACKED_SB = 1440
 
 
 def loip_k_pack(words, packed, raw_list=None, first_sb=0, raw_cap=0, stream=None):
-    """Pack words (int16 [n_sb * 1024]) into packed (uint8 [n_sb * 1568])."""
+    """Pack words (int16 [n_sb * 1024]) into packed (uint8 [n_sb * 1440])."""
     n_sb = words.numel() // 1024
     _check(lib().loip_k_pack(_ptr(words), n_sb, _ptr(packed), _ptr(raw_list), first_sb, raw_cap, _s(stream)))
 
