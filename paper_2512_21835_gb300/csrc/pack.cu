@@ -274,63 +274,53 @@ __global__ void __launch_bounds__(256) unpack_kernel(UnpackSeg s0, UnpackSeg s1)
         off2[3] = t0 + t1 + t2 + (xb >> 16);
     }
     // k of four words at once: the level-1 codes select bytes of the first three
-    // ranks (code 3 selects a 0, replaced below for the escapes)
-    const uint32_t R1 = (uint32_t)(ranks & 0xffffffu), R2 = (uint32_t)((ranks >> 24) & 0xffffffu);
+    // ranks; code 3 selects 0xff, which marks the escapes (no k is above 14)
+    const uint32_t R1 = (uint32_t)(ranks & 0xffffffu) | 0xff000000u;
+    const uint32_t R2 = (uint32_t)((ranks >> 24) & 0xffffffu) | 0xff000000u;  // ranks 3..5, 0xff: level 3
     const uint32_t E4 = emax * 0x01010101u;
-    // 2-bit fields at bits 2j -> 4-bit fields at bits 4j (j < 8); 4-bit fields at
-    // bits 4j -> bytes (j < 4)
+    // 2-bit fields at bits 2j -> 4-bit fields at bits 4j (j < 8)
     auto spread2 = [](uint32_t v) -> uint32_t {
         v = (v | (v << 8)) & 0x00ff00ffu;
         v = (v | (v << 4)) & 0x0f0f0f0fu;
         return (v | (v << 2)) & 0x33333333u;
     };
-    auto spread4 = [](uint32_t v) -> uint32_t {
-        v = (v | (v << 8)) & 0x00ff00ffu;
-        return (v | (v << 4)) & 0x0f0f0f0fu;
-    };
-    auto bytes2nib = [](uint32_t x) -> uint32_t {  // bytes (each < 16) -> nibbles
-        x = (x | (x >> 4)) & 0x00ff00ffu;
-        return (x | (x >> 8)) & 0xffffu;
-    };
     uint4 o[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-        const uint32_t c = c16[q];
-        const uint32_t sel = spread2(c);  // nibble e = level-1 code of word e
+        const uint32_t sel = spread2(c16[q]);  // nibble e = level-1 code of word e
         uint32_t k03 = __byte_perm(R1, 0u, sel), k47 = __byte_perm(R1, 0u, sel >> 16);
-        // level 2 without a loop: escape word e takes the level-2 code at its rank
-        // among the lane's escapes of the quarter (exclusive prefix count, nibble
-        // by nibble); the lane's codes, spread to bytes, are looked up by rank
-        const uint32_t escN = spread2(c & (c >> 1) & 0x5555u);  // nibble e = 1: word e escapes
-        const uint32_t rk = escN * 0x11111111u - escN;          // nibble e = escapes before word e
-        const uint32_t t4 = spread2(l2[q]);                     // nibble j = j-th level-2 code
-        const uint32_t B0 = spread4(t4 & 0xffffu), B1 = spread4(t4 >> 16);
-        const uint32_t d03 = __byte_perm(B0, B1, rk & 0x7777u), d47 = __byte_perm(B0, B1, (rk >> 16) & 0x7777u);
-        const uint32_t dn = bytes2nib(d03) | (bytes2nib(d47) << 16);  // nibble e = level-2 code of word e
-        const uint32_t M03 = spread4(escN & 0xffffu) * 0xffu, M47 = spread4(escN >> 16) * 0xffu;
-        // R2: ranks 3..5, byte 3 = 0 (level-3 words, set below)
-        k03 = (k03 & ~M03) | (__byte_perm(R2, 0u, dn) & M03);
-        k47 = (k47 & ~M47) | (__byte_perm(R2, 0u, dn >> 16) & M47);
-        // level 3 (rare): escape words with code 3, in word order; this lane's
+        // level 2 without a loop: T holds, for the lane's j-th escape of the
+        // quarter, the k its level-2 code names (0xff: level 3); escape word e
+        // takes entry rank(e), the number of escapes before it (a nibble-wise
+        // prefix product)
+        const uint32_t escN = sel & (sel >> 1) & 0x11111111u;  // nibble e = 1: word e escapes
+        const uint32_t rk = escN * 0x11111111u - escN;
+        const uint32_t t4 = spread2(l2[q]);  // nibble j = the j-th level-2 code
+        const uint32_t T0 = __byte_perm(R2, 0u, t4), T1 = __byte_perm(R2, 0u, t4 >> 16);
+        const uint32_t M03 = ((k03 & 0x80808080u) >> 7) * 0xffu, M47 = ((k47 & 0x80808080u) >> 7) * 0xffu;
+        k03 = (k03 & ~M03) | (__byte_perm(T0, T1, rk & 0x7777u) & M03);
+        k47 = (k47 & ~M47) | (__byte_perm(T0, T1, (rk >> 16) & 0x7777u) & M47);
+        // level 3 (rare): the words still marked 0xff, in word order; this lane's
         // nibbles of the quarter (at most 8: a 2-word window of words 22..31,
         // shuffled by the whole warp)
         const uint32_t wi = 22 + (off2[q] >> 3), sh = 4 * (off2[q] & 7);
         const uint32_t lo = __shfl_sync(0xffffffffu, lv, (int)wi & 31);
         const uint32_t hi = __shfl_sync(0xffffffffu, lv, (int)(wi + 1) & 31);
-        uint32_t m3 = dn & (dn >> 1) & escN;  // bit 4e: word e goes to level 3
-        if (m3) {
+        uint32_t m03 = k03 & 0x80808080u, m47 = k47 & 0x80808080u;
+        if (m03 | m47) {
             uint32_t l3 = wi < 32 ? __funnelshift_r(lo, wi + 1 < 32 ? hi : 0u, sh) : 0u;
-            do {
-                const int e = (__ffs(m3) - 1) >> 2;
-                m3 &= m3 - 1;
-                const uint32_t k = l3 & 15u;  // 15: an exception, patched below
+            while (m03) {
+                const uint32_t shb = (uint32_t)(__ffs(m03) - 8);  // 8 * byte
+                m03 &= m03 - 1;
+                k03 = (k03 & ~(0xffu << shb)) | ((l3 & 15u) << shb);  // 15: an exception, patched below
                 l3 >>= 4;
-                const uint32_t shb = 8 * (e & 3), keep = ~(0xffu << shb);
-                if (e < 4)
-                    k03 = (k03 & keep) | (k << shb);
-                else
-                    k47 = (k47 & keep) | (k << shb);
-            } while (m3);
+            }
+            while (m47) {
+                const uint32_t shb = (uint32_t)(__ffs(m47) - 8);
+                m47 &= m47 - 1;
+                k47 = (k47 & ~(0xffu << shb)) | ((l3 & 15u) << shb);
+                l3 >>= 4;
+            }
         }
         // exponent bytes: emax - k never borrows (k <= emax; the exception
         // placeholder 15 only where emax >= 15)
