@@ -1167,7 +1167,8 @@ cudaError_t launch_attn_t(AttnParams& p, cudaStream_t st, bool pdl) {
 // The page's unnormalised state (o, m, l) goes to scratch; the last block of
 // the (row, kv head) to arrive (completion ticket) combines every page's state
 // with the usual softmax merge: weights exp(m_c - max m) / sum, outputs summed in
-// page order, sixteen pages' loads in flight per thread.
+// page order, sixteen pages' loads in flight per thread (the first sixteen issued
+// together with the loads of the page maxima and sums).
 template <int G, int D>
 struct AttnPageSmem {
     alignas(16) uint16_t sK[64 * D];
@@ -1350,6 +1351,17 @@ __global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
     __syncthreads();
     if (!sm.last) return;
     __threadfence();
+    constexpr int NOUT = (G * D + NT - 1) / NT, PB = 16;
+    // the first PB pages' partial outputs do not depend on the weights: their
+    // loads go out together with those of the page maxima and sums
+    float v[PB][NOUT];
+#pragma unroll
+    for (int u = 0; u < PB; ++u)
+#pragma unroll
+        for (int k = 0; k < NOUT; ++k) {
+            const int e = tid + NT * k, g = e / D, j = e - g * D;
+            v[u][k] = (e < G * D && u < npages) ? __ldcg(base + g * hstride + (size_t)u * (D + 2) + j) : 0.f;
+        }
     // the stages are dead: page weights and denominators reuse them
     float(*s_w)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sm.sK[0]);
     float(*s_l)[kMaxChunks] = reinterpret_cast<float(*)[kMaxChunks]>(&sm.sV[0]);
@@ -1376,20 +1388,20 @@ __global__ void __launch_bounds__(256) attn_page_kernel(AttnParams p) {
         for (int c = lane; c < npages; c += 32) s_w[g][c] *= inv;
     }
     __syncthreads();
-    constexpr int NOUT = (G * D + NT - 1) / NT, PB = 16;
     float o[NOUT];
 #pragma unroll
     for (int k = 0; k < NOUT; ++k) o[k] = 0.f;
     for (int c0 = 0; c0 < npages; c0 += PB) {
-        float v[PB][NOUT];
+        if (c0 > 0)
 #pragma unroll
-        for (int u = 0; u < PB; ++u)
+            for (int u = 0; u < PB; ++u)
 #pragma unroll
-            for (int k = 0; k < NOUT; ++k) {
-                const int e = tid + NT * k, g = e / D, j = e - g * D;
-                v[u][k] = (e < G * D && c0 + u < npages) ? __ldcg(base + g * hstride + (size_t)(c0 + u) * (D + 2) + j)
-                                                          : 0.f;
-            }
+                for (int k = 0; k < NOUT; ++k) {
+                    const int e = tid + NT * k, g = e / D, j = e - g * D;
+                    v[u][k] = (e < G * D && c0 + u < npages)
+                                  ? __ldcg(base + g * hstride + (size_t)(c0 + u) * (D + 2) + j)
+                                  : 0.f;
+                }
 #pragma unroll
         for (int u = 0; u < PB; ++u)
 #pragma unroll
