@@ -93,9 +93,9 @@ typedef struct loip_config {
     const char* ssd_dir;          /* directory of the SSD tier's scratch file (caller-owned string,
                                    * read at create; NULL = /tmp) */
     int32_t pack_stream;          /* 1: streamed layers cross the host link losslessly packed
-                                   * (sign-and-mantissa bytes + 4-bit exponent codes per 1024-word
-                                   * superblock, ~77% of the bytes; unpacked into the slot on the
-                                   * device, bit for bit) -- see loip_k_pack.  Ignored in
+                                   * (sign-and-mantissa bytes + exponents coded in three levels
+                                   * per 1024-word superblock, 1440 of 2048 bytes; unpacked into
+                                   * the slot on the device, bit for bit) -- see loip_k_pack.  Ignored in
                                    * LOIP_MODE_DIRECT and with the SSD tier (host_budget_bytes > 0).
                                    * 0: raw blobs (default) */
     int32_t embed_on_host;        /* 1: the embedding table [vocab, hidden] stays in pinned host
@@ -524,8 +524,9 @@ int loip_k_gemm_split(const uint16_t* A2, const uint16_t* W, int32_t M, int32_t 
  *                     escape counts n1 | n2 << 16 | the exception count << 24,
  *                     [3..7] up to 5 exceptions as index | exponent << 16.
  * rank[] lists the six most frequent k in 0..14, most frequent first, ties to
- * the smaller k.  A superblock over one of the limits is not packed: its flag
- * is 0xff, every other byte of it 0, and its index (first_sb + i) is appended
+ * the smaller k.  A superblock over one of the limits is not packed: its
+ * record's first word is its largest exponent | 0xff << 8, every other byte of
+ * the superblock is 0, and its index (first_sb + i) is appended
  * to raw_list (dev uint32 [1 + raw_cap]: raw_list[0] counts every such
  * superblock, the first raw_cap indices follow, in no particular order;
  * raw_list may be NULL).  loip_k_unpack restores every packed superblock bit
