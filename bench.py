@@ -49,7 +49,7 @@ UNPACK_CLASS = 13  # kernel-timing class of the unpack of packed streamed chunks
 # kernel source they were taken on: when the decode kernels' source no longer
 # has this hash the figure is reported as null.
 GATE_UP_TRAFFIC = {"llama3-70b": 939_745_536, "llama3-8b": 235_113_984}
-GATE_UP_TRAFFIC_SRC = "5410ace14409a1585f865d64508e1e65cf509593325730d0e4619b6ae3b2e72e"
+GATE_UP_TRAFFIC_SRC = "a9c8cc3dcd122fa3d70d3d4bfa641301f6e3cb4caa4123b2fbe05cc51713aadc"
 
 
 def gate_up_traffic(model, batch):

@@ -135,7 +135,7 @@ loip_config normalized(const loip_config* c) {
 
 // Packed streaming (loip_config.pack_stream): not with direct access (kernels
 // read the host blobs in place) nor with the SSD tier (its blobs stay raw).
-constexpr uint64_t kPackChunkSb = 32768;  // superblocks per staging chunk (51 MB packed)
+constexpr uint64_t kPackChunkSb = 32768;  // superblocks per staging chunk (47 MB packed)
 constexpr uint32_t kPackRawCap = 256;     // superblocks per layer that may travel unpacked
 bool packing_enabled(const loip_config* c) {
     return c->pack_stream && c->mode != LOIP_MODE_DIRECT && c->host_budget_bytes == 0;

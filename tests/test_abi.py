@@ -104,6 +104,30 @@ def test_fixed_bytes(L):
     assert 2 * 128256 * 8192 * 2 < fb < 2 * 128256 * 8192 * 2 + 400 * 2 ** 20
 
 
+@pytest.mark.parametrize("model", ["tiny", "llama3-70b"])
+@pytest.mark.parametrize("mp, ring", [(256, 6), (512, 6), (1536, 6), (1792, 7), (2048, 8), (4096, 8)])
+def test_fixed_part_embedding_placement_and_staging_ring(L, model, mp, ring):
+    """The memory term the plan starts from: keeping the embedding table in host
+    memory takes exactly its V x H x 2 bytes out of the device's fixed part; the
+    packed stream adds a staging ring of R = max(6, min(8, prefill rows / 256))
+    chunks of min(32768, superblocks of the larger block) packed superblocks of
+    1440 bytes, plus the raw-superblock list (257 uint32), each part rounded up
+    to 256 bytes; with direct access or an SSD tier nothing is packed."""
+    m = configs.MODELS[model]
+    al = lambda b: (b + 255) // 256 * 256
+    base = dict(budget=60 * 10 ** 9, max_batch=1, max_ctx=1088, max_prefill_tokens=mp)
+    f0 = loip.loip_fixed_bytes(m, loip.config(**base))
+    assert f0 - loip.loip_fixed_bytes(m, loip.config(**base, embed_on_host=1)) == al(m["vocab"] * m["hidden"] * 2)
+    lay = loip.loip_layer_layout(m)
+    chunk = max(1, min(32768, max(lay["mha_bytes"], lay["mlp_bytes"]) // 2048))
+    fp = loip.loip_fixed_bytes(m, loip.config(**base, pack_stream=1))
+    assert fp - f0 == al(ring * chunk * 1440) + al(4 * 257)
+    assert loip.loip_fixed_bytes(m, loip.config(**base, pack_stream=1, mode=loip.MODE_DIRECT)) == f0
+    assert loip.loip_fixed_bytes(m, loip.config(**base, pack_stream=1, host_budget_bytes=10 ** 9)) == f0
+    if model == "llama3-70b" and mp == 512:  # the decode benchmark's ring: 6 x 47.2 MB
+        assert fp - f0 == 6 * 32768 * 1440 + 1280
+
+
 @pytest.mark.parametrize("model", ["tiny", "llama3-8b", "llama3-70b"])
 def test_block_refinement_and_eq7_match_planner_oracle(L, model):
     """loip_refine_blocks / loip_eq7_choice (C) against the planner oracle, on the
